@@ -1,0 +1,224 @@
+"""Seeded synthetic request traces and replica grids (inputs only).
+
+This module draws the inputs that both the CUDA path and the CPU oracle consume:
+token ids, prompt/output lengths, prefix-group structure and release times.  It
+holds none of the method's arithmetic (no hashing, no routing, no latency model):
+everything here is a random draw or a table of workload shapes.
+
+Workload shapes follow the paper's serving experiments, scaled up (§7.4: chat
+prompts drawn from a few shared templates, closed-loop concurrency C held by a
+semaphore; §7.7: the concurrency sweeps, the 4x4 (tau, omega) sweep, the
+adaptive-controller runs).  The paper's own prompt templates are not
+reproduced; prompts are uniform token ids with shared-prefix groups.
+
+Token layout: one int32 array, requests stored back to back (CSR `offsets`,
+int64, n+1 entries), the array padded with zeros to a multiple of 4 entries so
+that 16-byte vector loads never leave it.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field, replace
+from typing import Optional
+
+import numpy as np
+
+VOCAB = 32000
+BLOCK = 16
+
+POLICY_DYNAMO = 0    # router cost of Eq. (1): omega * prefill blocks + active blocks
+POLICY_LOADBAL = 1   # coordinated: the same cost with omega = 0, tau = 0
+
+
+@dataclass(frozen=True)
+class TraceSpec:
+    n_req: int
+    vocab: int = VOCAB
+    len_kind: str = "lognormal"       # "lognormal" | "uniform"
+    len_median: float = 1024.0
+    len_sigma: float = 0.75
+    len_min: int = 16
+    len_max: int = 8192
+    n_groups: int = 64
+    prefix_min: int = 512
+    prefix_max: int = 2048
+    zipf_s: Optional[float] = 1.1     # None: uniform group popularity
+    out_kind: str = "lognormal"       # "lognormal" | "uniform"
+    out_median: float = 256.0
+    out_sigma: float = 0.5
+    out_min: int = 1
+    out_max: int = 4096
+    rate: Optional[float] = None      # Poisson arrival rate (req/s); None = closed loop
+
+
+@dataclass
+class Trace:
+    tokens: np.ndarray    # int32 [round_up(offsets[-1], 4)]
+    offsets: np.ndarray   # int64 [n+1]
+    release: np.ndarray   # float64 [n], seconds
+    out_len: np.ndarray   # int32 [n]
+    group: np.ndarray     # int32 [n], prefix group (diagnostic)
+
+    @property
+    def n_req(self) -> int:
+        return int(self.offsets.shape[0] - 1)
+
+    @property
+    def n_tokens(self) -> int:
+        return int(self.offsets[-1])
+
+    def head(self, n: int) -> "Trace":
+        """The first n requests as a trace of their own (same token bytes)."""
+        n = min(n, self.n_req)
+        end = int(self.offsets[n])
+        pad = (-end) % 4
+        toks = self.tokens[:end]
+        if pad:
+            toks = np.concatenate([toks, np.zeros(pad, np.int32)])
+        return Trace(np.ascontiguousarray(toks), self.offsets[: n + 1].copy(),
+                     self.release[:n].copy(), self.out_len[:n].copy(), self.group[:n].copy())
+
+
+def _lengths(rng, kind, median, sigma, lo, hi, n):
+    if kind == "uniform":
+        return rng.integers(lo, hi + 1, size=n).astype(np.int64)
+    x = np.exp(rng.normal(np.log(median), sigma, size=n))
+    return np.clip(np.rint(x), lo, hi).astype(np.int64)
+
+
+def make_trace(spec: TraceSpec, seed: int) -> Trace:
+    """Draw one trace.  Same (spec, seed) -> same bytes on any machine with numpy."""
+    rng = np.random.default_rng([int(seed), 0x5EED7ACE])
+    n = int(spec.n_req)
+    G = int(spec.n_groups)
+    plen = rng.integers(spec.prefix_min, spec.prefix_max + 1, size=G).astype(np.int64)
+    prefixes = [rng.integers(0, spec.vocab, size=int(p), dtype=np.int32) for p in plen]
+    if spec.zipf_s is None:
+        group = rng.integers(0, G, size=n).astype(np.int32)
+    else:
+        w = 1.0 / np.power(np.arange(1, G + 1, dtype=np.float64), spec.zipf_s)
+        group = rng.choice(G, size=n, p=w / w.sum()).astype(np.int32)
+    L = _lengths(rng, spec.len_kind, spec.len_median, spec.len_sigma, spec.len_min, spec.len_max, n)
+    O = _lengths(rng, spec.out_kind, spec.out_median, spec.out_sigma, spec.out_min, spec.out_max, n)
+    if spec.rate is None:
+        release = np.zeros(n, np.float64)
+    else:
+        release = np.cumsum(rng.exponential(1.0 / spec.rate, size=n))
+    offsets = np.zeros(n + 1, np.int64)
+    np.cumsum(L, out=offsets[1:])
+    total = int(offsets[-1])
+    tokens = np.zeros(total + ((-total) % 4), np.int32)
+    tokens[:total] = rng.integers(0, spec.vocab, size=total, dtype=np.int32)
+    for i in range(n):
+        g = int(group[i])
+        k = int(min(plen[g], L[i]))
+        o = int(offsets[i])
+        tokens[o:o + k] = prefixes[g][:k]
+    return Trace(tokens, offsets, release.astype(np.float64), O.astype(np.int32), group)
+
+
+@dataclass
+class Replica:
+    trace: int            # index into Plan.trace_seeds
+    C: int                # closed-loop concurrency
+    policy: int           # POLICY_DYNAMO | POLICY_LOADBAL
+    controller: int       # 1: adaptive controller of §6 on
+    omega: float
+    tau: float
+    seed: int             # Philox key for temperature sampling
+    n_req: int            # requests of the trace this replica routes
+
+
+@dataclass
+class Plan:
+    name: str
+    W: int
+    K: int                                  # cache blocks per worker
+    spec: TraceSpec
+    trace_seeds: list
+    replicas: list = field(default_factory=list)
+    theta1: float = 0.3                     # s, 70B thresholds of §6.2
+    theta2: float = 2.0
+
+    def traces(self):
+        return [make_trace(self.spec, s) for s in self.trace_seeds]
+
+
+TINY_SPEC = TraceSpec(n_req=512, len_kind="uniform", len_min=64, len_max=512,
+                      n_groups=16, prefix_min=256, prefix_max=256, zipf_s=None,
+                      out_kind="uniform", out_min=16, out_max=256, rate=50.0)
+P2D_SPEC = TraceSpec(n_req=20000)
+P5D_SPEC = TraceSpec(n_req=50000)
+GRID_SPEC = TraceSpec(n_req=10000)
+LARGE_SPEC = TraceSpec(n_req=1_000_000, len_median=2048.0, len_max=32768, n_groups=1024,
+                       zipf_s=1.0)
+
+
+def plan(name: str, n_req: Optional[int] = None, replicas: Optional[list] = None) -> Plan:
+    """The replica grid of one workload.
+
+    n_req truncates every trace (tests run the oracle on a prefix); `replicas`
+    keeps only the listed replica indices (in that order).
+    """
+    if name == "tiny":
+        spec = TINY_SPEC
+        p = Plan(name, W=3, K=2048, spec=spec, trace_seeds=[0])
+        p.replicas = [Replica(0, 16, POLICY_DYNAMO, 0, 1.0, 0.0, 0, spec.n_req)]
+    elif name == "p2d":
+        # 70B 1P/2D-shaped: W=3, C sweep, selfish vs load-balanced on the same trace.
+        spec = P2D_SPEC
+        Cs = [16, 32, 64, 128, 256]
+        reps = []
+        for r in range(64):
+            pol = POLICY_DYNAMO if (r // 5) % 2 == 0 else POLICY_LOADBAL
+            om = 1.0 if pol == POLICY_DYNAMO else 0.0
+            reps.append(Replica(r // 10, Cs[r % 5], pol, 0, om, 0.0, r // 10, spec.n_req))
+        p = Plan(name, W=3, K=65536, spec=spec, trace_seeds=list(range(7)), replicas=reps)
+    elif name == "p5d":
+        # 70B 1P/5D-shaped: W=6, C x T cells, adaptive controller on.
+        spec = P5D_SPEC
+        Cs = [32, 64, 128, 256, 512]
+        Ts = [0.0, 0.5, 1.0]
+        reps = []
+        for r in range(256):
+            cell = r % 15
+            reps.append(Replica(r // 15, Cs[cell % 5], POLICY_DYNAMO, 1, 1.0, Ts[cell // 5],
+                                r // 15, spec.n_req))
+        p = Plan(name, W=6, K=65536, spec=spec, trace_seeds=list(range(18)), replicas=reps)
+    elif name == "grid":
+        # omega x C x T x seed; every cell also runs the coordinated policy on its trace.
+        spec = GRID_SPEC
+        Ws = [0.0, 0.25, 0.5, 1.0, 2.0, 4.0]
+        Cs = [16, 32, 64, 128, 256, 512]
+        Ts = [0.0, 0.5, 1.0]
+        reps = []
+        for r in range(4096):
+            cell = r % 108
+            rs = r // 108
+            ts = rs % 8
+            C = Cs[(cell // 6) % 6]
+            reps.append(Replica(ts, C, POLICY_DYNAMO, 0, Ws[cell % 6], Ts[cell // 36], rs, spec.n_req))
+            reps.append(Replica(ts, C, POLICY_LOADBAL, 0, 0.0, 0.0, rs, spec.n_req))
+        p = Plan(name, W=6, K=32768, spec=spec, trace_seeds=list(range(8)), replicas=reps)
+    elif name == "large":
+        spec = LARGE_SPEC
+        reps = []
+        for r in range(16):
+            pol = POLICY_DYNAMO if r < 8 else POLICY_LOADBAL
+            reps.append(Replica(r % 8, 4096, pol, 0, 1.0 if pol == POLICY_DYNAMO else 0.0, 0.0,
+                                r % 8, spec.n_req))
+        p = Plan(name, W=64, K=1 << 20, spec=spec, trace_seeds=list(range(8)), replicas=reps)
+    else:
+        raise ValueError(f"unknown workload {name!r}")
+    if n_req is not None:
+        p.spec = replace(p.spec, n_req=min(n_req, p.spec.n_req))
+        for r in p.replicas:
+            r.n_req = min(r.n_req, p.spec.n_req)
+    if replicas is not None:
+        keep = [p.replicas[i] for i in replicas]
+        used = sorted({r.trace for r in keep})
+        remap = {t: k for k, t in enumerate(used)}
+        p.trace_seeds = [p.trace_seeds[t] for t in used]
+        for r in keep:
+            r.trace = remap[r.trace]
+        p.replicas = keep
+    return p
