@@ -101,6 +101,7 @@ void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t ou
   out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
 }
 
+#define TICK_LIMIT (1ll << 24)   /* controller samples per replica */
 #define TAG_SIM 0x53494D31u    /* sampling stream of the simulation */
 #define TAG_ROUTE 0x52545231u  /* sampling stream of the live router */
 
@@ -406,6 +407,7 @@ typedef struct {
   ctl_t ctl;
   int64_t next_tick;
   int64_t* pending; int64_t npending;
+  int32_t err;
   double* window;
   double* tick_ewma; int32_t* tick_regime; int64_t max_ticks;
   orc_summary* sum;
@@ -536,6 +538,7 @@ static void controller_tick(sim_t* s) {
   s->sum->ticks_in_regime[s->ctl.regime]++;
   s->sum->ticks++;
   s->next_tick++;
+  if (s->sum->ticks >= TICK_LIMIT) s->err = ORC_ERR_CAPACITY;
 }
 
 static double next_tick_time(const sim_t* s) {
@@ -614,7 +617,11 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
     if (s.in_flight >= rep->C) {
       for (;;) {
         double tc = s.heap[0].t;
-        if (next_tick_time(&s) < tc) { controller_tick(&s); continue; }
+        if (next_tick_time(&s) < tc) {
+          controller_tick(&s);
+          if (s.err) { status = s.err; goto done; }
+          continue;
+        }
         cev e = heap_pop(s.heap, &s.nheap);
         complete(&s, e.q, e.t);
         if (e.t > T) T = e.t;
@@ -633,6 +640,7 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
       } else {
         if (tt > a) break;
         controller_tick(&s);
+        if (s.err) { status = s.err; goto done; }
       }
     }
 
@@ -1149,12 +1157,16 @@ int32_t orc_router_release(orc_router* r, int32_t inst, const int32_t* worker,
                            const int32_t* blocks, int64_t n) {
   if (!r || inst < 0 || inst >= r->ni) return ORC_ERR_INVALID;
   int64_t* A = r->A + (int64_t)inst * r->cfg.W;
+  int32_t status = ORC_OK;
   for (int64_t i = 0; i < n; i++) {
-    if (worker[i] < 0 || worker[i] >= r->cfg.W) return ORC_ERR_INVALID;
+    if (worker[i] < 0 || worker[i] >= r->cfg.W) {   /* skipped, reported */
+      status = ORC_ERR_INVALID;
+      continue;
+    }
     A[worker[i]] -= blocks[i];
     if (A[worker[i]] < 0) A[worker[i]] = 0;
   }
-  return ORC_OK;
+  return status;
 }
 
 int32_t orc_router_active(orc_router* r, int32_t inst, int64_t* active) {

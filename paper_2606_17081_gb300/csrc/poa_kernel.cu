@@ -1,0 +1,340 @@
+// PoA estimate of Eq. (12) (K4).
+//
+// k_poa_prep (one CTA per replica): window of every request = floor of its
+// completion time over the window length; frozen costs
+// c_ij = a n_ij + b + d/(C - n_ij)^2 - w_c o_ij of the §6.4 matrix; a stable
+// bucket sort of the requests by window (request order kept inside a window).
+//
+// k_poa_solve (one CTA per replica, one warp per window): OPT of the window =
+// minimum-cost assignment of its requests to W workers of capacity
+// max(C_j, ceil(n/W)) each (the replicated-column square matrix of §6.4).
+// Every request first takes its cheapest worker; that is optimal unless a
+// worker exceeds its capacity.  Otherwise the excess requests are taken out
+// (what stays is optimal for its own subset: every row sits at its minimum)
+// and put back one at a time along a shortest augmenting path (successive
+// shortest paths), found by Bellman-Ford on the W worker nodes with edge
+// weights min over the requests at j of (c_qk - c_qj).
+#include "rs_device.cuh"
+
+namespace rs {
+
+__device__ __forceinline__ double frozen_cost(const ModelConsts& mc, int nf, int m, int nbt) {
+  const double t1 = __dmul_rn(mc.lat_a, (double)nf);
+  const double t2 = __dadd_rn(t1, mc.lat_b);
+  const double den = (double)(mc.cap - nf);
+  const double f = __dadd_rn(t2, __ddiv_rn(mc.lat_d, __dmul_rn(den, den)));
+  const double o = nbt > 0 ? __ddiv_rn((double)m, (double)nbt) : 0.0;
+  return __dsub_rn(f, __dmul_rn(mc.w_c, o));
+}
+
+struct PoaPrepShared {
+  long long maxw;
+  int overflow;
+  int wn[NT_POA / 32];
+  int wk[NT_POA / 32][32];
+  int wc[NT_POA / 32][32];
+  long long scan_w[NT_POA / 32];
+  long long carry;
+};
+
+__global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restrict__ probs,
+                                                     PoaBuffers b, ModelConsts mc) {
+  __shared__ PoaPrepShared P;
+  const PoaProblem pr = probs[blockIdx.x];
+  const int W = mc.W;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    P.maxw = -1;
+    P.overflow = W > POA_WMAX;
+    P.carry = 0;
+  }
+  if (lane == 0) P.wn[warp] = 0;
+  __syncthreads();
+  if (P.overflow) {
+    if (threadIdx.x == 0) b.nwin[blockIdx.x] = -2;
+    return;
+  }
+  long long mx = -1;
+  for (int64_t q = threadIdx.x; q < pr.n; q += NT_POA) {
+    const int64_t r = pr.rec_base + q;
+    const int wk = b.rec.worker[r];
+    int key = -1;
+    if (wk >= 0) {
+      const long long w = (long long)floor(__ddiv_rn(b.rec.completion[r], mc.poa_window));
+      if (w >= pr.win_cap || w < 0) P.overflow = 1;
+      else key = (int)w;
+      mx = w > mx ? w : mx;
+      const int nbt = b.rec.nbt[r];
+      double* cr = b.cost + (pr.scratch_base + q) * W;
+      for (int j = 0; j < W; j++)
+        cr[j] = frozen_cost(mc, b.rec.n_frozen[r * W + j], b.rec.prefix[r * W + j], nbt);
+    }
+    b.wkey[pr.scratch_base + q] = key;
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const long long v = __shfl_xor_sync(FULL_MASK, mx, o);
+    mx = v > mx ? v : mx;
+  }
+  if (lane == 0 && mx >= 0) atomicMax(&P.maxw, mx);
+  __syncthreads();
+  if (P.overflow) {
+    if (threadIdx.x == 0) b.nwin[blockIdx.x] = -1;
+    return;
+  }
+  const int64_t nw = P.maxw + 1;
+  int64_t* cnt = b.wcnt + pr.win_base;
+  int64_t* wst = b.wstart + pr.win_base + blockIdx.x;   // nw + 1 entries
+  int64_t* fill = b.wfill + pr.win_base;
+  for (int64_t w = threadIdx.x; w < nw; w += NT_POA) cnt[w] = 0;
+  __syncthreads();
+  for (int64_t q = threadIdx.x; q < pr.n; q += NT_POA) {
+    const int key = b.wkey[pr.scratch_base + q];
+    if (key >= 0) atomicAdd(reinterpret_cast<unsigned long long*>(cnt + key), 1ull);
+  }
+  __syncthreads();
+  // exclusive scan of the window counts
+  for (int64_t w0 = 0; w0 < nw; w0 += NT_POA) {
+    const int64_t w = w0 + threadIdx.x;
+    long long v = w < nw ? (long long)cnt[w] : 0;
+    long long x = v;
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(FULL_MASK, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) P.scan_w[warp] = x;
+    __syncthreads();
+    long long off = P.carry;
+    for (int i = 0; i < warp; i++) off += P.scan_w[i];
+    if (w < nw) {
+      wst[w] = off + x - v;
+      fill[w] = off + x - v;
+    }
+    __syncthreads();
+    if (threadIdx.x == NT_POA - 1) {
+      long long tot = 0;
+      for (int i = 0; i < NT_POA / 32; i++) tot += P.scan_w[i];
+      P.carry += tot;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) wst[nw] = P.carry;
+  __syncthreads();
+  // stable scatter: rank inside the chunk = earlier warps' equal keys + earlier lanes
+  for (int64_t q0 = 0; q0 < pr.n; q0 += NT_POA) {
+    const int64_t q = q0 + threadIdx.x;
+    const int key = q < pr.n ? b.wkey[pr.scratch_base + q] : -1;
+    const unsigned peers = __match_any_sync(FULL_MASK, key);
+    const int intra = __popc(peers & ((1u << lane) - 1u));
+    const bool leader = (__ffs(peers) - 1) == lane;
+    if (leader) {
+      const int idx = atomicAdd(&P.wn[warp], 1);
+      P.wk[warp][idx] = key;
+      P.wc[warp][idx] = __popc(peers);
+    }
+    __syncthreads();
+    if (key >= 0) {
+      int cross = 0;
+      for (int v = 0; v < warp; v++)
+        for (int e = 0; e < P.wn[v]; e++)
+          if (P.wk[v][e] == key) cross += P.wc[v][e];
+      b.order[pr.scratch_base + fill[key] + cross + intra] = (int32_t)q;
+    }
+    __syncthreads();
+    if (leader && key >= 0)
+      atomicAdd(reinterpret_cast<unsigned long long*>(fill + key), (unsigned long long)__popc(peers));
+    if (lane == 0) P.wn[warp] = 0;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) b.nwin[blockIdx.x] = nw;
+}
+
+struct PoaWarpShared {
+  int counts[POA_WMAX];
+  double wmin[POA_WMAX][POA_WMAX];
+  int wrow[POA_WMAX][POA_WMAX];
+  double num, opt;
+  int err;
+};
+
+struct PoaSolveShared {
+  PoaWarpShared w[NT_POA / 32];
+};
+
+__device__ __forceinline__ double warp_sum(double v) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL_MASK, v, o);
+  return v;
+}
+
+__global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restrict__ probs,
+                                                      PoaBuffers b, ModelConsts mc) {
+  __shared__ PoaSolveShared P;
+  const PoaProblem pr = probs[blockIdx.x];
+  const int64_t nw = b.nwin[blockIdx.x];
+  if (nw < 0) {
+    if (threadIdx.x == 0) {
+      b.total[blockIdx.x] = __longlong_as_double(0x7FF8000000000000ll);
+      if (b.res) {
+        b.res[blockIdx.x].poa_total = __longlong_as_double(0x7FF8000000000000ll);
+        b.res[blockIdx.x].n_windows = nw;
+      }
+    }
+    return;
+  }
+  const int W = mc.W;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  PoaWarpShared& S = P.w[warp];
+  const int64_t* wst = b.wstart + pr.win_base + blockIdx.x;
+  for (int64_t w = warp; w < nw; w += NT_POA / 32) {
+    const int64_t s0 = wst[w];
+    const int64_t m = wst[w + 1] - s0;
+    const int64_t base = pr.scratch_base + s0;   // window rows in order[], asg[]
+    if (m == 0) {
+      if (lane == 0) {
+        b.wnum[pr.win_base + w] = 0.0;
+        b.wopt[pr.win_base + w] = 0.0;
+        b.wcnt[pr.win_base + w] = 0;
+      }
+      continue;
+    }
+    int64_t capw = (m + W - 1) / W;
+    if (capw < mc.cap) capw = mc.cap;
+    if (lane < W) S.counts[lane] = 0;
+    if (lane == 0) S.err = 0;
+    __syncwarp();
+    double num = 0.0;
+    for (int64_t r = lane; r < m; r += 32) {
+      const int q = b.order[base + r];
+      const double* cr = b.cost + (pr.scratch_base + q) * W;
+      int best = 0;
+      double bc = cr[0];
+      for (int j = 1; j < W; j++)
+        if (cr[j] < bc) { bc = cr[j]; best = j; }
+      b.asg[base + r] = best;
+      atomicAdd(&S.counts[best], 1);
+      num += b.rec.ttft[pr.rec_base + q];
+    }
+    num = warp_sum(num);
+    __syncwarp();
+    int over = 0;
+    for (int j = 0; j < W; j++) over |= S.counts[j] > capw;
+    if (over) {
+      // take out the excess, latest rows first
+      if (lane == 0) {
+        int64_t nrem = 0;
+        for (int64_t r = m - 1; r >= 0; r--) {
+          const int j = b.asg[base + r];
+          if (S.counts[j] > capw) {
+            S.counts[j]--;
+            b.asg[base + r] = -1;
+            b.wkey[base + nrem++] = (int32_t)r;   // wkey reused as the removal list
+          }
+        }
+        S.num = (double)nrem;
+      }
+      __syncwarp();
+      const int64_t nrem = (int64_t)S.num;
+      for (int64_t e = 0; e < nrem; e++) {
+        const int64_t r0 = b.wkey[base + e];
+        const double* c0 = b.cost + (pr.scratch_base + b.order[base + r0]) * W;
+        // edge weights j -> k: cheapest move of a request now at j to k
+        for (int j = 0; j < W; j++) {
+          double lm[POA_WMAX];
+          int lr[POA_WMAX];
+          for (int k = 0; k < W; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
+          for (int64_t r = lane; r < m; r += 32) {
+            if (b.asg[base + r] != j) continue;
+            const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
+            const double cj = cr[j];
+            for (int k = 0; k < W; k++) {
+              const double v = __dsub_rn(cr[k], cj);
+              if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
+            }
+          }
+          for (int k = 0; k < W; k++) {
+            double v = lm[k];
+            int rr = lr[k];
+            for (int o = 16; o > 0; o >>= 1) {
+              const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
+              const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
+              if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
+            }
+            if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) {
+          double dist[POA_WMAX];
+          int pred[POA_WMAX];
+          for (int k = 0; k < W; k++) { dist[k] = c0[k]; pred[k] = -1; }
+          for (int it = 0; it < W; it++) {
+            bool ch = false;
+            for (int j = 0; j < W; j++)
+              for (int k = 0; k < W; k++) {
+                if (k == j || S.wrow[j][k] < 0) continue;
+                const double nd = __dadd_rn(dist[j], S.wmin[j][k]);
+                if (nd < dist[k]) { dist[k] = nd; pred[k] = j; ch = true; }
+              }
+            if (!ch) break;
+          }
+          int tgt = -1;
+          for (int k = 0; k < W; k++)
+            if (S.counts[k] < capw && (tgt < 0 || dist[k] < dist[tgt])) tgt = k;
+          if (tgt < 0) {
+            S.err = 1;
+          } else {
+            int k = tgt, steps = 0;
+            while (pred[k] >= 0 && steps <= W) {
+              const int j = pred[k];
+              b.asg[base + S.wrow[j][k]] = k;
+              k = j;
+              steps++;
+            }
+            if (steps > W) S.err = 1;
+            b.asg[base + r0] = k;
+            S.counts[tgt]++;
+          }
+        }
+        __syncwarp();
+      }
+    }
+    double opt = 0.0;
+    for (int64_t r = lane; r < m; r += 32) {
+      const int q = b.order[base + r];
+      const int a = b.asg[base + r];
+      opt += a >= 0 ? b.cost[(pr.scratch_base + q) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
+    }
+    opt = warp_sum(opt);
+    if (lane == 0) {
+      b.wnum[pr.win_base + w] = num;
+      b.wopt[pr.win_base + w] = S.err ? __longlong_as_double(0x7FF8000000000000ll) : opt;
+      b.wcnt[pr.win_base + w] = m;
+    }
+    __syncwarp();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double tn = 0.0, to = 0.0;
+    for (int64_t w = 0; w < nw; w++) {
+      tn += b.wnum[pr.win_base + w];
+      to += b.wopt[pr.win_base + w];
+    }
+    const double tot = to > 0.0 ? tn / to : 0.0;
+    b.total[blockIdx.x] = tot;
+    if (b.res) {
+      b.res[blockIdx.x].poa_total = tot;
+      b.res[blockIdx.x].n_windows = nw;
+    }
+  }
+}
+
+cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
+                       const ModelConsts& mc, cudaStream_t st) {
+  if (nprob <= 0) return cudaSuccess;
+  k_poa_prep<<<nprob, NT_POA, 0, st>>>(d_prob, b, mc);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_poa_solve<<<nprob, NT_POA, 0, st>>>(d_prob, b, mc);
+  return cudaGetLastError();
+}
+
+}  // namespace rs

@@ -1,0 +1,516 @@
+// Device building blocks of the routing library (sm_103a).
+//
+// Block hashing, Philox, the softmax exp, worker selection (Eq. (1), Eq. (2)),
+// and the per-worker KV block cache: an open-addressing table of 64-bit block
+// hashes (buckets of four 8-byte keys = one 32-byte sector) whose slots carry
+// an LRU stamp, plus a ring "log" of slots in stamp order.  Exact LRU order is
+// stamp order: touching or inserting a block gives it the next stamp and
+// appends its slot to the log; a log entry is live iff its slot still holds
+// that stamp, so the least-recent entries are the first live entries of the
+// log.  A request's whole block list is applied in one CTA-wide step.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "rs_internal.h"
+
+namespace rs {
+
+constexpr uint64_t KEY_EMPTY = 0ull;
+constexpr uint64_t KEY_TOMB = 1ull;
+constexpr uint32_t STAMP_NONE = 0xFFFFFFFFu;
+constexpr uint32_t SLOT_NONE = 0xFFFFFFFFu;
+constexpr uint32_t STAMP_LIMIT = 0x7FFF0000u;   // compaction renumbers before this
+constexpr int64_t TICK_LIMIT = 1ll << 24;       // controller samples per replica
+constexpr unsigned FULL_MASK = 0xFFFFFFFFu;
+
+// ---------------------------------------------------------------- hashing
+
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// content hash g of one 16-token block given as 16 words
+__device__ __forceinline__ uint64_t block_content16(const uint32_t (&w)[16]) {
+  uint64_t x = 0x9E3779B97F4A7C15ull ^ 16ull;
+#pragma unroll
+  for (int q = 0; q < 8; q++) x = mix64(x ^ ((uint64_t)w[2 * q] | ((uint64_t)w[2 * q + 1] << 32)));
+  return x;
+}
+
+__device__ __forceinline__ uint64_t chain_step(uint64_t prev, uint64_t gk) {
+  // gk already carries the block index: g_k ^ k
+  uint64_t h = mix64(prev ^ gk);
+  return h < 2 ? h + 2 : h;
+}
+
+// ---------------------------------------------------------------- Philox4x32-10
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; r++) {
+    if (r) {
+      k.x += 0x9E3779B9u;
+      k.y += 0xBB67AE85u;
+    }
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+  }
+  return c;
+}
+
+constexpr uint32_t TAG_SIM = 0x53494D31u;
+constexpr uint32_t TAG_ROUTE = 0x52545231u;
+
+__device__ __forceinline__ uint32_t draw_u24(uint64_t seed, uint64_t ordinal, uint32_t stream,
+                                             uint32_t tag) {
+  uint4 c = make_uint4((uint32_t)ordinal, (uint32_t)(ordinal >> 32), stream, tag);
+  uint2 k = make_uint2((uint32_t)seed, (uint32_t)(seed >> 32));
+  return philox4x32_10(c, k).x >> 8;
+}
+
+// ---------------------------------------------------------------- exp of Eq. (2)
+
+// Cody-Waite reduction by ln2 (split in an 8-trailing-zero high part and a
+// low part) and the degree-7 Taylor polynomial of exp(r) in Horner form with
+// fused multiply-adds; 2^k through the exponent field.  x < -87 gives 0.
+__device__ __forceinline__ float exp_sm(float x) {
+  if (!(x >= -87.0f)) return 0.0f;
+  if (x > 88.0f) return __int_as_float(0x7F800000);
+  const float t = __fmul_rn(x, 0x1.715476p+0f);
+  const float kf = rintf(t);
+  float r = __fmaf_rn(-kf, 0x1.62e4p-1f, x);
+  r = __fmaf_rn(-kf, 0x1.7f7d1cp-20f, r);
+  float p = 0x1.a01a02p-13f;
+  p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);
+  p = __fmaf_rn(p, r, 0x1.111112p-7f);
+  p = __fmaf_rn(p, r, 0x1.555556p-5f);
+  p = __fmaf_rn(p, r, 0x1.555556p-3f);
+  p = __fmaf_rn(p, r, 0.5f);
+  p = __fmaf_rn(p, r, 1.0f);
+  p = __fmaf_rn(p, r, 1.0f);
+  const int k = (int)kf;
+  return __fmul_rn(p, __int_as_float((k + 127) << 23));
+}
+
+// ---------------------------------------------------------------- selection
+
+// Eq. (1) in fp32, rounded per operation: omega * b^prefill + b^active.
+__device__ __forceinline__ float router_cost(float omega, int64_t bprefill, int64_t active) {
+  return __fadd_rn(__fmul_rn(omega, (float)bprefill), (float)active);
+}
+
+// Lowest-index argmin over c[0..W) (one thread).
+__device__ __forceinline__ int argmin_lowest(const float* c, int W) {
+  int b = 0;
+  for (int j = 1; j < W; j++)
+    if (c[j] < c[b]) b = j;
+  return b;
+}
+
+// Eq. (2): tau == 0 -> argmin; tau > 0 -> the first j whose cumulative weight
+// (sequential fp32 sum in worker order) exceeds u * S.  One thread.
+// *near_bd = the scaled draw lies within 1e-6 S of a cumulative boundary.
+__device__ __forceinline__ int select_worker(const float* c, int W, float tau, uint32_t u24,
+                                             int* near_bd) {
+  const int b = argmin_lowest(c, W);
+  *near_bd = 0;
+  if (tau == 0.0f) return b;
+  const float cmin = c[b];
+  float S = 0.0f;
+  for (int j = 0; j < W; j++) S = __fadd_rn(S, exp_sm(-__fdiv_rn(__fsub_rn(c[j], cmin), tau)));
+  const float target = __fmul_rn(__fmul_rn((float)u24, 0x1p-24f), S);
+  float cum = 0.0f;
+  int pick = -1, last = b;
+  for (int j = 0; j < W; j++) {
+    const float e = exp_sm(-__fdiv_rn(__fsub_rn(c[j], cmin), tau));
+    cum = __fadd_rn(cum, e);
+    if (e > 0.0f) last = j;
+    if (fabs((double)target - (double)cum) <= 1e-6 * (double)S) *near_bd = 1;
+    if (pick < 0 && target < cum) pick = j;
+  }
+  return pick >= 0 ? pick : last;
+}
+
+// ---------------------------------------------------------------- CTA helpers
+
+// Exclusive rank of `flag` among the CTA's threads (thread order) and the
+// total; two barriers.  warp_tot: shared int[NT/32].
+template <int NT>
+__device__ __forceinline__ int cta_rank(bool flag, int* warp_tot, int* total) {
+  const unsigned m = __ballot_sync(FULL_MASK, flag);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (lane == 0) warp_tot[w] = __popc(m);
+  __syncthreads();
+  int off = 0, tot = 0;
+#pragma unroll
+  for (int i = 0; i < NT / 32; i++) {
+    const int v = warp_tot[i];
+    off += i < w ? v : 0;
+    tot += v;
+  }
+  __syncthreads();
+  *total = tot;
+  return off + __popc(m & ((1u << lane) - 1u));
+}
+
+// ---------------------------------------------------------------- cache table
+
+struct TableView {
+  uint64_t* keys;     // [4 * nbuckets]
+  uint32_t* stamp;    // [4 * nbuckets]
+  uint32_t* log;      // [rmask + 1]
+  uint32_t bmask;     // nbuckets - 1
+  uint32_t rmask;     // log ring size - 1
+};
+
+__device__ __forceinline__ uint32_t home_bucket(uint64_t h, uint32_t bmask) {
+  return (uint32_t)(h ^ (h >> 32)) & bmask;
+}
+
+__device__ __forceinline__ ulonglong2 ld_keys2(const uint64_t* p) {
+  return __ldcg(reinterpret_cast<const ulonglong2*>(p));
+}
+
+// Slot holding h, or SLOT_NONE.  Buckets are scanned from h's home bucket;
+// an EMPTY key ends the search (keys are never moved, and slots only go from
+// EMPTY to a key, key to TOMB, TOMB to a key).  *err set if the scan wraps.
+__device__ __forceinline__ uint32_t table_find(const TableView& t, uint64_t h, int* err) {
+  uint32_t b = home_bucket(h, t.bmask);
+  for (uint32_t it = 0; it <= t.bmask; it++) {
+    const ulonglong2 x = ld_keys2(t.keys + 4 * (size_t)b);
+    const ulonglong2 y = ld_keys2(t.keys + 4 * (size_t)b + 2);
+    if (x.x == h) return 4 * b;
+    if (x.y == h) return 4 * b + 1;
+    if (y.x == h) return 4 * b + 2;
+    if (y.y == h) return 4 * b + 3;
+    if (x.x == KEY_EMPTY || x.y == KEY_EMPTY || y.x == KEY_EMPTY || y.y == KEY_EMPTY)
+      return SLOT_NONE;
+    b = (b + 1) & t.bmask;
+  }
+  *err = 1;
+  return SLOT_NONE;
+}
+
+// Claims the first EMPTY or TOMB slot of h's probe sequence (h known absent;
+// other threads of the CTA may insert concurrently).  *was_tomb reports a
+// reclaimed tombstone.
+__device__ __forceinline__ uint32_t table_insert(const TableView& t, uint64_t h, int* was_tomb,
+                                                 int* err) {
+  uint32_t b = home_bucket(h, t.bmask);
+  for (uint32_t it = 0; it <= t.bmask; it++) {
+#pragma unroll
+    for (int q = 0; q < 4; q++) {
+      unsigned long long* p = reinterpret_cast<unsigned long long*>(t.keys + 4 * (size_t)b + q);
+      unsigned long long cur = __ldcg(p);
+      while (cur == KEY_EMPTY || cur == KEY_TOMB) {
+        const unsigned long long prev = atomicCAS(p, cur, (unsigned long long)h);
+        if (prev == cur) {
+          *was_tomb = cur == KEY_TOMB;
+          return 4 * b + q;
+        }
+        cur = prev;
+      }
+    }
+    b = (b + 1) & t.bmask;
+  }
+  *err = 1;
+  return SLOT_NONE;
+}
+
+// Scratch of one CTA-wide cache update (shared memory).
+struct UpdateScratch {
+  uint32_t* slot;     // [nbmax] slot per request block
+  uint32_t* pst;      // [nbmax] stamp of present blocks
+  uint8_t* kind;      // [nbmax] 1 = insert, 0 = touch
+  uint8_t* evk;       // [nbmax] present block evicted before its turn
+  uint32_t* vslot;    // [2*nbmax] first live log entries: slot
+  uint32_t* vt;       // [2*nbmax]                          stamp
+  int32_t* owner;     // [2*nbmax] request block owning that entry, or -1
+  uint8_t* touched;   // [2*nbmax]
+  int32_t* victim;    // [2*nbmax] indices into vslot/vt of the evicted entries
+  uint64_t* dupset;   // [2*nbmax_pow2] duplicate detector
+  uint32_t dupmask;
+};
+
+struct UpdateShared {   // small shared scalars of the update
+  int n_absent, n_ins, reclaimed, n_victims, slow, err, dup;
+  uint32_t pmin, gathered;
+};
+
+// Rebuilds the table and log of one worker from its live entries in LRU
+// order (stamps renumbered 0..size-1).  tmp: global scratch of >= size keys.
+template <int NT>
+__device__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, uint64_t* tmp,
+                              int* warp_tot, UpdateShared* us) {
+  const uint32_t head = meta->head, T = meta->T;
+  uint32_t base = 0;
+  for (uint32_t p0 = head; p0 < T; p0 += NT) {
+    const uint32_t p = p0 + threadIdx.x;
+    bool live = false;
+    uint32_t x = 0;
+    if (p < T) {
+      x = t.log[p & t.rmask];
+      live = __ldcg(t.stamp + x) == p;
+    }
+    int tot;
+    const int r = cta_rank<NT>(live, warp_tot, &tot);
+    if (live && base + r < K) tmp[base + r] = __ldcg(t.keys + x);
+    base += tot;
+  }
+  __syncthreads();
+  if (base > K) {   // more live log entries than the cache holds: inconsistent state
+    if (threadIdx.x == 0) us->err = RS_ERR_TIMEOUT;
+    __syncthreads();
+    return;
+  }
+  const size_t nslots = 4 * ((size_t)t.bmask + 1);
+  for (size_t s = threadIdx.x; s < nslots; s += NT) {
+    t.keys[s] = KEY_EMPTY;
+    t.stamp[s] = STAMP_NONE;
+  }
+  __syncthreads();
+  for (uint32_t r = threadIdx.x; r < base; r += NT) {
+    int wt = 0, e = 0;
+    const uint32_t sl = table_insert(t, __ldcg(tmp + r), &wt, &e);
+    if (e) us->err = RS_ERR_TIMEOUT;
+    else {
+      t.stamp[sl] = r;
+      t.log[r & t.rmask] = sl;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (base != meta->size) us->err = RS_ERR_TIMEOUT;
+    meta->head = 0;
+    meta->T = base;
+    meta->tombs = 0;
+  }
+  __syncthreads();
+}
+
+// Resets the shared scalars of one cache update.
+__device__ __forceinline__ void update_reset(UpdateShared* us) {
+  us->n_absent = 0;
+  us->n_ins = 0;
+  us->reclaimed = 0;
+  us->n_victims = 0;
+  us->slow = 0;
+  us->dup = 0;
+  us->pmin = STAMP_NONE;
+  us->gathered = 0;
+}
+
+// Looks up every block of a request in one worker's cache (CTA-wide);
+// fills slot[] and pst[]; counts absent blocks; detects duplicate hashes
+// within the request (a shared-memory open-addressing set; each thread clears
+// the slot it claimed).  us must be reset before the call.
+template <int NT>
+__device__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int nb,
+                                 UpdateScratch& sc, UpdateShared* us,
+                                 unsigned long long* probes) {
+  int nabs = 0, err = 0, dup = 0;
+  uint32_t pmin = STAMP_NONE;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const uint64_t h = hbuf[k];
+    const uint32_t sl = table_find(t, h, &err);
+    sc.slot[k] = sl;
+    uint32_t st = STAMP_NONE;
+    if (sl != SLOT_NONE) {
+      st = __ldcg(t.stamp + sl);
+      pmin = min(pmin, st);
+    } else {
+      nabs++;
+    }
+    sc.pst[k] = st;
+    sc.evk[k] = 0;
+    uint32_t d = (uint32_t)(h ^ (h >> 29)) & sc.dupmask;
+    int32_t claimed = -1;
+    for (uint32_t it = 0; it <= sc.dupmask; it++) {
+      const unsigned long long prev = atomicCAS(
+          reinterpret_cast<unsigned long long*>(sc.dupset + d), 0ull, (unsigned long long)h);
+      if (prev == 0ull) { claimed = (int32_t)d; break; }
+      if (prev == h) { dup = 1; break; }
+      d = (d + 1) & sc.dupmask;
+    }
+    sc.owner[k] = claimed;
+  }
+  if (nabs) atomicAdd(&us->n_absent, nabs);
+  if (pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  if (err) us->err = RS_ERR_TIMEOUT;
+  if (dup) us->dup = 1;
+  if (threadIdx.x == 0) atomicAdd(probes, (unsigned long long)nb);
+  __syncthreads();
+  for (int k = threadIdx.x; k < nb; k += NT)
+    if (sc.owner[k] >= 0) sc.dupset[sc.owner[k]] = 0ull;
+}
+
+// Gathers live log entries starting at meta->head until `want` are held
+// (or the log ends).  Continues from us->gathered entries already held.
+template <int NT>
+__device__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t* pos,
+                            uint32_t want, UpdateScratch& sc, UpdateShared* us, int* warp_tot) {
+  const uint32_t T = meta->T;
+  uint32_t have = us->gathered;
+  uint32_t p0 = *pos;
+  while (have < want && p0 < T) {
+    const uint32_t p = p0 + threadIdx.x;
+    bool live = false;
+    uint32_t x = 0;
+    if (p < T) {
+      x = t.log[p & t.rmask];
+      live = __ldcg(t.stamp + x) == p;
+    }
+    int tot;
+    const int r = cta_rank<NT>(live, warp_tot, &tot);
+    if (live && have + r < want) {
+      sc.vslot[have + r] = x;
+      sc.vt[have + r] = p;
+    }
+    have = min(want, have + (uint32_t)tot);
+    p0 += NT;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    us->gathered = have;
+    *pos = p0;
+  }
+  __syncthreads();
+}
+
+// Applies one request's block list to the chosen worker's cache: exact LRU
+// semantics of touching blocks 0..nb-1 in order (hits -> most recent, misses
+// inserted, the least-recent entry evicted whenever the cache is full).
+// Returns through us: n_victims, n_ins; updates meta.  CTA-wide.
+template <int NT>
+__device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, const uint64_t* hbuf,
+                            int nb, UpdateScratch& sc, UpdateShared* us, int* warp_tot,
+                            uint32_t* scan_pos) {
+  const uint32_t size = meta->size;
+  const int nabs = us->n_absent;
+  const uint32_t free_slots = K - size;
+  const uint32_t E0 = (uint32_t)nabs > free_slots ? (uint32_t)nabs - free_slots : 0u;
+  if (threadIdx.x == 0) {
+    us->gathered = 0;
+    *scan_pos = meta->head;
+  }
+  __syncthreads();
+  if (E0 > 0) gather_live<NT>(t, meta, scan_pos, E0, sc, us, warp_tot);
+  if (E0 > 0 && us->gathered < E0) {   // fewer live entries than the size says
+    if (threadIdx.x == 0) us->err = RS_ERR_TIMEOUT;
+    __syncthreads();
+    return;
+  }
+  const bool fast = E0 == 0 || us->pmin > sc.vt[E0 - 1];
+  if (fast) {
+    for (int k = threadIdx.x; k < nb; k += NT) sc.kind[k] = sc.slot[k] == SLOT_NONE;
+    for (uint32_t v = threadIdx.x; v < E0; v += NT) sc.victim[v] = (int32_t)v;
+    if (threadIdx.x == 0) us->n_victims = (int)E0;
+    __syncthreads();
+  } else {
+    // exact sequential emulation over the first live entries (gathered again
+    // from the head: the first pass dropped live entries past the E0-th)
+    const uint32_t want = min(size, 2u * (uint32_t)nb);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      us->gathered = 0;
+      *scan_pos = meta->head;
+    }
+    __syncthreads();
+    gather_live<NT>(t, meta, scan_pos, want, sc, us, warp_tot);
+    const uint32_t G = us->gathered;
+    for (uint32_t p = threadIdx.x; p < G; p += NT) {
+      sc.owner[p] = -1;
+      sc.touched[p] = 0;
+    }
+    __syncthreads();
+    const uint32_t last = G ? sc.vt[G - 1] : 0u;
+    for (int k = threadIdx.x; k < nb; k += NT) {
+      const uint32_t st = sc.pst[k];
+      if (st != STAMP_NONE && G && st <= last) {
+        uint32_t lo = 0, hi = G;   // vt is increasing: lower bound of st
+        while (lo < hi) {
+          const uint32_t mid = (lo + hi) >> 1;
+          if (sc.vt[mid] < st) lo = mid + 1; else hi = mid;
+        }
+        sc.owner[lo] = k;
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      uint32_t ptr = 0, sz = size;
+      int E = 0;
+      // position of each present block inside the gathered list (or none)
+      for (int k = 0; k < nb; k++) {
+        const bool present = sc.slot[k] != SLOT_NONE && !sc.evk[k];
+        if (present) {
+          sc.kind[k] = 0;
+          const uint32_t st = sc.pst[k];
+          if (G && st <= last) {
+            uint32_t lo = 0, hi = G;
+            while (lo < hi) {
+              const uint32_t mid = (lo + hi) >> 1;
+              if (sc.vt[mid] < st) lo = mid + 1; else hi = mid;
+            }
+            sc.touched[lo] = 1;
+          }
+        } else {
+          sc.kind[k] = 1;
+          if (sz == K) {
+            while (ptr < G && sc.touched[ptr]) ptr++;
+            if (ptr >= G) { us->err = RS_ERR_TIMEOUT; break; }
+            sc.victim[E++] = (int32_t)ptr;
+            if (sc.owner[ptr] >= 0) sc.evk[sc.owner[ptr]] = 1;
+            ptr++;
+          } else {
+            sz++;
+          }
+        }
+      }
+      us->n_victims = E;
+      us->slow = 1;
+    }
+    __syncthreads();
+  }
+  const int E = us->n_victims;
+  // evictions first (tombstones), then inserts, then stamps and log
+  for (int v = threadIdx.x; v < E; v += NT) {
+    const uint32_t x = sc.vslot[sc.victim[v]];
+    t.keys[x] = KEY_TOMB;
+    t.stamp[x] = STAMP_NONE;
+  }
+  __syncthreads();
+  const uint32_t T = meta->T;
+  int nins = 0, recl = 0, err = 0;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    uint32_t sl = sc.slot[k];
+    if (sc.kind[k]) {
+      int wt = 0;
+      sl = table_insert(t, hbuf[k], &wt, &err);
+      nins++;
+      recl += wt;
+      sc.slot[k] = sl;
+    }
+    if (sl != SLOT_NONE) {
+      t.stamp[sl] = T + (uint32_t)k;
+      t.log[(T + (uint32_t)k) & t.rmask] = sl;
+    }
+  }
+  if (nins) atomicAdd(&us->n_ins, nins);
+  if (recl) atomicAdd(&us->reclaimed, recl);
+  if (err) us->err = RS_ERR_TIMEOUT;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    meta->tombs = meta->tombs + (uint32_t)E - (uint32_t)us->reclaimed;
+    meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
+    if (E > 0) meta->head = sc.vt[sc.victim[E - 1]] + 1;
+    meta->T = T + (uint32_t)nb;
+  }
+  __syncthreads();
+}
+
+}  // namespace rs

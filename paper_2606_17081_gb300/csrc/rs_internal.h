@@ -1,0 +1,135 @@
+// Internal declarations of the routing library (host + device, not public).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "routesim.h"
+
+namespace rs {
+
+constexpr int NT_SIM = 256;      // threads of a simulation / router CTA
+constexpr int NT_POA = 256;      // threads of a PoA CTA (8 warps, one window each)
+constexpr int POA_WMAX = 16;     // workers supported by the PoA solver
+constexpr int WMAX = 64;         // workers supported by the simulation
+
+// Per-worker cache bookkeeping (shared memory while a kernel runs, global
+// memory between calls).
+struct CacheMeta {
+  uint32_t size;    // live entries
+  uint32_t T;       // next stamp
+  uint32_t head;    // log position at or before the least-recent live entry
+  uint32_t tombs;   // tombstoned slots
+};
+
+// Geometry of one worker's table: 4 * nbuckets slots (>= 2 K) and a log ring
+// of R entries (>= 4 K).
+struct TableGeom {
+  uint32_t K;
+  uint32_t bmask;      // nbuckets - 1
+  uint32_t rmask;      // R - 1
+  size_t slots;        // 4 * nbuckets
+  size_t R;
+};
+
+TableGeom table_geom(int64_t K);
+
+// One simulated replica as the kernel sees it.
+struct SimDesc {
+  const int64_t* offsets;
+  const double* release;
+  const int32_t* out_len;
+  const uint64_t* hashes;   // block hashes of the replica's trace
+  int64_t n_req;
+  int64_t rec_base;         // first record row
+  int32_t C, policy, controller, reserved;
+  float omega, tau;
+  uint64_t seed;
+};
+
+struct ModelConsts {
+  double lat_a, lat_b, lat_d, w_c, itl, dt, alpha, theta1, theta2, eps_frac, poa_window;
+  int32_t cap, hyst_k, W, write_cost;
+  float regime_tau[3], regime_omega[3];
+};
+
+struct SimBuffers {
+  uint64_t* keys;           // [nsim][W][slots]
+  uint32_t* stamp;          // [nsim][W][slots]
+  uint32_t* log;            // [nsim][W][R]
+  uint64_t* tmp;            // [nsim][K] rebuild scratch
+  double* pend;             // [nsim][4][pend_cap]: 2 buffers x (first token, TTFT)
+  int64_t pend_cap;
+  CacheMeta* meta_out;      // [nsim][W]
+  rs_replica_result* res;   // [nsim]
+  rs_records rec;           // every field non-NULL except possibly cost
+};
+
+struct SimLaunch {
+  int nsim;
+  int nbmax;                // max full blocks of any routed prompt
+  int cmax;                 // max concurrency over replicas
+  TableGeom g;
+  ModelConsts mc;
+};
+
+size_t sim_smem_bytes(int W, int nbmax, int cmax);
+cudaError_t launch_block_hash(const int32_t* tokens, const int64_t* offsets, int64_t n_req,
+                              uint64_t seed, uint64_t* out, int64_t* nbmax_out,
+                              cudaStream_t st);
+cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
+                       cudaStream_t st);
+
+// PoA of Eq. (12): one "problem" per replica.
+struct PoaProblem {
+  int64_t rec_base;         // first record row
+  int64_t n;                // rows
+  int64_t scratch_base;     // first row of this problem in the row-indexed scratch
+  int64_t win_base;         // first window slot in the window-indexed scratch
+  int64_t win_cap;          // window slots available
+};
+
+struct PoaBuffers {
+  rs_records rec;
+  double* cost;             // [rows][W]
+  int32_t* order;           // [rows] row (relative) sorted by window, stable
+  int32_t* asg;             // [rows]
+  int32_t* wkey;            // [rows] window of each row (-1 skipped)
+  int64_t* wstart;          // [win slots + problems]
+  int64_t* wfill;           // [win slots]
+  double* wnum;             // [win slots]
+  double* wopt;             // [win slots]
+  int64_t* wcnt;            // [win slots]
+  double* total;            // [problems]: PoA total
+  int64_t* nwin;            // [problems]: windows spanned (or -1 on overflow)
+  rs_replica_result* res;   // optional [problems] (poa_total, n_windows filled)
+};
+
+cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
+                       const ModelConsts& mc, cudaStream_t st);
+
+// Live router kernels.
+struct RouterState {
+  uint64_t* keys;           // [W][slots]
+  uint32_t* stamp;
+  uint32_t* log;
+  uint64_t* tmp;            // [K]
+  CacheMeta* meta;          // [W]
+  int64_t* active;          // [W]
+  uint64_t* ordinal;        // [1]
+  int32_t* status;          // [1] sticky device error
+};
+
+cudaError_t launch_route_batch(const RouterState& s, int32_t instance, const int64_t* offsets,
+                               const uint64_t* hashes, int32_t n_req, const int32_t* out_len,
+                               int32_t* worker_out, float* cost_out, int32_t* prefix_out,
+                               int nbmax, const TableGeom& g, const ModelConsts& mc, float omega,
+                               float tau, uint64_t seed, cudaStream_t st);
+size_t router_smem(int W, int nbmax);
+cudaError_t launch_route_release(const RouterState& s, const int32_t* worker, const int32_t* blocks,
+                                 int32_t n, int32_t W, cudaStream_t st);
+cudaError_t launch_clear_tables(uint64_t* keys, uint32_t* stamp, size_t nslots, CacheMeta* meta,
+                                size_t nmeta, cudaStream_t st);
+
+}  // namespace rs

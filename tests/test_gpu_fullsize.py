@@ -1,0 +1,50 @@
+"""Parity at the workloads' own sizes, in the launch configuration the
+benchmark times: every replica of a grid runs in one simulate_replicas call;
+the oracle recomputes sampled replicas one by one."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2606_17081_gb300 import routesim as rs
+from paper_2606_17081_gb300 import workloads as wk
+
+from gpu_helpers import assert_replica_equal, gpu_run, oracle_cfg, oracle_run
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA device", allow_module_level=True)
+
+
+def _check(p, sample, poa=True):
+    traces = p.traces()
+    ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
+    st, g = gpu_run(ctx, traces, p.replicas, with_cost=False)
+    assert st == 0
+    cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
+    for k in sample:
+        r = p.replicas[k]
+        o = oracle_run(cfg, traces[r.trace], r)
+        assert_replica_equal(g[k], o, p.W, check_cost=False)
+        if poa:
+            _, _, _, tot = O.poa(cfg, o)
+            assert abs(g[k]["result"]["poa_total"] - tot) <= 1e-4 * tot
+    return g
+
+
+def test_p2d_full_size_sampled_replicas():
+    p = wk.plan("p2d")
+    g = _check(p, [0, 5, 37, 63])
+    assert all(x["result"]["status"] == 0 for x in g)
+    assert sum(x["result"]["evicted_blocks"] for x in g) > 0
+
+
+def test_p5d_grid_reduced():
+    p = wk.plan("p5d", n_req=3000, replicas=list(range(0, 256, 17)) + [255])
+    _check(p, range(len(p.replicas)))
+
+
+def test_grid_reduced():
+    p = wk.plan("grid", n_req=1500, replicas=list(range(0, 8192, 173)))
+    _check(p, range(len(p.replicas)))
