@@ -858,6 +858,7 @@ static double assign_mcf(const double* cost, int64_t n, int32_t W, int64_t capw,
       for (int64_t k = head[x.v]; k < head[x.v + 1]; k++) {
         if (e[k].capa <= 0) continue;
         double rc = e[k].cost + pot[x.v] - pot[e[k].to];
+        if (rc < 0.0) rc = 0.0;   /* exact reduced costs are >= 0; rounding can dip below */
         double nd = dist[x.v] + rc;
         if (nd < dist[e[k].to]) {
           dist[e[k].to] = nd;
@@ -867,6 +868,7 @@ static double assign_mcf(const double* cost, int64_t n, int32_t W, int64_t capw,
         }
       }
     }
+    if (pe[T] < 0) break;   /* cannot happen while capacity remains */
     for (int64_t v = 0; v < V; v++)
       if (dist[v] < INFINITY) pot[v] += dist[v];
     for (int64_t v = T; v != S;) {
@@ -876,12 +878,17 @@ static double assign_mcf(const double* cost, int64_t n, int32_t W, int64_t capw,
       v = e[e[k].rev].to;
     }
   }
-  for (int64_t i = 0; i < n; i++)
+  int ok = 1;
+  for (int64_t i = 0; i < n; i++) {
+    assign[i] = -1;
     for (int64_t k = head[1 + i]; k < head[2 + i]; k++)
       if (e[k].to >= 1 + n && e[k].to <= n + W && e[k].capa == 0) {
         assign[i] = (int32_t)(e[k].to - 1 - n);
       }
+    if (assign[i] < 0) ok = 0;
+  }
   free(e); free(head); free(deg); free(fill); free(pot); free(dist); free(pe); free(hp);
+  if (!ok) return NAN;
   double total = 0.0;
   for (int64_t i = 0; i < n; i++) total += cost[i * W + assign[i]];
   return total;

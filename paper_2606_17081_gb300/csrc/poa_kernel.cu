@@ -271,8 +271,10 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
             for (int j = 0; j < W; j++)
               for (int k = 0; k < W; k++) {
                 if (k == j || S.wrow[j][k] < 0) continue;
+                // exact cycles are >= 0; relaxing only on gains above 1e-12 keeps
+                // rounding-level negative cycles from looping the predecessors
                 const double nd = __dadd_rn(dist[j], S.wmin[j][k]);
-                if (nd < dist[k]) { dist[k] = nd; pred[k] = j; ch = true; }
+                if (nd < dist[k] - 1e-12) { dist[k] = nd; pred[k] = j; ch = true; }
               }
             if (!ch) break;
           }

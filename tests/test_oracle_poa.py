@@ -159,3 +159,18 @@ def test_game_brute_force_small_by_hand():
     # (0,0): moving costs 1 vs staying 2 - 1.5 = 0.5 -> NE; split profiles: the
     # worker-1 player moving to 0 pays 2 - 1.5 = 0.5 < 1 -> not NE.
     assert g["n_ne"] == 1 and g["worst_ne"] == 1.0
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_assignment_with_heavy_ties(seed):
+    # frozen-cost matrices repeat the same few rows many times (equal loads,
+    # no overlap): every method must still return the same optimum
+    rng = np.random.default_rng(seed)
+    n, W = int(rng.integers(60, 140)), 3
+    loads = rng.integers(1, 6, size=(n, W))
+    c = 0.005 * loads + 0.020 + 0.010 / (64 - loads) ** 2
+    capw = max(64, -(-n // W)) if seed % 2 else -(-n // W)
+    vh, _ = O.assign(c, capw, 1)
+    vm, am = O.assign(c, capw, 2)
+    assert abs(vh - vm) <= 1e-12 * vh
+    assert np.all(np.bincount(am, minlength=W) <= capw)
