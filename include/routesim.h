@@ -189,6 +189,9 @@ typedef struct {
   int64_t ticks_in_regime[3];
   double final_ewma;        /* -1 if no sample */
   int64_t probes;           /* hash-table lookups issued (work counter) */
+  int64_t probe_blocks;     /* sum over decisions and workers of min(m_ij + 1, nb_i):
+                               the lookups a first-miss probe needs */
+  int64_t hashed_blocks;    /* sum of nb_i (full blocks) over routed requests */
   int64_t slow_path;        /* updates that needed the exact sequential path */
   int64_t rebuilds;         /* table/log compactions */
 } rs_replica_result;

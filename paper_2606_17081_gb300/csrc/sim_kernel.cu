@@ -82,7 +82,7 @@ struct SimScalars {
   double prev_arrival, a_cur, rel, rel_next, makespan, sum_ttft, sum_e2e, min_ft, lastL, ewma;
   int64_t next_tick, np, off0, off1, noff0, noff1;
   int64_t near_ties, exact_ties, sampled, near_bd, hit_blocks, inserted, evicted, slow, rebuilds;
-  int64_t ticks, switches, tir[3], n_routed;
+  int64_t ticks, switches, tir[3], n_routed, probe_blocks, hashed_blocks;
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, phase, evres, status, O, nO, jstar, regime, up_cnt, down_cnt;
@@ -633,6 +633,8 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
     __syncthreads();
     // ---- Eq. (2) choice
     if (threadIdx.x == 0) {
+      for (int j = 0; j < W; j++) S.probe_blocks += min(c.wm[j] + 1, nb);
+      S.hashed_blocks += nb;
       const float tau = S.tau_cur;
       const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
       int nbd = 0;
@@ -719,6 +721,8 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
     r.ticks_in_regime[2] = S.tir[2];
     r.final_ewma = S.have_ewma ? S.ewma : -1.0;
     r.probes = (int64_t)S.probes;
+    r.probe_blocks = S.probe_blocks;
+    r.hashed_blocks = S.hashed_blocks;
     r.slow_path = S.slow;
     r.rebuilds = S.rebuilds;
     b.res[sid] = r;

@@ -55,8 +55,9 @@ class rs_replica_result(C.Structure):
                 ("evicted_blocks", C.c_int64), ("ticks", C.c_int64),
                 ("regime_switches", C.c_int64), ("max_regime", C.c_int32),
                 ("reserved0", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
-                ("final_ewma", C.c_double), ("probes", C.c_int64), ("slow_path", C.c_int64),
-                ("rebuilds", C.c_int64)]
+                ("final_ewma", C.c_double), ("probes", C.c_int64),
+                ("probe_blocks", C.c_int64), ("hashed_blocks", C.c_int64),
+                ("slow_path", C.c_int64), ("rebuilds", C.c_int64)]
 
     def as_dict(self) -> dict:
         return {f: (list(getattr(self, f)) if f == "ticks_in_regime" else getattr(self, f))

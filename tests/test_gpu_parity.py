@@ -185,12 +185,11 @@ def test_edge_cases():
     assert st == rs.RS_ERR_CAPACITY == g[0]["result"]["status"]
     assert oracle_run(oracle_cfg(ctx), tr2, rep[0])["status"] == O.ERR_CAPACITY
     # invalid arguments are rejected before any launch
-    with pytest.raises(rs.RoutesimError) as e:
-        gpu_run(ctx, [tr], [wk.Replica(0, 0, 0, 0, 1.0, 0.0, 0, 5)])
-    with pytest.raises(rs.RoutesimError):
-        gpu_run(ctx, [tr], [wk.Replica(3, 2, 0, 0, 1.0, 0.0, 0, 5)])
-    with pytest.raises(rs.RoutesimError):
-        gpu_run(ctx, [tr], [wk.Replica(0, 2, 0, 0, -1.0, 0.0, 0, 5)])
+    for bad in (wk.Replica(0, 0, 0, 0, 1.0, 0.0, 0, 5), wk.Replica(3, 2, 0, 0, 1.0, 0.0, 0, 5),
+                wk.Replica(0, 2, 0, 0, -1.0, 0.0, 0, 5), wk.Replica(0, 2, 7, 0, 1.0, 0.0, 0, 5),
+                wk.Replica(0, 2, 0, 0, 1.0, 0.0, 0, 51)):
+        st, _ = gpu_run(ctx, [tr], [bad])
+        assert st == rs.RS_ERR_INVALID
 
 
 # ------------------------------------------------------------------ PoA (K4)
