@@ -254,6 +254,38 @@ typedef struct {
 } rs_timing;
 rs_status route_last_timing(const rs_ctx* ctx, rs_timing* out);
 
+/* Entry point that allocates nothing.  The paper has no counterpart: this
+ * is a library service for callers that cannot allocate device memory when
+ * they need an estimate -- a serving process whose GPU memory is owned up
+ * front by another allocator, or a latency-critical path where cudaMalloc /
+ * cudaFree would synchronise the device.
+ *
+ * Same result as poa_estimate (Eq. (12) per window of completion time) for
+ * caller records of one replica (device pointers, n rows, cfg->W <= 16
+ * columns), computed in a fixed static device array of RS_NOALLOC_POA_BYTES
+ * bytes that every GPU loading the library holds until the process exits.
+ * No context is needed; nothing is allocated (no cudaMalloc, cudaFree or
+ * allocating library call) and nothing is read back to the host: the work is
+ * enqueued on cuda_stream (NULL = legacy default stream).
+ *   cfg: host struct; poa_window, cap, the latency constants and W are used.
+ *   numer_dev/opt_dev (double) and count_dev (int64), each NULL or
+ *   max_windows entries: the first min(windows, max_windows) windows.
+ *   poa_total_dev (double) and n_windows_dev (int64): one entry each;
+ *   *n_windows_dev = -1 if the records span more than n + 2 windows.
+ * Returns RS_ERR_CAPACITY (before any work) when n rows of W columns need
+ * more than the static array: about n * (8 W + 60) + 2 KB bytes, i.e. up to
+ * roughly 390 000 rows at W = 3.  The first call on a device takes the
+ * array's device address (cudaGetSymbolAddress) for that device; make that
+ * first call before any stream capture.  All calls on a device share the one
+ * array and every call rewrites what it reads, so calls that overlap on the
+ * GPU (other streams, other host threads) race and must be serialised by
+ * the caller. */
+#define RS_NOALLOC_POA_BYTES (32u * 1024u * 1024u)
+rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records* records, int64_t n,
+                               double* numer_dev, double* opt_dev, int64_t* count_dev,
+                               int64_t max_windows, double* poa_total_dev,
+                               int64_t* n_windows_dev, void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -78,7 +78,8 @@ class rs_timing(C.Structure):
 
 EXPORTS = ["rs_config_default", "route_init", "route_destroy", "route_last_error",
            "route_hash_blocks", "route_batch", "route_release", "route_active",
-           "simulate_replicas", "poa_estimate", "route_cache_dump", "route_last_timing"]
+           "simulate_replicas", "poa_estimate", "route_cache_dump", "route_last_timing",
+           "poa_estimate_noalloc"]
 
 _lib = None
 
@@ -114,6 +115,8 @@ def lib():
                                    C.POINTER(C.c_int64), C.POINTER(C.c_double)]),
             "route_cache_dump": (i32, [vp, i32, i32, i32, vp, i64, C.POINTER(C.c_int64)]),
             "route_last_timing": (i32, [vp, C.POINTER(rs_timing)]),
+            "poa_estimate_noalloc": (i32, [C.POINTER(rs_config), C.POINTER(rs_records), i64, vp,
+                                           vp, vp, i64, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -225,6 +228,19 @@ def route_last_timing(ctx) -> rs_timing:
     t = rs_timing()
     lib().route_last_timing(ctx, C.byref(t))
     return t
+
+
+def poa_estimate_noalloc(cfg: rs_config, records: rs_records, n: int, numer_dev, opt_dev,
+                         count_dev, max_windows: int, poa_total_dev, n_windows_dev,
+                         stream: int = 0) -> None:
+    """Eq. (12) estimate in the library's static scratch (no allocation);
+    outputs stay in device memory."""
+    st = lib().poa_estimate_noalloc(C.byref(cfg), C.byref(records), n, _ptr(numer_dev),
+                                    _ptr(opt_dev), _ptr(count_dev), max_windows,
+                                    _ptr(poa_total_dev), _ptr(n_windows_dev),
+                                    C.c_void_p(stream or None))
+    if st != RS_OK:
+        raise RoutesimError(st, "poa_estimate_noalloc rejected the call")
 
 
 # ----------------------------------------------------------------- marshalling helpers
