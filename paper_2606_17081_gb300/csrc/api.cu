@@ -35,7 +35,7 @@ struct rs_ctx {
   int32_t ninst = 0;
   DevBuf r_keys, r_stamp, r_log, r_tmp, r_meta, r_active, r_ord, r_status, r_hash, r_stats;
   // simulation scratch (grow-only)
-  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats;
+  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs;
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -261,7 +261,7 @@ void route_destroy(rs_ctx* ctx) {
   DevBuf* all[] = {&ctx->r_keys, &ctx->r_stamp, &ctx->r_log, &ctx->r_tmp, &ctx->r_meta,
                    &ctx->r_active, &ctx->r_ord, &ctx->r_status, &ctx->r_hash, &ctx->r_stats,
                    &ctx->keys, &ctx->stamp, &ctx->log, &ctx->tmp, &ctx->pend, &ctx->meta_out,
-                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->rec_worker,
+                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->rec_worker,
                    &ctx->rec_arrival, &ctx->rec_start, &ctx->rec_first, &ctx->rec_completion,
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
@@ -274,6 +274,8 @@ void route_destroy(rs_ctx* ctx) {
   delete ctx;
 }
 
+static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbmax_dev);
+
 rs_status route_hash_blocks(rs_ctx* ctx, const int32_t* tokens_dev, const int64_t* offsets_dev,
                             int64_t n_req, uint64_t* hashes_dev) {
   if (!ctx) return fail(nullptr, RS_ERR_INVALID, "ctx is NULL");
@@ -282,9 +284,34 @@ rs_status route_hash_blocks(rs_ctx* ctx, const int32_t* tokens_dev, const int64_
   if (n_req == 0) return RS_OK;
   if (!tokens_dev || !offsets_dev || !hashes_dev) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
   if (!aligned16(tokens_dev)) return fail(ctx, RS_ERR_INVALID, "tokens must be 16-byte aligned");
-  CK(launch_block_hash(tokens_dev, offsets_dev, n_req, ctx->cfg.hash_seed, hashes_dev, nullptr,
-                       ctx->st),
-     "block hash launch");
+  std::vector<HashJob> jobs(1);
+  jobs[0] = HashJob{tokens_dev, offsets_dev, hashes_dev, n_req, 0};
+  return hash_jobs(ctx, jobs, nullptr);
+}
+
+// Hashes every job (trace) in launches of up to HASH_MAX_JOBS traces.
+static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbmax_dev) {
+  if (jobs.empty()) return RS_OK;
+  rs_status r = ensure(ctx, ctx->hjobs, sizeof(HashJob) * jobs.size(), "hash jobs");
+  if (r != RS_OK) return r;
+  CK(cudaMemcpyAsync(ctx->hjobs.p, jobs.data(), sizeof(HashJob) * jobs.size(),
+                     cudaMemcpyHostToDevice, ctx->st),
+     "copy hash jobs");
+  for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
+    const int64_t base = jobs[g0].req_base;
+    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - base;
+    // the kernels number requests from 0 within a launch
+    std::vector<HashJob> grp(jobs.begin() + g0, jobs.begin() + g1);
+    for (auto& j : grp) j.req_base -= base;
+    if (g0 > 0 || base != 0)
+      CK(cudaMemcpyAsync(P<HashJob>(ctx->hjobs) + g0, grp.data(), sizeof(HashJob) * grp.size(),
+                         cudaMemcpyHostToDevice, ctx->st),
+         "copy hash jobs");
+    CK(launch_block_hash(P<HashJob>(ctx->hjobs) + g0, (int)grp.size(), total, ctx->cfg.hash_seed,
+                         nbmax_dev, ctx->st),
+       "block hash launch");
+  }
   return RS_OK;
 }
 
@@ -325,9 +352,11 @@ rs_status route_batch(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
   if (total < 0) return fail(ctx, RS_ERR_INVALID, "offsets[n_req] < 0");
   if ((r = ensure(ctx, ctx->r_hash, (size_t)(total / 16 + 1) * 8, "batch hashes")) != RS_OK) return r;
   CK(cudaMemsetAsync(ctx->r_stats.p, 0, 8, ctx->st), "memset");
-  CK(launch_block_hash(tokens_dev, offsets_dev, n_req, ctx->cfg.hash_seed, P<uint64_t>(ctx->r_hash),
-                       P<int64_t>(ctx->r_stats), ctx->st),
-     "block hash launch");
+  {
+    std::vector<HashJob> jobs(1);
+    jobs[0] = HashJob{tokens_dev, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, 0};
+    if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->r_stats))) != RS_OK) return r;
+  }
   CK(cudaMemcpyAsync(ctx->pinned, ctx->r_stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");
   CK(cudaStreamSynchronize(ctx->st), "sync");
   int64_t nbmax = ctx->pinned[0];
@@ -586,23 +615,24 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   int64_t launches = 0, hashed_tokens = 0;
   CK(cudaEventRecord(ctx->ev[0], ctx->st), "event");
   CK(cudaMemsetAsync(ctx->stats.p, 0, (size_t)n_traces * 8, ctx->st), "memset");
-  for (int t = 0; t < n_traces; t++) {
-    if (!used[t] || traces[t].n_req == 0) continue;
-    CK(launch_block_hash(dtok[t], doff[t], traces[t].n_req, ctx->cfg.hash_seed,
-                         P<uint64_t>(ctx->hashes) + hoff[t], P<int64_t>(ctx->stats) + t, ctx->st),
-       "block hash launch");
-    launches++;
-    hashed_tokens += tot[t];
+  {
+    std::vector<HashJob> jobs;
+    int64_t rb = 0;
+    for (int t = 0; t < n_traces; t++) {
+      if (!used[t] || traces[t].n_req == 0) continue;
+      jobs.push_back(HashJob{dtok[t], doff[t], P<uint64_t>(ctx->hashes) + hoff[t], traces[t].n_req, rb});
+      rb += traces[t].n_req;
+      hashed_tokens += tot[t];
+    }
+    if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->stats))) != RS_OK) return r;
+    launches += 2 * (((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS);
   }
   CK(cudaEventRecord(ctx->ev[1], ctx->st), "event");
-  CK(cudaMemcpyAsync(ctx->pinned, ctx->stats.p, (size_t)n_traces * 8, cudaMemcpyDeviceToHost, ctx->st),
-     "read stats");
+  CK(cudaMemcpyAsync(ctx->pinned, ctx->stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");
   CK(cudaStreamSynchronize(ctx->st), "sync");
-  int64_t nbmax = 1;
-  for (int t = 0; t < n_traces; t++)
-    if (used[t]) nbmax = std::max(nbmax, ctx->pinned[t]);
+  int64_t nbmax = std::max<int64_t>(1, ctx->pinned[0]);
   if (nbmax > (int64_t)g.K) nbmax = g.K;   // longer prompts stop their replica with RS_ERR_CAPACITY
-  const size_t smem = sim_smem_bytes(W, (int)nbmax, cmax);
+  const size_t smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap);
   int maxsmem = 0;
   cudaDeviceGetAttribute(&maxsmem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device);
   if (smem + sizeof(int) * 2048 > (size_t)maxsmem)

@@ -138,6 +138,18 @@ __device__ __forceinline__ int select_worker(const float* c, int W, float tau, u
 
 // ---------------------------------------------------------------- CTA helpers
 
+// Barrier of a thread group made of the CTA's first NT threads: the whole
+// 256-thread CTA uses __syncthreads, a smaller leading group the named
+// barrier 1 (so the remaining warps can work on something else meanwhile).
+template <int NT>
+__device__ __forceinline__ void grp_bar() {
+  if constexpr (NT == 256) {
+    __syncthreads();
+  } else {
+    asm volatile("bar.sync 1, %0;" ::"n"(NT) : "memory");
+  }
+}
+
 // Exclusive rank of `flag` among the CTA's threads (thread order) and the
 // total; two barriers.  warp_tot: shared int[NT/32].
 template <int NT>
@@ -145,7 +157,7 @@ __device__ __forceinline__ int cta_rank(bool flag, int* warp_tot, int* total) {
   const unsigned m = __ballot_sync(FULL_MASK, flag);
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   if (lane == 0) warp_tot[w] = __popc(m);
-  __syncthreads();
+  grp_bar<NT>();
   int off = 0, tot = 0;
 #pragma unroll
   for (int i = 0; i < NT / 32; i++) {
@@ -153,9 +165,33 @@ __device__ __forceinline__ int cta_rank(bool flag, int* warp_tot, int* total) {
     off += i < w ? v : 0;
     tot += v;
   }
-  __syncthreads();
+  grp_bar<NT>();
   *total = tot;
   return off + __popc(m & ((1u << lane) - 1u));
+}
+
+// Exclusive prefix sum of v over the group (thread order) and the total.
+template <int NT>
+__device__ __forceinline__ int grp_excl_scan(int v, int* warp_tot, int* total) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(FULL_MASK, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[w] = x;
+  grp_bar<NT>();
+  int off = 0, tot = 0;
+#pragma unroll
+  for (int i = 0; i < NT / 32; i++) {
+    const int t = warp_tot[i];
+    off += i < w ? t : 0;
+    tot += t;
+  }
+  grp_bar<NT>();
+  *total = tot;
+  return off + x - v;
 }
 
 // ---------------------------------------------------------------- cache table
@@ -245,27 +281,37 @@ struct UpdateShared {   // small shared scalars of the update
 // Rebuilds the table and log of one worker from its live entries in LRU
 // order (stamps renumbered 0..size-1).  tmp: global scratch of >= size keys.
 template <int NT>
-__device__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, uint64_t* tmp,
+__device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, uint64_t* tmp,
                               int* warp_tot, UpdateShared* us) {
   const uint32_t head = meta->head, T = meta->T;
+  constexpr int PER = 8;   // log entries per thread per step: independent loads in flight
   uint32_t base = 0;
-  for (uint32_t p0 = head; p0 < T; p0 += NT) {
-    const uint32_t p = p0 + threadIdx.x;
-    bool live = false;
-    uint32_t x = 0;
-    if (p < T) {
-      x = t.log[p & t.rmask];
-      live = __ldcg(t.stamp + x) == p;
+  for (uint32_t p0 = head; p0 < T; p0 += NT * PER) {
+    const uint32_t pb = p0 + threadIdx.x * PER;
+    uint32_t x[PER];
+    bool live[PER];
+    int cnt = 0;
+#pragma unroll
+    for (int e = 0; e < PER; e++) x[e] = pb + e < T ? t.log[(pb + e) & t.rmask] : 0u;
+#pragma unroll
+    for (int e = 0; e < PER; e++) {
+      live[e] = pb + e < T && __ldcg(t.stamp + x[e]) == pb + e;
+      cnt += live[e];
     }
     int tot;
-    const int r = cta_rank<NT>(live, warp_tot, &tot);
-    if (live && base + r < K) tmp[base + r] = __ldcg(t.keys + x);
+    int off = grp_excl_scan<NT>(cnt, warp_tot, &tot);
+#pragma unroll
+    for (int e = 0; e < PER; e++)
+      if (live[e]) {
+        if (base + off < K) tmp[base + off] = __ldcg(t.keys + x[e]);
+        off++;
+      }
     base += tot;
   }
-  __syncthreads();
+  grp_bar<NT>();
   if (base > K) {   // more live log entries than the cache holds: inconsistent state
     if (threadIdx.x == 0) us->err = RS_ERR_TIMEOUT;
-    __syncthreads();
+    grp_bar<NT>();
     return;
   }
   const size_t nslots = 4 * ((size_t)t.bmask + 1);
@@ -273,7 +319,7 @@ __device__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, u
     t.keys[s] = KEY_EMPTY;
     t.stamp[s] = STAMP_NONE;
   }
-  __syncthreads();
+  grp_bar<NT>();
   for (uint32_t r = threadIdx.x; r < base; r += NT) {
     int wt = 0, e = 0;
     const uint32_t sl = table_insert(t, __ldcg(tmp + r), &wt, &e);
@@ -283,14 +329,14 @@ __device__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, u
       t.log[r & t.rmask] = sl;
     }
   }
-  __syncthreads();
+  grp_bar<NT>();
   if (threadIdx.x == 0) {
     if (base != meta->size) us->err = RS_ERR_TIMEOUT;
     meta->head = 0;
     meta->T = base;
     meta->tombs = 0;
   }
-  __syncthreads();
+  grp_bar<NT>();
 }
 
 // Resets the shared scalars of one cache update.
@@ -310,7 +356,7 @@ __device__ __forceinline__ void update_reset(UpdateShared* us) {
 // within the request (a shared-memory open-addressing set; each thread clears
 // the slot it claimed).  us must be reset before the call.
 template <int NT>
-__device__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int nb,
+__device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int nb,
                                  UpdateScratch& sc, UpdateShared* us,
                                  unsigned long long* probes) {
   int nabs = 0, err = 0, dup = 0;
@@ -339,12 +385,16 @@ __device__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int n
     }
     sc.owner[k] = claimed;
   }
-  if (nabs) atomicAdd(&us->n_absent, nabs);
-  if (pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  nabs = __reduce_add_sync(FULL_MASK, (unsigned)nabs);
+  pmin = __reduce_min_sync(FULL_MASK, pmin);
+  if ((threadIdx.x & 31) == 0) {
+    if (nabs) atomicAdd(&us->n_absent, nabs);
+    if (pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  }
   if (err) us->err = RS_ERR_TIMEOUT;
   if (dup) us->dup = 1;
   if (threadIdx.x == 0) atomicAdd(probes, (unsigned long long)nb);
-  __syncthreads();
+  grp_bar<NT>();
   for (int k = threadIdx.x; k < nb; k += NT)
     if (sc.owner[k] >= 0) sc.dupset[sc.owner[k]] = 0ull;
 }
@@ -352,7 +402,7 @@ __device__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int n
 // Gathers live log entries starting at meta->head until `want` are held
 // (or the log ends).  Continues from us->gathered entries already held.
 template <int NT>
-__device__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t* pos,
+__device__ __forceinline__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t* pos,
                             uint32_t want, UpdateScratch& sc, UpdateShared* us, int* warp_tot) {
   const uint32_t T = meta->T;
   uint32_t have = us->gathered;
@@ -374,12 +424,12 @@ __device__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t*
     have = min(want, have + (uint32_t)tot);
     p0 += NT;
   }
-  __syncthreads();
+  grp_bar<NT>();
   if (threadIdx.x == 0) {
     us->gathered = have;
     *pos = p0;
   }
-  __syncthreads();
+  grp_bar<NT>();
 }
 
 // Applies one request's block list to the chosen worker's cache: exact LRU
@@ -387,7 +437,7 @@ __device__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t*
 // inserted, the least-recent entry evicted whenever the cache is full).
 // Returns through us: n_victims, n_ins; updates meta.  CTA-wide.
 template <int NT>
-__device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, const uint64_t* hbuf,
+__device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, const uint64_t* hbuf,
                             int nb, UpdateScratch& sc, UpdateShared* us, int* warp_tot,
                             uint32_t* scan_pos) {
   const uint32_t size = meta->size;
@@ -398,11 +448,11 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
     us->gathered = 0;
     *scan_pos = meta->head;
   }
-  __syncthreads();
+  grp_bar<NT>();
   if (E0 > 0) gather_live<NT>(t, meta, scan_pos, E0, sc, us, warp_tot);
   if (E0 > 0 && us->gathered < E0) {   // fewer live entries than the size says
     if (threadIdx.x == 0) us->err = RS_ERR_TIMEOUT;
-    __syncthreads();
+    grp_bar<NT>();
     return;
   }
   const bool fast = E0 == 0 || us->pmin > sc.vt[E0 - 1];
@@ -410,24 +460,24 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
     for (int k = threadIdx.x; k < nb; k += NT) sc.kind[k] = sc.slot[k] == SLOT_NONE;
     for (uint32_t v = threadIdx.x; v < E0; v += NT) sc.victim[v] = (int32_t)v;
     if (threadIdx.x == 0) us->n_victims = (int)E0;
-    __syncthreads();
+    grp_bar<NT>();
   } else {
     // exact sequential emulation over the first live entries (gathered again
     // from the head: the first pass dropped live entries past the E0-th)
     const uint32_t want = min(size, 2u * (uint32_t)nb);
-    __syncthreads();
+    grp_bar<NT>();
     if (threadIdx.x == 0) {
       us->gathered = 0;
       *scan_pos = meta->head;
     }
-    __syncthreads();
+    grp_bar<NT>();
     gather_live<NT>(t, meta, scan_pos, want, sc, us, warp_tot);
     const uint32_t G = us->gathered;
     for (uint32_t p = threadIdx.x; p < G; p += NT) {
       sc.owner[p] = -1;
       sc.touched[p] = 0;
     }
-    __syncthreads();
+    grp_bar<NT>();
     const uint32_t last = G ? sc.vt[G - 1] : 0u;
     for (int k = threadIdx.x; k < nb; k += NT) {
       const uint32_t st = sc.pst[k];
@@ -440,7 +490,7 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
         sc.owner[lo] = k;
       }
     }
-    __syncthreads();
+    grp_bar<NT>();
     if (threadIdx.x == 0) {
       uint32_t ptr = 0, sz = size;
       int E = 0;
@@ -474,7 +524,7 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
       us->n_victims = E;
       us->slow = 1;
     }
-    __syncthreads();
+    grp_bar<NT>();
   }
   const int E = us->n_victims;
   // evictions first (tombstones), then inserts, then stamps and log
@@ -483,7 +533,7 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
     t.keys[x] = KEY_TOMB;
     t.stamp[x] = STAMP_NONE;
   }
-  __syncthreads();
+  grp_bar<NT>();
   const uint32_t T = meta->T;
   int nins = 0, recl = 0, err = 0;
   for (int k = threadIdx.x; k < nb; k += NT) {
@@ -500,17 +550,21 @@ __device__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, con
       t.log[(T + (uint32_t)k) & t.rmask] = sl;
     }
   }
-  if (nins) atomicAdd(&us->n_ins, nins);
-  if (recl) atomicAdd(&us->reclaimed, recl);
+  nins = __reduce_add_sync(FULL_MASK, (unsigned)nins);
+  recl = __reduce_add_sync(FULL_MASK, (unsigned)recl);
+  if ((threadIdx.x & 31) == 0) {
+    if (nins) atomicAdd(&us->n_ins, nins);
+    if (recl) atomicAdd(&us->reclaimed, recl);
+  }
   if (err) us->err = RS_ERR_TIMEOUT;
-  __syncthreads();
+  grp_bar<NT>();
   if (threadIdx.x == 0) {
     meta->tombs = meta->tombs + (uint32_t)E - (uint32_t)us->reclaimed;
     meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
     if (E > 0) meta->head = sc.vt[sc.victim[E - 1]] + 1;
     meta->T = T + (uint32_t)nb;
   }
-  __syncthreads();
+  grp_bar<NT>();
 }
 
 }  // namespace rs

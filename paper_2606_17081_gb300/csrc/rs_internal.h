@@ -74,10 +74,20 @@ struct SimLaunch {
   ModelConsts mc;
 };
 
-size_t sim_smem_bytes(int W, int nbmax, int cmax);
-cudaError_t launch_block_hash(const int32_t* tokens, const int64_t* offsets, int64_t n_req,
-                              uint64_t seed, uint64_t* out, int64_t* nbmax_out,
-                              cudaStream_t st);
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap);
+
+// One trace for the block-hash kernels: requests req_base .. req_base+n_req-1
+// of the launch's global request numbering.
+struct HashJob {
+  const int32_t* tokens;
+  const int64_t* offsets;
+  uint64_t* out;
+  int64_t n_req;
+  int64_t req_base;
+};
+constexpr int HASH_MAX_JOBS = 64;
+cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
+                              int64_t* nbmax_out, cudaStream_t st);
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st);
 

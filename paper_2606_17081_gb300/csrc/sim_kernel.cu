@@ -8,28 +8,40 @@
 // current Eq. (11) regime when the controller is on), the chosen worker's
 // LRU cache update and load update -- and its Eq. (9) latency.
 //
-// Thread 0 owns the scalar event state (completion heap, FIFO queues,
-// controller) in shared memory; every data-parallel step (hash staging,
-// probes, the cache update, controller percentile) uses the whole CTA.
-// Floating point follows the paper's formulas operation by operation
-// (explicit _rn intrinsics, no contraction).
+// Per request i (256 threads, 8 warps):
+//   probe      all warps: cached prefix m_ij on every worker;
+//   choose     warp 0: Eq. (1) costs and the Eq. (2) choice; warp 1: tie stats;
+//   update     warps 0-6 (named barrier): the chosen worker's cache;
+//   control    warp 7, at the same time: request i's load, service start and
+//              latency, then request i+1's completions and controller samples
+//              up to its arrival, and its block hashes into the other buffer.
+// The control work is serial and runs on float64, whose dependent-operation
+// latency on this GPU is long; the cache update is memory-bound.  Neither needs
+// the other's results, so they overlap.  Times are ordered through an integer
+// key of their bit patterns (same order as the float64 comparison, no FP64
+// compare on the serial path).  Floating point follows the paper's formulas
+// operation by operation (explicit _rn intrinsics, no contraction).
 #include "rs_device.cuh"
 
 namespace rs {
 
+constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (warps 0-6)
+constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
+constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
+
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct SimLayout {
-  size_t f_a, f_o, h_t, hbuf, dupset;
-  size_t f_req, f_worker, f_blk, f_O, f_next, h_f, freestk, owner, victim;
+  size_t ftab, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
+  size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
   size_t slot, pst, vslot, vt;
-  size_t wmeta, winserv, wA, wqh, wqt, wm, wcost, wopen;
+  size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen;
   size_t kind, evk, touched;
   size_t total;
   uint32_t dupmask;
 };
 
-__host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax) {
+__host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax, int nft) {
   SimLayout L;
   size_t o = 0;
   const size_t nb = (size_t)(nbmax > 0 ? nbmax : 1);
@@ -42,16 +54,18 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax)
   o = align_up(o, al);         \
   L.field = o;                 \
   o += (bytes);
-  TAKE(f_a, 8 * C, 16)
+  TAKE(ftab, 8 * (size_t)(nft > 0 ? nft : 1), 16)
+  TAKE(f_oitl, 8 * C, 8)
+  TAKE(f_a, 8 * C, 8)
   TAKE(f_o, 8 * C, 8)
-  TAKE(h_t, 8 * C, 8)
-  TAKE(hbuf, 8 * nb, 16)
+  TAKE(h_k, 8 * C, 8)
+  TAKE(hbuf0, 8 * nb, 16)
+  TAKE(hbuf1, 8 * nb, 16)
   TAKE(dupset, 8 * dup, 16)
   TAKE(wA, 8 * (size_t)W, 8)
   TAKE(f_req, 4 * C, 4)
   TAKE(f_worker, 4 * C, 4)
   TAKE(f_blk, 4 * C, 4)
-  TAKE(f_O, 4 * C, 4)
   TAKE(f_next, 4 * C, 4)
   TAKE(h_f, 4 * C, 4)
   TAKE(freestk, 4 * C, 4)
@@ -76,18 +90,32 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax)
   return L;
 }
 
-size_t sim_smem_bytes(int W, int nbmax, int cmax) { return make_sim_layout(W, nbmax, cmax).total; }
+__host__ __device__ inline int ftab_size(int cap) { return cap < FTAB_MAX ? cap : FTAB_MAX; }
+
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap) {
+  return make_sim_layout(W, nbmax, cmax, ftab_size(cap)).total;
+}
+
+// One request as the loop sees it (two live at once: i and i+1).
+struct ReqState {
+  int64_t off0;
+  int64_t blk;     // ceil((L + O) / 16): active blocks while unfinished
+  double a;        // arrival
+  double rel;      // client release time
+  int nb, nbt, O, phase;
+  float tau, omega;
+};
 
 struct SimScalars {
-  double prev_arrival, a_cur, rel, rel_next, makespan, sum_ttft, sum_e2e, min_ft, lastL, ewma;
-  int64_t next_tick, np, off0, off1, noff0, noff1;
+  ReqState q[2];
+  double prev_arrival, min_ft, tick_t, lastL, ewma, sum_ttft, sum_e2e, makespan;
+  int64_t next_tick, np;
   int64_t near_ties, exact_ties, sampled, near_bd, hit_blocks, inserted, evicted, slow, rebuilds;
   int64_t ticks, switches, tir[3], n_routed, probe_blocks, hashed_blocks;
   unsigned long long probes;
   uint64_t sel_prefix;
-  int32_t in_flight, nheap, nfree, phase, evres, status, O, nO, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, nw;
-  float tau_cur, omega_cur;
+  int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
+  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild;
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
@@ -102,9 +130,10 @@ struct SimCtx {
   const SimBuffers* b;
   const SimLaunch* L;
   int sid;
-  double *f_a, *f_o, *h_t;
-  uint64_t* hbuf;
-  int32_t *f_req, *f_worker, *f_blk, *f_O, *f_next, *h_f, *freestk;
+  double *f_a, *f_o, *ftab, *f_oitl;
+  uint64_t* h_k;
+  uint64_t* hbuf[2];
+  int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
   int32_t *winserv, *wqh, *wqt, *wm, *wopen;
   int64_t* wA;
@@ -112,7 +141,7 @@ struct SimCtx {
   UpdateScratch sc;
   double *pend_ft[2], *pend_tt[2], *pend_win;
 
-  __device__ TableView table(int j) const {
+  __device__ __forceinline__ TableView table(int j) const {
     TableView t;
     const size_t wi = (size_t)sid * L->mc.W + j;
     t.keys = b->keys + wi * L->g.slots;
@@ -124,42 +153,56 @@ struct SimCtx {
   }
 };
 
-// ------------------------------------------------------------ event machinery (thread 0)
+// Monotone integer key of a float64 (same order as the float64 comparison
+// for every non-NaN value) and its inverse.
+__device__ __forceinline__ uint64_t tkey(double x) {
+  const uint64_t b = (uint64_t)__double_as_longlong(x);
+  return (b >> 63) ? ~b : (b | 0x8000000000000000ull);
+}
+__device__ __forceinline__ double tval(uint64_t k) {
+  const uint64_t b = (k >> 63) ? (k & 0x7FFFFFFFFFFFFFFFull) : ~k;
+  return __longlong_as_double((long long)b);
+}
+constexpr uint64_t KEY_INF = 0xFFF0000000000000ull;   // tkey(+infinity)
 
-__device__ __forceinline__ bool ev_less(const SimCtx& c, double ta, int fa, double tb, int fb) {
-  return ta < tb || (ta == tb && c.f_req[fa] < c.f_req[fb]);
+// ------------------------------------------------------------ event machinery (control thread)
+
+__device__ __forceinline__ bool ev_less(const SimCtx& c, uint64_t ka, int fa, uint64_t kb, int fb) {
+  return ka < kb || (ka == kb && c.f_req[fa] < c.f_req[fb]);
 }
 
-__device__ void heap_push(SimCtx& c, double t, int f) {
+__device__ __forceinline__ void heap_push(SimCtx& c, uint64_t k, int f) {
   int i = c.S->nheap++;
-  c.h_t[i] = t;
-  c.h_f[i] = f;
   while (i > 0) {
     const int p = (i - 1) >> 1;
-    if (!ev_less(c, c.h_t[i], c.h_f[i], c.h_t[p], c.h_f[p])) break;
-    const double tt = c.h_t[i]; c.h_t[i] = c.h_t[p]; c.h_t[p] = tt;
-    const int ff = c.h_f[i]; c.h_f[i] = c.h_f[p]; c.h_f[p] = ff;
+    if (!ev_less(c, k, f, c.h_k[p], c.h_f[p])) break;
+    c.h_k[i] = c.h_k[p];
+    c.h_f[i] = c.h_f[p];
     i = p;
   }
+  c.h_k[i] = k;
+  c.h_f[i] = f;
 }
 
-__device__ void heap_pop(SimCtx& c, double* t, int* f) {
-  *t = c.h_t[0];
+__device__ __forceinline__ void heap_pop(SimCtx& c, uint64_t* k, int* f) {
+  *k = c.h_k[0];
   *f = c.h_f[0];
   const int n = --c.S->nheap;
-  c.h_t[0] = c.h_t[n];
-  c.h_f[0] = c.h_f[n];
+  const uint64_t lk = c.h_k[n];
+  const int lf = c.h_f[n];
   int i = 0;
   for (;;) {
     const int l = 2 * i + 1, r = l + 1;
-    int s = i;
-    if (l < n && ev_less(c, c.h_t[l], c.h_f[l], c.h_t[s], c.h_f[s])) s = l;
-    if (r < n && ev_less(c, c.h_t[r], c.h_f[r], c.h_t[s], c.h_f[s])) s = r;
-    if (s == i) break;
-    const double tt = c.h_t[i]; c.h_t[i] = c.h_t[s]; c.h_t[s] = tt;
-    const int ff = c.h_f[i]; c.h_f[i] = c.h_f[s]; c.h_f[s] = ff;
+    if (l >= n) break;
+    int s = l;
+    if (r < n && ev_less(c, c.h_k[r], c.h_f[r], c.h_k[l], c.h_f[l])) s = r;
+    if (!ev_less(c, c.h_k[s], c.h_f[s], lk, lf)) break;
+    c.h_k[i] = c.h_k[s];
+    c.h_f[i] = c.h_f[s];
     i = s;
   }
+  c.h_k[i] = lk;
+  c.h_f[i] = lf;
 }
 
 // Eq. (9) with beta = 2: f(n) = a n + b + d / (cap - n)^2
@@ -171,40 +214,37 @@ __device__ __forceinline__ double latency_f(const ModelConsts& mc, int n) {
   return __dadd_rn(t2, t3);
 }
 
-__device__ void start_service(SimCtx& c, int f, int j, double t) {
+// Service of slot f starts on worker j at time t: TTFT = wait + f(n) - w_c o.
+__device__ __forceinline__ void start_service(SimCtx& c, int f, int j, double t) {
   SimScalars& S = *c.S;
   const ModelConsts& mc = c.L->mc;
   const int n = ++c.winserv[j];
-  const double fv = latency_f(mc, n);
-  const double svc = __dsub_rn(fv, __dmul_rn(mc.w_c, c.f_o[f]));
+  const double fv = n < FTAB_MAX ? c.ftab[n] : latency_f(mc, n);
+  const double svc = __dsub_rn(fv, c.f_o[f]);          // f_o holds w_c * o
   const double ft = __dadd_rn(t, svc);
-  const double a = c.f_a[f];
-  const double tt = __dsub_rn(ft, a);
-  const double ct = __dadd_rn(ft, __dmul_rn((double)c.f_O[f], mc.itl));
+  const double tt = __dsub_rn(ft, c.f_a[f]);
+  const double ct = __dadd_rn(ft, c.f_oitl[f]);         // O * itl
   const int64_t row = c.d->rec_base + c.f_req[f];
   c.b->rec.start[row] = t;
   c.b->rec.first_token[row] = ft;
   c.b->rec.ttft[row] = tt;
   c.b->rec.completion[row] = ct;
-  heap_push(c, ct, f);
+  heap_push(c, tkey(ct), f);
   if (c.d->controller) {
     const int cur = S.pend_cur;
     c.pend_ft[cur][S.np] = ft;
     c.pend_tt[cur][S.np] = tt;
     S.np++;
-    if (ft < S.min_ft) S.min_ft = ft;
+    if (tkey(ft) < tkey(S.min_ft)) S.min_ft = ft;
   }
-  S.sum_ttft = __dadd_rn(S.sum_ttft, tt);
-  S.sum_e2e = __dadd_rn(S.sum_e2e, __dsub_rn(ct, a));
 }
 
-__device__ void complete(SimCtx& c, int f, double t) {
+__device__ __forceinline__ void complete(SimCtx& c, int f, double t) {
   SimScalars& S = *c.S;
   const int j = c.f_worker[f];
   c.winserv[j]--;
   c.wA[j] -= c.f_blk[f];
   S.in_flight--;
-  if (t > S.makespan) S.makespan = t;
   c.freestk[S.nfree++] = f;
   const int f2 = c.wqh[j];
   if (f2 >= 0) {
@@ -215,7 +255,7 @@ __device__ void complete(SimCtx& c, int f, double t) {
 }
 
 // EWMA of Eq. (10) and the hysteretic regime of Eq. (11); one sample.
-__device__ void ctl_sample(SimCtx& c, bool has_window, double Lw) {
+__device__ __forceinline__ void ctl_sample(SimCtx& c, bool has_window, double Lw) {
   SimScalars& S = *c.S;
   const ModelConsts& mc = c.L->mc;
   double L = 0.0;
@@ -256,61 +296,60 @@ __device__ void ctl_sample(SimCtx& c, bool has_window, double Lw) {
   S.tir[S.regime]++;
   S.ticks++;
   S.next_tick++;
+  S.tick_t = __dmul_rn((double)S.next_tick, mc.dt);
   if (S.ticks >= TICK_LIMIT) S.status = RS_ERR_CAPACITY;
 }
 
-__device__ __forceinline__ double tick_time(const SimCtx& c) {
-  return c.d->controller ? __dmul_rn((double)c.S->next_tick, c.L->mc.dt) : __longlong_as_double(0x7FF0000000000000ll);
+__device__ __forceinline__ uint64_t tick_key(const SimCtx& c) {
+  return c.d->controller ? tkey(c.S->tick_t) : KEY_INF;
 }
 
-// Advances events for the current request (thread 0).  Returns 1 when a
-// controller sample with a non-empty window is due (the CTA computes it),
-// 0 when the arrival time is known and every event up to it is processed.
-__device__ int events_advance(SimCtx& c) {
+// Advances events for request q (control thread).  Returns 1 when a
+// controller sample with a non-empty window is due (the CTA computes it), 0
+// when the arrival time is known and every event up to it is processed.
+__device__ __forceinline__ int events_advance(SimCtx& c, ReqState& q) {
   SimScalars& S = *c.S;
-  const double INF = __longlong_as_double(0x7FF0000000000000ll);
-  if (S.phase == 0) {
+  if (q.phase == 0) {
     double T = S.prev_arrival;
     if (S.in_flight >= c.d->C) {
       for (;;) {
         if (S.status != RS_OK) return 0;
         if (S.nheap == 0) {   // cannot happen: every request in flight is in service or queued
           S.status = RS_ERR_TIMEOUT;
-          S.a_cur = T;
-          S.phase = 1;
           return 0;
         }
-        const double tc = c.h_t[0];
-        const double tt = tick_time(c);
-        if (tt < tc) {
-          if (S.min_ft >= tt) { ctl_sample(c, false, 0.0); continue; }
+        const uint64_t kc = c.h_k[0];
+        const uint64_t kt = tick_key(c);
+        if (kt < kc) {
+          if (tkey(S.min_ft) >= kt) { ctl_sample(c, false, 0.0); continue; }
           return 1;
         }
-        double t;
+        uint64_t k;
         int f;
-        heap_pop(c, &t, &f);
+        heap_pop(c, &k, &f);
+        const double t = tval(k);
         complete(c, f, t);
-        if (t > T) T = t;
+        if (k > tkey(T)) T = t;
         break;
       }
     }
-    S.a_cur = S.rel > T ? S.rel : T;
-    S.phase = 1;
+    q.a = tkey(q.rel) > tkey(T) ? q.rel : T;
+    q.phase = 1;
   }
-  const double a = S.a_cur;
+  const uint64_t ka = tkey(q.a);
   for (;;) {
     if (S.status != RS_OK) return 0;
-    const double tc = S.nheap > 0 ? c.h_t[0] : INF;
-    const double tt = tick_time(c);
-    if (tc <= tt) {
-      if (tc > a) break;
-      double t;
+    const uint64_t kc = S.nheap > 0 ? c.h_k[0] : KEY_INF;
+    const uint64_t kt = tick_key(c);
+    if (kc <= kt) {
+      if (kc > ka) break;
+      uint64_t k;
       int f;
-      heap_pop(c, &t, &f);
-      complete(c, f, t);
+      heap_pop(c, &k, &f);
+      complete(c, f, tval(k));
     } else {
-      if (tt > a) break;
-      if (S.min_ft >= tt) { ctl_sample(c, false, 0.0); continue; }
+      if (kt > ka) break;
+      if (tkey(S.min_ft) >= kt) { ctl_sample(c, false, 0.0); continue; }
       return 1;
     }
   }
@@ -322,9 +361,9 @@ __device__ int events_advance(SimCtx& c) {
 // The window holds the TTFTs of requests whose first token came before the
 // sample time and after the previous sample; its nearest-rank P99 (exact
 // radix selection over the float64 bit patterns, TTFT > 0) feeds Eq. (10).
-__device__ void tick_cta(SimCtx& c) {
+__device__ __forceinline__ void tick_cta(SimCtx& c) {
   SimScalars& S = *c.S;
-  const double tt = __dmul_rn((double)S.next_tick, c.L->mc.dt);
+  const double tt = S.tick_t;
   const int cur = S.pend_cur;
   const int64_t np = S.np;
   const double* sft = c.pend_ft[cur];
@@ -332,7 +371,8 @@ __device__ void tick_cta(SimCtx& c) {
   double* dft = c.pend_ft[cur ^ 1];
   double* dtt = c.pend_tt[cur ^ 1];
   int64_t nkeep = 0, nwin = 0;
-  double mft = __longlong_as_double(0x7FF0000000000000ll);
+  uint64_t mft = KEY_INF;
+  const uint64_t ktt = tkey(tt);
   for (int64_t p0 = 0; p0 < np; p0 += NT_SIM) {
     const int64_t p = p0 + threadIdx.x;
     bool keep = false, inwin = false;
@@ -340,7 +380,7 @@ __device__ void tick_cta(SimCtx& c) {
     if (p < np) {
       f = sft[p];
       v = stt[p];
-      inwin = f < tt;
+      inwin = tkey(f) < ktt;
       keep = !inwin;
     }
     int t1, t2;
@@ -349,15 +389,18 @@ __device__ void tick_cta(SimCtx& c) {
     if (keep) {
       dft[nkeep + r1] = f;
       dtt[nkeep + r1] = v;
-      mft = fmin(mft, f);
+      const uint64_t kf = tkey(f);
+      mft = kf < mft ? kf : mft;
     }
     if (inwin) c.pend_win[nwin + r2] = v;
     nkeep += t1;
     nwin += t2;
   }
-  // CTA minimum of the kept first-token times
-  for (int o = 16; o > 0; o >>= 1) mft = fmin(mft, __shfl_xor_sync(FULL_MASK, mft, o));
-  if ((threadIdx.x & 31) == 0) S.red[threadIdx.x >> 5] = mft;
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t v = __shfl_xor_sync(FULL_MASK, mft, o);
+    mft = v < mft ? v : mft;
+  }
+  if ((threadIdx.x & 31) == 0) S.red[threadIdx.x >> 5] = tval(mft);
   if (threadIdx.x == 0) {
     S.sel_prefix = 0;
     S.sel_kk = (int)((99 * nwin + 99) / 100);
@@ -390,40 +433,52 @@ __device__ void tick_cta(SimCtx& c) {
     }
     L = __longlong_as_double((long long)S.sel_prefix);
   }
-  if (threadIdx.x == 0) {
-    double m = S.red[0];
-    for (int w = 1; w < NT_SIM / 32; w++) m = fmin(m, S.red[w]);
+  if (threadIdx.x == CTL) {
+    uint64_t m = tkey(S.red[0]);
+    for (int w = 1; w < NT_SIM / 32; w++) {
+      const uint64_t k = tkey(S.red[w]);
+      m = k < m ? k : m;
+    }
     S.np = nkeep;
     S.pend_cur = cur ^ 1;
-    S.min_ft = m;
+    S.min_ft = tval(m);
     ctl_sample(c, nwin > 0, L);
   }
   __syncthreads();
 }
 
-// ------------------------------------------------------------ routing step (CTA)
+// ------------------------------------------------------------ routing step
 
-// m_j: leading blocks of the prompt found in worker j's cache, for every j.
-// Rounds of CH blocks per still-undecided worker; a worker is decided once a
-// miss is found below the round's end.
-__device__ void probe_prefixes(SimCtx& c, int nb) {
+// m_j: leading blocks of the prompt found in worker j's cache, for every j
+// (all threads).  Rounds of CH blocks per still-undecided worker; a worker is
+// decided once a miss is found below the round's end.
+__device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
   const int CH = max(32, ((4 * NT_SIM) / W) & ~31);
   int c0 = 0;
   int err = 0;
-  unsigned long long cnt = 0;
+  unsigned cnt = 0;
   for (;;) {
     const int nopen = S.nopen;
     const int len = min(CH, nb - c0);
     const int total = len > 0 ? nopen * len : 0;
-    for (int it = threadIdx.x; it < total; it += NT_SIM) {
-      const int jj = c.wopen[it / len];
-      const int k = c0 + it % len;
-      if (k < c.wm[jj]) {
-        cnt++;
-        if (table_find(c.table(jj), c.hbuf[k], &err) == SLOT_NONE) atomicMin(&c.wm[jj], k);
+    const int rounds = (total + NT_SIM - 1) / NT_SIM;
+    for (int q = 0; q < rounds; q++) {        // uniform trip count: warp reductions below
+      const int it = q * NT_SIM + threadIdx.x;
+      int jj = -1, miss = 0x7FFFFFFF;
+      if (it < total) {
+        jj = c.wopen[it / len];
+        const int k = c0 + it % len;
+        if (k < c.wm[jj]) {
+          cnt++;
+          if (table_find(c.table(jj), hbuf[k], &err) == SLOT_NONE) miss = k;
+        }
       }
+      const unsigned grp = __match_any_sync(FULL_MASK, jj);
+      const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
+      if (jj >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
+        atomicMin(&c.wm[jj], m);
     }
     __syncthreads();
     c0 += CH;
@@ -437,42 +492,108 @@ __device__ void probe_prefixes(SimCtx& c, int nb) {
     __syncthreads();
     if (S.nopen == 0) break;
   }
-  if (cnt) atomicAdd(&S.probes, cnt);
+  cnt = __reduce_add_sync(FULL_MASK, cnt);
+  if ((threadIdx.x & 31) == 0 && cnt) atomicAdd(&S.probes, (unsigned long long)cnt);
   if (err) S.status = RS_ERR_TIMEOUT;
 }
 
-// Cache update of the chosen worker (CTA).
-__device__ void update_chosen(SimCtx& c, int j, int nb) {
+// Cache update of the chosen worker (update group, warps 0-6).
+__device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb) {
   SimScalars& S = *c.S;
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
   CacheMeta* meta = &c.wmeta[j];
   if (threadIdx.x == 0) {
     const uint64_t span = (uint64_t)meta->T - meta->head + (uint64_t)nb;
-    S.rebuild = span > g.R || meta->tombs > g.slots / 8 || (uint64_t)meta->T + nb > STAMP_LIMIT;
+    S.rebuild = span > g.R || meta->tombs > g.slots / 4 || (uint64_t)meta->T + nb > STAMP_LIMIT;
     update_reset(&S.us);
     S.us.err = 0;
   }
-  __syncthreads();
+  grp_bar<NT_UPD>();
   if (S.rebuild) {
-    cache_rebuild<NT_SIM>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
+    cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
     if (threadIdx.x == 0) S.rebuilds++;
   }
-  cache_lookup_all<NT_SIM>(tv, c.hbuf, nb, c.sc, &S.us, &S.probes);
-  __syncthreads();
+  cache_lookup_all<NT_UPD>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
+  grp_bar<NT_UPD>();
   if (S.us.dup) {
     if (threadIdx.x == 0) S.status = RS_ERR_COLLISION;
-    __syncthreads();
     return;
   }
-  cache_apply<NT_SIM>(tv, meta, g.K, c.hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos);
+  cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos);
   if (threadIdx.x == 0) {
     if (S.us.err) S.status = S.us.err;
     S.inserted += S.us.n_ins;
     S.evicted += S.us.n_victims;
     S.slow += S.us.slow;
   }
-  __syncthreads();
+}
+
+// Request i's load, records and service start (control thread).
+__device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64_t i) {
+  SimScalars& S = *c.S;
+  const ModelConsts& mc = c.L->mc;
+  const int js = S.jstar;
+  const int f = c.freestk[--S.nfree];
+  c.f_req[f] = (int32_t)i;
+  c.f_worker[f] = js;
+  c.f_blk[f] = (int32_t)q.blk;
+  c.f_a[f] = q.a;
+  const double o = q.nbt > 0 ? __ddiv_rn((double)c.wm[js], (double)q.nbt) : 0.0;
+  c.f_o[f] = __dmul_rn(mc.w_c, o);
+  c.f_oitl[f] = __dmul_rn((double)q.O, mc.itl);
+  c.wA[js] += q.blk;
+  S.in_flight++;
+  S.hit_blocks += c.wm[js];
+  const int64_t row = c.d->rec_base + i;
+  c.b->rec.worker[row] = js;
+  c.b->rec.arrival[row] = q.a;
+  c.b->rec.nbt[row] = q.nbt;
+  if (c.winserv[js] < mc.cap - 1) {
+    start_service(c, f, js, q.a);
+  } else {
+    c.f_next[f] = -1;
+    if (c.wqt[js] >= 0) c.f_next[c.wqt[js]] = f; else c.wqh[js] = f;
+    c.wqt[js] = f;
+  }
+  S.prev_arrival = q.a;
+  S.n_routed++;
+}
+
+// Reads request i's scalars (control thread).
+__device__ __forceinline__ void load_request(const SimCtx& c, ReqState& q, int64_t i) {
+  const int64_t o0 = c.d->offsets[i], o1 = c.d->offsets[i + 1];
+  const int O = c.d->out_len[i];
+  const int64_t L = o1 - o0;
+  q.off0 = o0;
+  q.rel = c.d->release[i];
+  q.O = O;
+  q.nb = (L >> 4) > 0x7FFFFFFF ? 0x7FFFFFFF : (int)(L >> 4);
+  q.nbt = (int)((L + 15) >> 4);
+  q.blk = (L + O + 15) >> 4;
+  q.phase = 0;
+}
+
+// Algorithm 1: the router parameters of the current regime (control thread).
+__device__ __forceinline__ void regime_params(const SimCtx& c, ReqState& q) {
+  float tau = c.d->tau, om = c.d->omega;
+  if (c.d->policy == RS_POLICY_LOADBAL) {
+    tau = 0.0f;
+    om = 0.0f;
+  } else if (c.d->controller && c.S->regime > 0) {
+    tau = c.L->mc.regime_tau[c.S->regime];
+    om = c.L->mc.regime_omega[c.S->regime];
+  }
+  q.tau = tau;
+  q.omega = om;
+}
+
+// Block hashes of a request into a staging buffer (lanes of one warp).
+__device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q, uint64_t* dst,
+                                             int lane) {
+  if (q.nb > (int)c.L->g.K) return;
+  const uint64_t* src = c.d->hashes + (q.off0 >> 4);
+  for (int k = lane; k < q.nb; k += 32) dst[k] = __ldg(src + k);
 }
 
 __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
@@ -483,21 +604,25 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
   const SimDesc d = descs[sid];
   const int W = L.mc.W;
   const ModelConsts& mc = L.mc;
-  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax);
+  const int nft = ftab_size(mc.cap);
+  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax, nft);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   SimCtx c;
   c.S = &S;
   c.d = &d;
   c.b = &b;
   c.L = &L;
   c.sid = sid;
+  c.ftab = reinterpret_cast<double*>(smem + lay.ftab);
+  c.f_oitl = reinterpret_cast<double*>(smem + lay.f_oitl);
   c.f_a = reinterpret_cast<double*>(smem + lay.f_a);
   c.f_o = reinterpret_cast<double*>(smem + lay.f_o);
-  c.h_t = reinterpret_cast<double*>(smem + lay.h_t);
-  c.hbuf = reinterpret_cast<uint64_t*>(smem + lay.hbuf);
+  c.h_k = reinterpret_cast<uint64_t*>(smem + lay.h_k);
+  c.hbuf[0] = reinterpret_cast<uint64_t*>(smem + lay.hbuf0);
+  c.hbuf[1] = reinterpret_cast<uint64_t*>(smem + lay.hbuf1);
   c.f_req = reinterpret_cast<int32_t*>(smem + lay.f_req);
   c.f_worker = reinterpret_cast<int32_t*>(smem + lay.f_worker);
   c.f_blk = reinterpret_cast<int32_t*>(smem + lay.f_blk);
-  c.f_O = reinterpret_cast<int32_t*>(smem + lay.f_O);
   c.f_next = reinterpret_cast<int32_t*>(smem + lay.f_next);
   c.h_f = reinterpret_cast<int32_t*>(smem + lay.h_f);
   c.freestk = reinterpret_cast<int32_t*>(smem + lay.freestk);
@@ -537,6 +662,7 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
     for (size_t s = threadIdx.x; s < nsl / 4; s += NT_SIM)
       reinterpret_cast<uint4*>(st)[s] = make_uint4(STAMP_NONE, STAMP_NONE, STAMP_NONE, STAMP_NONE);
     for (uint32_t s = threadIdx.x; s <= lay.dupmask; s += NT_SIM) c.sc.dupset[s] = 0ull;
+    for (int q = 1 + threadIdx.x; q < nft; q += NT_SIM) c.ftab[q] = latency_f(mc, q);
     for (int p = threadIdx.x; p < d.C; p += NT_SIM) c.freestk[p] = d.C - 1 - p;
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
       c.wmeta[j] = CacheMeta{0u, 0u, 0u, 0u};
@@ -546,155 +672,163 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
       c.wqt[j] = -1;
     }
     if (threadIdx.x == 0) {
-      SimScalars z;
-      memset(&z, 0, sizeof z);
-      S = z;
+      memset(&S, 0, sizeof(SimScalars));
       S.min_ft = __longlong_as_double(0x7FF0000000000000ll);
       S.next_tick = 1;
+      S.tick_t = mc.dt;
       S.nfree = d.C;
-      if (d.n_req > 0) {
-        S.noff0 = d.offsets[0];
-        S.noff1 = d.offsets[1];
-        S.rel_next = d.release[0];
-        S.nO = d.out_len[0];
-      }
     }
     __syncthreads();
   }
 
   const int64_t n = d.n_req;
-  for (int64_t i = 0; i < n; i++) {
-    if (threadIdx.x == 0) {
-      S.off0 = S.noff0;
-      S.off1 = S.noff1;
-      S.rel = S.rel_next;
-      S.O = S.nO;
-      S.phase = 0;
+  // ---- prologue: request 0's arrival and hashes
+  if (n > 0) {
+    if (threadIdx.x == CTL) {
+      load_request(c, S.q[0], 0);
+      S.evres = events_advance(c, S.q[0]);
     }
     __syncthreads();
-    // ---- completions and controller samples up to the arrival
+    if (warp == NT_SIM / 32 - 1) stage_hashes(c, S.q[0], c.hbuf[0], lane);
+  }
+  for (int64_t i = 0; i < n; i++) {
+    const int p = (int)(i & 1);
+    // ---- controller samples that need the CTA, before request i arrives
     for (;;) {
-      if (threadIdx.x == 0) S.evres = events_advance(c);
       __syncthreads();
       if (S.evres == 0) break;
       tick_cta(c);
+      if (threadIdx.x == CTL) S.evres = events_advance(c, S.q[p]);
     }
     if (S.status != RS_OK) break;
-    // ---- prefetch the next request's scalars
-    if (threadIdx.x == 32 && i + 1 < n) {
-      S.noff0 = d.offsets[i + 1];
-      S.noff1 = d.offsets[i + 2];
-      S.rel_next = d.release[i + 1];
-      S.nO = d.out_len[i + 1];
-    }
-    const int64_t Lp = S.off1 - S.off0;
-    const int64_t nb64 = Lp >> 4;
-    if (nb64 > (int64_t)L.g.K) {
+    const int nb = S.q[p].nb;
+    if (nb > (int)L.g.K) {
       if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
       break;
     }
-    const int nb = (int)nb64;
-    const int nbt = (int)((Lp + 15) >> 4);
-    const int64_t blk = (Lp + S.O + 15) >> 4;
-    const double a = S.a_cur;
+    const int nbt = S.q[p].nbt;
+    const uint64_t* hb = c.hbuf[p];
     const int64_t row = d.rec_base + i;
-    // ---- stage the prompt's block hashes; regime parameters (Algorithm 1)
-    const uint64_t* hsrc = d.hashes + (S.off0 >> 4);
-    for (int k = threadIdx.x; k < nb; k += NT_SIM) c.hbuf[k] = __ldg(hsrc + k);
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
       c.wm[j] = nb;
       c.wopen[j] = j;
     }
-    if (threadIdx.x == 0) {
-      S.nopen = W;
-      float tau = d.tau, om = d.omega;
-      if (d.policy == RS_POLICY_LOADBAL) {
-        tau = 0.0f;
-        om = 0.0f;
-      } else if (d.controller && S.regime > 0) {
-        tau = mc.regime_tau[S.regime];
-        om = mc.regime_omega[S.regime];
-      }
-      S.tau_cur = tau;
-      S.omega_cur = om;
-    }
+    if (threadIdx.x == 0) S.nopen = W;
+    if (threadIdx.x == CTL) regime_params(c, S.q[p]);
     __syncthreads();
     // ---- cached prefix on every worker
-    probe_prefixes(c, nb);
-    // ---- Eq. (1) costs and the frozen loads of Eq. (12)
-    for (int j = threadIdx.x; j < W; j += NT_SIM) {
-      const float cj = router_cost(S.omega_cur, (int64_t)nbt - c.wm[j], c.wA[j]);
-      c.wcost[j] = cj;
-      const int nf = min(c.winserv[j] + 1, mc.cap - 1);
-      b.rec.n_frozen[row * W + j] = (uint16_t)nf;
-      b.rec.prefix[row * W + j] = (uint16_t)c.wm[j];
-      if (mc.write_cost) b.rec.cost[row * W + j] = cj;
-    }
-    __syncthreads();
-    // ---- Eq. (2) choice
-    if (threadIdx.x == 0) {
-      for (int j = 0; j < W; j++) S.probe_blocks += min(c.wm[j] + 1, nb);
-      S.hashed_blocks += nb;
-      const float tau = S.tau_cur;
-      const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
-      int nbd = 0;
-      S.jstar = select_worker(c.wcost, W, tau, u24, &nbd);
-      if (W >= 2) {
-        const int bmin = argmin_lowest(c.wcost, W);
-        float c2 = __int_as_float(0x7F800000);
-        for (int j = 0; j < W; j++)
-          if (j != bmin && c.wcost[j] < c2) c2 = c.wcost[j];
-        const double diff = (double)c2 - (double)c.wcost[bmin];
-        if (diff <= 1e-6 * fabs((double)c2)) S.near_ties++;
-        if (c2 == c.wcost[bmin]) S.exact_ties++;
+    probe_prefixes(c, hb, nb);
+    // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
+    if (warp == 0) {
+      const float om = S.q[p].omega, tau = S.q[p].tau;
+      for (int j = lane; j < W; j += 32) {
+        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+        c.wcost[j] = cj;
+        b.rec.n_frozen[row * W + j] = (uint16_t)min(c.winserv[j] + 1, mc.cap - 1);
+        b.rec.prefix[row * W + j] = (uint16_t)c.wm[j];
+        if (mc.write_cost) b.rec.cost[row * W + j] = cj;
       }
-      if (tau > 0.0f) {
-        S.sampled++;
-        S.near_bd += nbd;
+      __syncwarp();
+      if (lane == 0) {
+        const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
+        int nbd = 0;
+        S.jstar = select_worker(c.wcost, W, tau, u24, &nbd);
+        if (tau > 0.0f) {
+          S.sampled++;
+          S.near_bd += nbd;
+        }
+      }
+    } else if (warp == 1 && lane == 0) {
+      // statistics of the decision, beside the choice: work done by the probe,
+      // and whether the two lowest Eq. (1) costs tie within 1e-6 (recomputed
+      // from the probe results so as not to wait for warp 0)
+      int64_t pb = 0;
+      for (int j = 0; j < W; j++) pb += min(c.wm[j] + 1, nb);
+      S.probe_blocks += pb;
+      S.hashed_blocks += nb;
+      if (W >= 2) {
+        const float om = S.q[p].omega;
+        int bmin = 0;
+        float c1 = router_cost(om, (int64_t)nbt - c.wm[0], c.wA[0]);
+        for (int j = 1; j < W; j++) {
+          const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+          if (cj < c1) { c1 = cj; bmin = j; }
+        }
+        float c2 = __int_as_float(0x7F800000);
+        for (int j = 0; j < W; j++) {
+          const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+          if (j != bmin && cj < c2) c2 = cj;
+        }
+        const double diff = (double)c2 - (double)c1;
+        if (diff <= 1e-6 * fabs((double)c2)) S.near_ties++;
+        if (c2 == c1) S.exact_ties++;
       }
     }
     __syncthreads();
     const int js = S.jstar;
-    // ---- the chosen worker's LRU cache
-    update_chosen(c, js, nb);
-    if (S.status != RS_OK) break;
-    // ---- load, records, service start or FIFO queue
-    if (threadIdx.x == 0) {
-      const int f = c.freestk[--S.nfree];
-      c.f_req[f] = (int32_t)i;
-      c.f_worker[f] = js;
-      c.f_blk[f] = (int32_t)blk;
-      c.f_O[f] = S.O;
-      c.f_a[f] = a;
-      c.f_o[f] = nbt > 0 ? __ddiv_rn((double)c.wm[js], (double)nbt) : 0.0;
-      c.f_next[f] = -1;
-      c.wA[js] += blk;
-      S.in_flight++;
-      S.hit_blocks += c.wm[js];
-      b.rec.worker[row] = js;
-      b.rec.arrival[row] = a;
-      b.rec.nbt[row] = nbt;
-      if (c.winserv[js] < mc.cap - 1) {
-        start_service(c, f, js, a);
-      } else {
-        if (c.wqt[js] >= 0) c.f_next[c.wqt[js]] = f; else c.wqh[js] = f;
-        c.wqt[js] = f;
+    if (warp < NT_SIM / 32 - 1) {
+      // ---- the chosen worker's LRU cache (warps 0-6)
+      update_chosen(c, hb, js, nb);
+    } else {
+      // ---- control warp: request i's load and latency; request i+1's arrival
+      ReqState& nq = S.q[p ^ 1];
+      if (lane == 0) {
+        book_request(c, S.q[p], i);
+        if (i + 1 < n) load_request(c, nq, i + 1);
       }
-      S.prev_arrival = a;
-      S.n_routed++;
-    }
-    __syncthreads();
-  }
-  // ---- drain: remaining completions start the queued requests
-  if (threadIdx.x == 0 && S.status == RS_OK) {
-    while (S.nheap > 0) {
-      double t;
-      int f;
-      heap_pop(c, &t, &f);
-      complete(c, f, t);
+      __syncwarp();
+      if (i + 1 < n) {
+        stage_hashes(c, nq, c.hbuf[p ^ 1], lane);
+        if (lane == 0) S.evres = events_advance(c, nq);
+      }
     }
   }
   __syncthreads();
+  // ---- drain: remaining completions start the queued requests
+  if (threadIdx.x == CTL && S.status == RS_OK) {
+    while (S.nheap > 0) {
+      uint64_t k;
+      int f;
+      heap_pop(c, &k, &f);
+      complete(c, f, tval(k));
+    }
+  }
+  __syncthreads();
+  {
+    double st = 0.0, se = 0.0, mk = 0.0;
+    if (S.status == RS_OK)
+      for (int64_t q = threadIdx.x; q < S.n_routed; q += NT_SIM) {
+        const int64_t row = d.rec_base + q;
+        const double ct = b.rec.completion[row];
+        st = __dadd_rn(st, b.rec.ttft[row]);
+        se = __dadd_rn(se, __dsub_rn(ct, b.rec.arrival[row]));
+        mk = fmax(mk, ct);
+      }
+    for (int o = 16; o > 0; o >>= 1) {
+      st = __dadd_rn(st, __shfl_xor_sync(FULL_MASK, st, o));
+      se = __dadd_rn(se, __shfl_xor_sync(FULL_MASK, se, o));
+      mk = fmax(mk, __shfl_xor_sync(FULL_MASK, mk, o));
+    }
+    __shared__ double red3[3][NT_SIM / 32];
+    if (lane == 0) {
+      red3[0][warp] = st;
+      red3[1][warp] = se;
+      red3[2][warp] = mk;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      double a0 = 0.0, a1 = 0.0, a2 = 0.0;
+      for (int w = 0; w < NT_SIM / 32; w++) {
+        a0 = __dadd_rn(a0, red3[0][w]);
+        a1 = __dadd_rn(a1, red3[1][w]);
+        a2 = fmax(a2, red3[2][w]);
+      }
+      S.sum_ttft = a0;
+      S.sum_e2e = a1;
+      S.makespan = a2;
+    }
+    __syncthreads();
+  }
   if (threadIdx.x == 0) {
     rs_replica_result r;
     memset(&r, 0, sizeof r);
@@ -704,8 +838,6 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
     r.sum_ttft = S.sum_ttft;
     r.sum_e2e = S.sum_e2e;
     r.makespan = S.makespan;
-    r.poa_total = 0.0;
-    r.n_windows = 0;
     r.near_ties = S.near_ties;
     r.exact_ties = S.exact_ties;
     r.sampled = S.sampled;
@@ -733,7 +865,7 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st) {
   if (L.nsim <= 0) return cudaSuccess;
-  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax);
+  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap);
   cudaError_t e = cudaFuncSetAttribute(k_sim, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
