@@ -132,14 +132,18 @@ struct SimCtx {
   int sid;
   double *f_a, *f_o, *ftab, *f_oitl;
   uint64_t* h_k;
-  uint64_t* hbuf[2];
+  uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
   int32_t *winserv, *wqh, *wqt, *wm, *wopen;
   int64_t* wA;
   float* wcost;
   UpdateScratch sc;
-  double *pend_ft[2], *pend_tt[2], *pend_win;
+  double *pend_ft0, *pend_tt0, *pend_ft1, *pend_tt1, *pend_win;
+
+  __device__ __forceinline__ uint64_t* hbuf(int p) const { return p ? hbuf1 : hbuf0; }
+  __device__ __forceinline__ double* pend_ft(int p) const { return p ? pend_ft1 : pend_ft0; }
+  __device__ __forceinline__ double* pend_tt(int p) const { return p ? pend_tt1 : pend_tt0; }
 
   __device__ __forceinline__ TableView table(int j) const {
     TableView t;
@@ -232,8 +236,8 @@ __device__ __forceinline__ void start_service(SimCtx& c, int f, int j, double t)
   heap_push(c, tkey(ct), f);
   if (c.d->controller) {
     const int cur = S.pend_cur;
-    c.pend_ft[cur][S.np] = ft;
-    c.pend_tt[cur][S.np] = tt;
+    c.pend_ft(cur)[S.np] = ft;
+    c.pend_tt(cur)[S.np] = tt;
     S.np++;
     if (tkey(ft) < tkey(S.min_ft)) S.min_ft = ft;
   }
@@ -366,10 +370,10 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
   const double tt = S.tick_t;
   const int cur = S.pend_cur;
   const int64_t np = S.np;
-  const double* sft = c.pend_ft[cur];
-  const double* stt = c.pend_tt[cur];
-  double* dft = c.pend_ft[cur ^ 1];
-  double* dtt = c.pend_tt[cur ^ 1];
+  const double* sft = c.pend_ft(cur);
+  const double* stt = c.pend_tt(cur);
+  double* dft = c.pend_ft(cur ^ 1);
+  double* dtt = c.pend_tt(cur ^ 1);
   int64_t nkeep = 0, nwin = 0;
   uint64_t mft = KEY_INF;
   const uint64_t ktt = tkey(tt);
@@ -596,7 +600,7 @@ __device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q,
   for (int k = lane; k < q.nb; k += 32) dst[k] = __ldg(src + k);
 }
 
-__global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
+__global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ SimScalars S;
@@ -618,8 +622,8 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
   c.f_a = reinterpret_cast<double*>(smem + lay.f_a);
   c.f_o = reinterpret_cast<double*>(smem + lay.f_o);
   c.h_k = reinterpret_cast<uint64_t*>(smem + lay.h_k);
-  c.hbuf[0] = reinterpret_cast<uint64_t*>(smem + lay.hbuf0);
-  c.hbuf[1] = reinterpret_cast<uint64_t*>(smem + lay.hbuf1);
+  c.hbuf0 = reinterpret_cast<uint64_t*>(smem + lay.hbuf0);
+  c.hbuf1 = reinterpret_cast<uint64_t*>(smem + lay.hbuf1);
   c.f_req = reinterpret_cast<int32_t*>(smem + lay.f_req);
   c.f_worker = reinterpret_cast<int32_t*>(smem + lay.f_worker);
   c.f_blk = reinterpret_cast<int32_t*>(smem + lay.f_blk);
@@ -646,10 +650,10 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
   c.sc.dupset = reinterpret_cast<uint64_t*>(smem + lay.dupset);
   c.sc.dupmask = lay.dupmask;
   double* pend = b.pend + (size_t)sid * 5 * b.pend_cap;
-  c.pend_ft[0] = pend;
-  c.pend_tt[0] = pend + b.pend_cap;
-  c.pend_ft[1] = pend + 2 * b.pend_cap;
-  c.pend_tt[1] = pend + 3 * b.pend_cap;
+  c.pend_ft0 = pend;
+  c.pend_tt0 = pend + b.pend_cap;
+  c.pend_ft1 = pend + 2 * b.pend_cap;
+  c.pend_tt1 = pend + 3 * b.pend_cap;
   c.pend_win = pend + 4 * b.pend_cap;
 
   // ---- initial state: empty caches, idle workers
@@ -689,7 +693,7 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
       S.evres = events_advance(c, S.q[0]);
     }
     __syncthreads();
-    if (warp == NT_SIM / 32 - 1) stage_hashes(c, S.q[0], c.hbuf[0], lane);
+    if (warp == NT_SIM / 32 - 1) stage_hashes(c, S.q[0], c.hbuf0, lane);
   }
   for (int64_t i = 0; i < n; i++) {
     const int p = (int)(i & 1);
@@ -707,7 +711,7 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
       break;
     }
     const int nbt = S.q[p].nbt;
-    const uint64_t* hb = c.hbuf[p];
+    const uint64_t* hb = c.hbuf(p);
     const int64_t row = d.rec_base + i;
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
       c.wm[j] = nb;
@@ -778,7 +782,7 @@ __global__ void __launch_bounds__(NT_SIM) k_sim(const SimDesc* __restrict__ desc
       }
       __syncwarp();
       if (i + 1 < n) {
-        stage_hashes(c, nq, c.hbuf[p ^ 1], lane);
+        stage_hashes(c, nq, c.hbuf(p ^ 1), lane);
         if (lane == 0) S.evres = events_advance(c, nq);
       }
     }
