@@ -49,9 +49,9 @@ def _dist():
     return ws, rank, local
 
 
-def _plan(rank: int):
+def _plan(rank: int, n_req=None):
     from paper_2606_17081_gb300 import workloads as wk
-    p = wk.plan(WORKLOAD)
+    p = wk.plan(WORKLOAD, n_req=n_req)
     if rank:
         p.trace_seeds = [s + 1000 * rank for s in p.trace_seeds]
         for r in p.replicas:
@@ -152,7 +152,7 @@ def run_gpu(args):
     torch.cuda.set_device(local)
     if ws > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    p = _plan(rank)
+    p = _plan(rank, args.n_req)
     traces = p.traces()
     ctx = rs.Context(W=p.W, K=p.K)
     dev = [rs.device_trace(t) for t in traces]
@@ -343,6 +343,8 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--n-req", type=int, default=None,
+                    help="truncate every replica's trace (profiling of a small case)")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

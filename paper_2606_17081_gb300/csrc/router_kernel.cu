@@ -44,6 +44,7 @@ __global__ void __launch_bounds__(NT_SIM) k_route_batch(
   CacheMeta* meta = reinterpret_cast<CacheMeta*>(take(sizeof(CacheMeta) * (size_t)W));
   sc.slot = reinterpret_cast<uint32_t*>(take(4 * nb_cap));
   sc.pst = reinterpret_cast<uint32_t*>(take(4 * nb_cap));
+  sc.fslot = reinterpret_cast<uint32_t*>(take(4 * nb_cap));
   sc.vslot = reinterpret_cast<uint32_t*>(take(8 * nb_cap));
   sc.vt = reinterpret_cast<uint32_t*>(take(8 * nb_cap));
   sc.owner = reinterpret_cast<int32_t*>(take(8 * nb_cap));
@@ -173,7 +174,7 @@ size_t router_smem(int W, int nbmax) {
   while (dup < 2 * nb) dup <<= 1;
   auto r16 = [](size_t x) { return (x + 15) & ~(size_t)15; };
   return r16(8 * nb) + r16(8 * dup) + r16(8 * (size_t)W) + r16(sizeof(CacheMeta) * (size_t)W) +
-         2 * r16(4 * nb) + 4 * r16(8 * nb) + 3 * r16(4 * (size_t)W) + 2 * r16(nb) + r16(2 * nb);
+         3 * r16(4 * nb) + 4 * r16(8 * nb) + 3 * r16(4 * (size_t)W) + 2 * r16(nb) + r16(2 * nb);
 }
 
 cudaError_t launch_route_batch(const RouterState& s, int32_t instance, const int64_t* offsets,

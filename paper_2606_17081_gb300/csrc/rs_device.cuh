@@ -232,6 +232,39 @@ __device__ __forceinline__ uint32_t table_find(const TableView& t, uint64_t h, i
   return SLOT_NONE;
 }
 
+// Slot holding h, or SLOT_NONE; *free_slot = the first EMPTY or TOMB slot of
+// h's probe sequence (where an insert of h would go), with FREE_TOMB set when
+// that slot held a tombstone, or SLOT_NONE.
+constexpr uint32_t FREE_TOMB = 0x80000000u;
+__device__ __forceinline__ uint32_t table_find_free(const TableView& t, uint64_t h, int* err,
+                                                    uint32_t* free_slot) {
+  uint32_t b = home_bucket(h, t.bmask);
+  uint32_t fr = SLOT_NONE;
+  for (uint32_t it = 0; it <= t.bmask; it++) {
+    const ulonglong2 x = ld_keys2(t.keys + 4 * (size_t)b);
+    const ulonglong2 y = ld_keys2(t.keys + 4 * (size_t)b + 2);
+    const uint64_t v[4] = {x.x, x.y, y.x, y.y};
+    bool empty = false;
+#pragma unroll
+    for (int q = 0; q < 4; q++) {
+      if (v[q] == h) {
+        *free_slot = fr;
+        return 4 * b + q;
+      }
+      if (v[q] < 2 && fr == SLOT_NONE) fr = (4 * b + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
+      empty |= v[q] == KEY_EMPTY;
+    }
+    if (empty) {
+      *free_slot = fr;
+      return SLOT_NONE;
+    }
+    b = (b + 1) & t.bmask;
+  }
+  *err = 1;
+  *free_slot = SLOT_NONE;
+  return SLOT_NONE;
+}
+
 // Claims the first EMPTY or TOMB slot of h's probe sequence (h known absent;
 // other threads of the CTA may insert concurrently).  *was_tomb reports a
 // reclaimed tombstone.
@@ -262,6 +295,7 @@ __device__ __forceinline__ uint32_t table_insert(const TableView& t, uint64_t h,
 struct UpdateScratch {
   uint32_t* slot;     // [nbmax] slot per request block
   uint32_t* pst;      // [nbmax] stamp of present blocks
+  uint32_t* fslot;    // [nbmax] insert position seen by the lookup (FREE_TOMB flag) or SLOT_NONE
   uint8_t* kind;      // [nbmax] 1 = insert, 0 = touch
   uint8_t* evk;       // [nbmax] present block evicted before its turn
   uint32_t* vslot;    // [2*nbmax] first live log entries: slot
@@ -339,6 +373,24 @@ __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* met
   grp_bar<NT>();
 }
 
+// Duplicate detector of one request's block hashes: an open-addressing set in
+// shared memory; returns the slot this thread claimed (to clear it later), or
+// -1, and sets *dup when h was already there.
+__device__ __forceinline__ int32_t dup_claim(UpdateScratch& sc, uint64_t h, int* dup) {
+  uint32_t d = (uint32_t)(h ^ (h >> 29)) & sc.dupmask;
+  for (uint32_t it = 0; it <= sc.dupmask; it++) {
+    const unsigned long long prev = atomicCAS(
+        reinterpret_cast<unsigned long long*>(sc.dupset + d), 0ull, (unsigned long long)h);
+    if (prev == 0ull) return (int32_t)d;
+    if (prev == h) {
+      *dup = 1;
+      return -1;
+    }
+    d = (d + 1) & sc.dupmask;
+  }
+  return -1;
+}
+
 // Resets the shared scalars of one cache update.
 __device__ __forceinline__ void update_reset(UpdateShared* us) {
   us->n_absent = 0;
@@ -355,7 +407,7 @@ __device__ __forceinline__ void update_reset(UpdateShared* us) {
 // fills slot[] and pst[]; counts absent blocks; detects duplicate hashes
 // within the request (a shared-memory open-addressing set; each thread clears
 // the slot it claimed).  us must be reset before the call.
-template <int NT>
+template <int NT, bool DETECT_DUP = true>
 __device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint64_t* hbuf, int nb,
                                  UpdateScratch& sc, UpdateShared* us,
                                  unsigned long long* probes) {
@@ -363,8 +415,10 @@ __device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint6
   uint32_t pmin = STAMP_NONE;
   for (int k = threadIdx.x; k < nb; k += NT) {
     const uint64_t h = hbuf[k];
-    const uint32_t sl = table_find(t, h, &err);
+    uint32_t fr;
+    const uint32_t sl = table_find_free(t, h, &err, &fr);
     sc.slot[k] = sl;
+    sc.fslot[k] = fr;
     uint32_t st = STAMP_NONE;
     if (sl != SLOT_NONE) {
       st = __ldcg(t.stamp + sl);
@@ -374,16 +428,7 @@ __device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint6
     }
     sc.pst[k] = st;
     sc.evk[k] = 0;
-    uint32_t d = (uint32_t)(h ^ (h >> 29)) & sc.dupmask;
-    int32_t claimed = -1;
-    for (uint32_t it = 0; it <= sc.dupmask; it++) {
-      const unsigned long long prev = atomicCAS(
-          reinterpret_cast<unsigned long long*>(sc.dupset + d), 0ull, (unsigned long long)h);
-      if (prev == 0ull) { claimed = (int32_t)d; break; }
-      if (prev == h) { dup = 1; break; }
-      d = (d + 1) & sc.dupmask;
-    }
-    sc.owner[k] = claimed;
+    if (DETECT_DUP) sc.owner[k] = dup_claim(sc, h, &dup);
   }
   nabs = __reduce_add_sync(FULL_MASK, (unsigned)nabs);
   pmin = __reduce_min_sync(FULL_MASK, pmin);
@@ -395,8 +440,40 @@ __device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint6
   if (dup) us->dup = 1;
   if (threadIdx.x == 0) atomicAdd(probes, (unsigned long long)nb);
   grp_bar<NT>();
-  for (int k = threadIdx.x; k < nb; k += NT)
-    if (sc.owner[k] >= 0) sc.dupset[sc.owner[k]] = 0ull;
+  if (DETECT_DUP)
+    for (int k = threadIdx.x; k < nb; k += NT)
+      if (sc.owner[k] >= 0) sc.dupset[sc.owner[k]] = 0ull;
+}
+
+// The chosen worker's lookup from slots captured by the probe (no table
+// reads): stamps of present blocks, absent count, insert positions.
+template <int NT>
+__device__ __forceinline__ void cache_lookup_captured(const TableView& t, const uint32_t* pslot,
+                                                      const uint32_t* pfree, int nb,
+                                                      UpdateScratch& sc, UpdateShared* us) {
+  int nabs = 0;
+  uint32_t pmin = STAMP_NONE;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const uint32_t sl = pslot[k];
+    sc.slot[k] = sl;
+    sc.fslot[k] = pfree[k];
+    sc.evk[k] = 0;
+    uint32_t st = STAMP_NONE;
+    if (sl != SLOT_NONE) {
+      st = __ldcg(t.stamp + sl);
+      pmin = min(pmin, st);
+    } else {
+      nabs++;
+    }
+    sc.pst[k] = st;
+  }
+  nabs = __reduce_add_sync(FULL_MASK, (unsigned)nabs);
+  pmin = __reduce_min_sync(FULL_MASK, pmin);
+  if ((threadIdx.x & 31) == 0) {
+    if (nabs) atomicAdd(&us->n_absent, nabs);
+    if (pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  }
+  grp_bar<NT>();
 }
 
 // Gathers live log entries starting at meta->head until `want` are held
@@ -540,7 +617,18 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
     uint32_t sl = sc.slot[k];
     if (sc.kind[k]) {
       int wt = 0;
-      sl = table_insert(t, hbuf[k], &wt, &err);
+      const uint32_t fr = sc.fslot[k];
+      sl = SLOT_NONE;
+      if (fr != SLOT_NONE) {   // the position the lookup saw free: one CAS
+        const uint32_t x = fr & ~FREE_TOMB;
+        const unsigned long long want = (fr & FREE_TOMB) ? KEY_TOMB : KEY_EMPTY;
+        if (atomicCAS(reinterpret_cast<unsigned long long*>(t.keys + x), want,
+                      (unsigned long long)hbuf[k]) == want) {
+          sl = x;
+          wt = (fr & FREE_TOMB) != 0;
+        }
+      }
+      if (sl == SLOT_NONE) sl = table_insert(t, hbuf[k], &wt, &err);
       nins++;
       recl += wt;
       sc.slot[k] = sl;

@@ -28,13 +28,15 @@ namespace rs {
 constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (warps 0-6)
 constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
 constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
+constexpr int PROBE_CAP = 2048;          // W * nb up to which the probe captures every slot
+constexpr int PROBE_ILP = 4;             // lookups a thread keeps in flight
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct SimLayout {
   size_t ftab, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
-  size_t slot, pst, vslot, vt;
+  size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
   size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen;
   size_t kind, evk, touched;
   size_t total;
@@ -73,6 +75,10 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(victim, 4 * nv, 4)
   TAKE(slot, 4 * nb, 4)
   TAKE(pst, 4 * nb, 4)
+  TAKE(fslot, 4 * nb, 4)
+  TAKE(pslot, 4 * (size_t)PROBE_CAP, 16)
+  TAKE(pfree, 4 * (size_t)PROBE_CAP, 16)
+  TAKE(dclaim, 4 * nb, 4)
   TAKE(vslot, 4 * nv, 4)
   TAKE(vt, 4 * nv, 4)
   TAKE(wmeta, sizeof(CacheMeta) * (size_t)W, 16)
@@ -115,7 +121,7 @@ struct SimScalars {
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild;
+  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, full;
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
@@ -135,7 +141,8 @@ struct SimCtx {
   uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
-  int32_t *winserv, *wqh, *wqt, *wm, *wopen;
+  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *dclaim;
+  uint32_t *pslot, *pfree;
   int64_t* wA;
   float* wcost;
   UpdateScratch sc;
@@ -501,6 +508,72 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
   if (err) S.status = RS_ERR_TIMEOUT;
 }
 
+// The same m_j with every (worker, block) pair looked up at once (W nb <=
+// PROBE_CAP): each thread issues the first-bucket loads of PROBE_ILP pairs
+// before resolving them, and the slot found (or the first free slot of the
+// probe path) is kept for the chosen worker's update.
+__device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int nb) {
+  SimScalars& S = *c.S;
+  const int W = c.L->mc.W;
+  const int total = W * nb;
+  int err = 0;
+  for (int base = 0; base < total; base += NT_SIM * PROBE_ILP) {   // uniform
+    int jj[PROBE_ILP], kk[PROBE_ILP];
+    uint64_t hv[PROBE_ILP];
+    ulonglong2 x[PROBE_ILP], y[PROBE_ILP];
+    uint32_t bk[PROBE_ILP];
+#pragma unroll
+    for (int r = 0; r < PROBE_ILP; r++) {
+      const int it = base + r * NT_SIM + threadIdx.x;
+      jj[r] = -1;
+      if (it < total) {
+        const int j = it / nb;
+        jj[r] = j;
+        kk[r] = it - j * nb;
+        hv[r] = hbuf[kk[r]];
+        const TableView t = c.table(j);
+        bk[r] = home_bucket(hv[r], t.bmask);
+        x[r] = ld_keys2(t.keys + 4 * (size_t)bk[r]);
+        y[r] = ld_keys2(t.keys + 4 * (size_t)bk[r] + 2);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < PROBE_ILP; r++) {
+      const int it = base + r * NT_SIM + threadIdx.x;
+      int miss = 0x7FFFFFFF;
+      if (jj[r] >= 0) {
+        const uint64_t v[4] = {x[r].x, x[r].y, y[r].x, y[r].y};
+        uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
+        bool done = false;
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+          if (!done && v[q] == hv[r]) { sl = 4 * bk[r] + q; done = true; }
+          if (!done && v[q] < 2 && fr == SLOT_NONE)
+            fr = (4 * bk[r] + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
+        }
+        const bool empty = v[0] == KEY_EMPTY || v[1] == KEY_EMPTY || v[2] == KEY_EMPTY ||
+                           v[3] == KEY_EMPTY;
+        if (!done && !empty) {
+          // bucket full of other keys: continue along the probe sequence
+          uint32_t fr2;
+          sl = table_find_free(c.table(jj[r]), hv[r], &err, &fr2);
+          if (fr == SLOT_NONE) fr = fr2;
+        }
+        c.pslot[it] = sl;
+        c.pfree[it] = fr;
+        if (sl == SLOT_NONE) miss = kk[r];
+      }
+      const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
+      const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
+      if (jj[r] >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
+        atomicMin(&c.wm[jj[r]], m);
+    }
+  }
+  if (threadIdx.x == 0) S.probes += (unsigned long long)total;
+  if (err) S.status = RS_ERR_TIMEOUT;
+  __syncthreads();
+}
+
 // Cache update of the chosen worker (update group, warps 0-6).
 __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb) {
   SimScalars& S = *c.S;
@@ -510,20 +583,23 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
   if (threadIdx.x == 0) {
     const uint64_t span = (uint64_t)meta->T - meta->head + (uint64_t)nb;
     S.rebuild = span > g.R || meta->tombs > g.slots / 4 || (uint64_t)meta->T + nb > STAMP_LIMIT;
-    update_reset(&S.us);
-    S.us.err = 0;
   }
-  grp_bar<NT_UPD>();
-  if (S.rebuild) {
-    cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
-    if (threadIdx.x == 0) S.rebuilds++;
-  }
-  cache_lookup_all<NT_UPD>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
+  for (int k = threadIdx.x; k < nb; k += NT_UPD)   // release the duplicate detector
+    if (c.dclaim[k] >= 0) c.sc.dupset[c.dclaim[k]] = 0ull;
   grp_bar<NT_UPD>();
   if (S.us.dup) {
     if (threadIdx.x == 0) S.status = RS_ERR_COLLISION;
     return;
   }
+  if (S.rebuild) {
+    cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
+    if (threadIdx.x == 0) S.rebuilds++;
+  }
+  if (S.full && !S.rebuild)
+    cache_lookup_captured<NT_UPD>(tv, c.pslot + (size_t)j * nb, c.pfree + (size_t)j * nb, nb,
+                                  c.sc, &S.us);
+  else
+    cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
   cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos);
   if (threadIdx.x == 0) {
     if (S.us.err) S.status = S.us.err;
@@ -640,6 +716,10 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   c.wcost = reinterpret_cast<float*>(smem + lay.wcost);
   c.sc.slot = reinterpret_cast<uint32_t*>(smem + lay.slot);
   c.sc.pst = reinterpret_cast<uint32_t*>(smem + lay.pst);
+  c.sc.fslot = reinterpret_cast<uint32_t*>(smem + lay.fslot);
+  c.pslot = reinterpret_cast<uint32_t*>(smem + lay.pslot);
+  c.pfree = reinterpret_cast<uint32_t*>(smem + lay.pfree);
+  c.dclaim = reinterpret_cast<int32_t*>(smem + lay.dclaim);
   c.sc.kind = smem + lay.kind;
   c.sc.evk = smem + lay.evk;
   c.sc.vslot = reinterpret_cast<uint32_t*>(smem + lay.vslot);
@@ -717,11 +797,17 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       c.wm[j] = nb;
       c.wopen[j] = j;
     }
-    if (threadIdx.x == 0) S.nopen = W;
+    if (threadIdx.x == 0) {
+      S.nopen = W;
+      S.full = W * nb <= PROBE_CAP;
+      update_reset(&S.us);
+      S.us.err = 0;
+    }
     if (threadIdx.x == CTL) regime_params(c, S.q[p]);
     __syncthreads();
     // ---- cached prefix on every worker
-    probe_prefixes(c, hb, nb);
+    if (W * nb <= PROBE_CAP) probe_full(c, hb, nb);
+    else probe_prefixes(c, hb, nb);
     // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
     if (warp == 0) {
       const float om = S.q[p].omega, tau = S.q[p].tau;
@@ -767,6 +853,12 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
         if (diff <= 1e-6 * fabs((double)c2)) S.near_ties++;
         if (c2 == c1) S.exact_ties++;
       }
+    } else if (warp >= 2 && warp < NT_SIM / 32 - 1) {
+      // two blocks of one prompt with the same chained hash (a 64-bit
+      // collision) would break the batched update: detect them here
+      int dup = 0;
+      for (int k = threadIdx.x - 64; k < nb; k += NT_SIM - 96) c.dclaim[k] = dup_claim(c.sc, hb[k], &dup);
+      if (dup) S.us.dup = 1;
     }
     __syncthreads();
     const int js = S.jstar;
