@@ -119,10 +119,10 @@ class ClockSampler:
 
 
 def _table_bytes(K: int) -> int:
-    """Device bytes of one worker's cache: keys + stamps (>= 2K slots) and the
-    stamp log (>= 4K entries)."""
-    slots = 1
-    while slots < 2 * K:
+    """Device bytes of one worker's cache: keys + stamps (>= 4K slots in
+    buckets of 8) and the stamp log (>= 4K entries)."""
+    slots = 8
+    while slots < 4 * K:
         slots <<= 1
     ring = 1
     while ring < 4 * K:

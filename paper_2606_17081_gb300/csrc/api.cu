@@ -35,7 +35,7 @@ struct rs_ctx {
   int32_t ninst = 0;
   DevBuf r_keys, r_stamp, r_log, r_tmp, r_meta, r_active, r_ord, r_status, r_hash, r_stats;
   // simulation scratch (grow-only)
-  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs;
+  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, dstat, wco;
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -149,12 +149,12 @@ namespace rs {
 TableGeom table_geom(int64_t K) {
   TableGeom g;
   g.K = (uint32_t)K;
-  uint64_t nbk = 1;
-  while (nbk * 4 < (uint64_t)(2 * K)) nbk <<= 1;
+  uint64_t nbk = 1;   // buckets of 8 keys, at least 4 K slots (live load <= 1/4)
+  while (nbk * 8 < (uint64_t)(4 * K)) nbk <<= 1;
   uint64_t R = 1;
   while (R < (uint64_t)(4 * K)) R <<= 1;
   g.bmask = (uint32_t)(nbk - 1);
-  g.slots = (size_t)(nbk * 4);
+  g.slots = (size_t)(nbk * 8);
   g.R = (size_t)R;
   g.rmask = (uint32_t)(R - 1);
   return g;
@@ -261,7 +261,7 @@ void route_destroy(rs_ctx* ctx) {
   DevBuf* all[] = {&ctx->r_keys, &ctx->r_stamp, &ctx->r_log, &ctx->r_tmp, &ctx->r_meta,
                    &ctx->r_active, &ctx->r_ord, &ctx->r_status, &ctx->r_hash, &ctx->r_stats,
                    &ctx->keys, &ctx->stamp, &ctx->log, &ctx->tmp, &ctx->pend, &ctx->meta_out,
-                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->rec_worker,
+                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
                    &ctx->rec_arrival, &ctx->rec_start, &ctx->rec_first, &ctx->rec_completion,
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
@@ -649,7 +649,14 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       (r = ensure(ctx, ctx->pend, nsim * 5 * (size_t)std::max<int64_t>(pend_cap, 1) * 8, "controller windows")) ||
       (r = ensure(ctx, ctx->meta_out, nsim * W * sizeof(CacheMeta), "cache meta")) ||
       (r = ensure(ctx, ctx->res, nsim * sizeof(rs_replica_result), "results")) ||
-      (r = ensure(ctx, ctx->desc, nsim * sizeof(SimDesc), "replica descriptors")))
+      (r = ensure(ctx, ctx->desc, nsim * sizeof(SimDesc), "replica descriptors")) ||
+      (r = ensure(ctx, ctx->dstat, (size_t)std::max<int64_t>(rows, 1) * 6 * sizeof(float),
+                  "decision statistics")))
+    return r;
+  // w_c * (m / nbt) table for prompts up to nbmax blocks (none beyond 2048)
+  const bool use_tab = nbmax <= 2048;
+  if (use_tab &&
+      (r = ensure(ctx, ctx->wco, (size_t)(nbmax + 1) * (nbmax + 2) * sizeof(double), "w_c o table")))
     return r;
   rs_records rec;
   const bool want_cost = records && records->cost;
@@ -693,6 +700,9 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   sb.meta_out = P<CacheMeta>(ctx->meta_out);
   sb.res = P<rs_replica_result>(ctx->res);
   sb.rec = rec;
+  sb.dstat = P<float>(ctx->dstat);
+  sb.wco_tab = use_tab ? P<double>(ctx->wco) : nullptr;
+  sb.wco_dim = (int)nbmax + 2;
   SimLaunch L;
   L.nsim = (int)nsim;
   L.nbmax = (int)nbmax;
@@ -700,8 +710,13 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   L.g = g;
   L.mc = ctx->mc;
   L.mc.write_cost = want_cost ? 1 : 0;
+  if (use_tab) {
+    CK(launch_wco_table(P<double>(ctx->wco), (int)nbmax, ctx->cfg.w_c, ctx->st), "table launch");
+    launches++;
+  }
   CK(launch_sim(P<SimDesc>(ctx->desc), sb, L, ctx->st), "simulation launch");
-  launches++;
+  CK(launch_decision_stats(P<SimDesc>(ctx->desc), sb, L, ctx->st), "statistics launch");
+  launches += 2;
   CK(cudaEventRecord(ctx->ev[2], ctx->st), "event");
   if (!(flags & RS_SIM_NO_POA)) {
     if ((r = run_poa(ctx, rec, probs, rows, win_slots, sb.res)) != RS_OK) return r;

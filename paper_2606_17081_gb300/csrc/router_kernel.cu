@@ -129,8 +129,7 @@ __global__ void __launch_bounds__(NT_SIM) k_route_batch(
     __syncthreads();
     if (threadIdx.x == 0) {
       const uint32_t u24 = tau > 0.0f ? draw_u24(seed, R.ordinal, (uint32_t)instance, TAG_ROUTE) : 0u;
-      int nbd;
-      R.jstar = select_worker(wcost, W, tau, u24, &nbd);
+      R.jstar = select_worker(wcost, W, tau, u24, nullptr);
       CacheMeta* mt = &meta[R.jstar];
       const uint64_t span = (uint64_t)mt->T - mt->head + (uint64_t)nb;
       R.rebuild = span > g.R || mt->tombs > g.slots / 8 || (uint64_t)mt->T + nb > STAMP_LIMIT;

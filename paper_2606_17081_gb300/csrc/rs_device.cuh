@@ -100,8 +100,10 @@ __device__ __forceinline__ float exp_sm(float x) {
 // ---------------------------------------------------------------- selection
 
 // Eq. (1) in fp32, rounded per operation: omega * b^prefill + b^active.
+// Both counts are below 2^31 (and exact in fp32 below 2^24), so they are
+// converted from 32-bit integers (the 64-bit conversion is a slower path).
 __device__ __forceinline__ float router_cost(float omega, int64_t bprefill, int64_t active) {
-  return __fadd_rn(__fmul_rn(omega, (float)bprefill), (float)active);
+  return __fadd_rn(__fmul_rn(omega, __int2float_rn((int)bprefill)), __int2float_rn((int)active));
 }
 
 // Lowest-index argmin over c[0..W) (one thread).
@@ -114,24 +116,35 @@ __device__ __forceinline__ int argmin_lowest(const float* c, int W) {
 
 // Eq. (2): tau == 0 -> argmin; tau > 0 -> the first j whose cumulative weight
 // (sequential fp32 sum in worker order) exceeds u * S.  One thread.
-// *near_bd = the scaled draw lies within 1e-6 S of a cumulative boundary.
+// ds (nullable) receives the draw's position for the near-boundary
+// statistic: {u S, S, largest cumulative weight <= u S (or NaN), smallest
+// cumulative weight > u S (or NaN)}.
 __device__ __forceinline__ int select_worker(const float* c, int W, float tau, uint32_t u24,
-                                             int* near_bd) {
+                                             float* ds) {
   const int b = argmin_lowest(c, W);
-  *near_bd = 0;
   if (tau == 0.0f) return b;
   const float cmin = c[b];
   float S = 0.0f;
   for (int j = 0; j < W; j++) S = __fadd_rn(S, exp_sm(-__fdiv_rn(__fsub_rn(c[j], cmin), tau)));
   const float target = __fmul_rn(__fmul_rn((float)u24, 0x1p-24f), S);
-  float cum = 0.0f;
+  const float qnan = __int_as_float(0x7FC00000);
+  float cum = 0.0f, lo = qnan, hi = qnan;
   int pick = -1, last = b;
   for (int j = 0; j < W; j++) {
     const float e = exp_sm(-__fdiv_rn(__fsub_rn(c[j], cmin), tau));
     cum = __fadd_rn(cum, e);
     if (e > 0.0f) last = j;
-    if (fabs((double)target - (double)cum) <= 1e-6 * (double)S) *near_bd = 1;
-    if (pick < 0 && target < cum) pick = j;
+    if (pick < 0 && target < cum) {
+      pick = j;
+      hi = cum;
+    }
+    if (!(target < cum)) lo = cum;
+  }
+  if (ds) {
+    ds[0] = target;
+    ds[1] = S;
+    ds[2] = lo;
+    ds[3] = hi;
   }
   return pick >= 0 ? pick : last;
 }
@@ -196,9 +209,11 @@ __device__ __forceinline__ int grp_excl_scan(int v, int* warp_tot, int* total) {
 
 // ---------------------------------------------------------------- cache table
 
+constexpr int BUCKET = 8;   // keys per bucket: 64 bytes, two 32-byte sectors
+
 struct TableView {
-  uint64_t* keys;     // [4 * nbuckets]
-  uint32_t* stamp;    // [4 * nbuckets]
+  uint64_t* keys;     // [BUCKET * nbuckets]
+  uint32_t* stamp;    // [BUCKET * nbuckets]
   uint32_t* log;      // [rmask + 1]
   uint32_t bmask;     // nbuckets - 1
   uint32_t rmask;     // log ring size - 1
@@ -212,57 +227,67 @@ __device__ __forceinline__ ulonglong2 ld_keys2(const uint64_t* p) {
   return __ldcg(reinterpret_cast<const ulonglong2*>(p));
 }
 
-// Slot holding h, or SLOT_NONE.  Buckets are scanned from h's home bucket;
-// an EMPTY key ends the search (keys are never moved, and slots only go from
-// EMPTY to a key, key to TOMB, TOMB to a key).  *err set if the scan wraps.
-__device__ __forceinline__ uint32_t table_find(const TableView& t, uint64_t h, int* err) {
-  uint32_t b = home_bucket(h, t.bmask);
+// The BUCKET keys of bucket b (four independent 16-byte loads).
+__device__ __forceinline__ void ld_bucket(const uint64_t* keys, uint32_t b, uint64_t (&v)[BUCKET]) {
+  const uint64_t* p = keys + (size_t)BUCKET * b;
+#pragma unroll
+  for (int q = 0; q < BUCKET / 2; q++) {
+    const ulonglong2 x = ld_keys2(p + 2 * q);
+    v[2 * q] = x.x;
+    v[2 * q + 1] = x.y;
+  }
+}
+
+// Slot holding h, or SLOT_NONE; *free_slot = the first EMPTY or TOMB slot of
+// h's probe sequence (where an insert of h would go), with FREE_TOMB set when
+// that slot held a tombstone, or SLOT_NONE.  Buckets are scanned from h's
+// home bucket; a bucket with an EMPTY key ends the search (keys are never
+// moved, and slots only go from EMPTY to a key, key to TOMB, TOMB to a key).
+// *err is set if the scan wraps around the table.
+constexpr uint32_t FREE_TOMB = 0x80000000u;
+
+// Resolves one loaded bucket: returns 1 (found, *slot set), 0 (absent: the
+// bucket holds an EMPTY key) or -1 (continue with the next bucket).
+__device__ __forceinline__ int bucket_scan(const uint64_t (&v)[BUCKET], uint32_t b, uint64_t h,
+                                           uint32_t* slot, uint32_t* fr) {
+  bool empty = false;
+#pragma unroll
+  for (int q = 0; q < BUCKET; q++) {
+    if (v[q] == h) {
+      *slot = (uint32_t)BUCKET * b + q;
+      return 1;
+    }
+    if (v[q] < 2 && *fr == SLOT_NONE)
+      *fr = ((uint32_t)BUCKET * b + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
+    empty |= v[q] == KEY_EMPTY;
+  }
+  return empty ? 0 : -1;
+}
+
+__device__ __forceinline__ uint32_t table_find_free_from(const TableView& t, uint64_t h,
+                                                         uint32_t b, int* err,
+                                                         uint32_t* free_slot) {
   for (uint32_t it = 0; it <= t.bmask; it++) {
-    const ulonglong2 x = ld_keys2(t.keys + 4 * (size_t)b);
-    const ulonglong2 y = ld_keys2(t.keys + 4 * (size_t)b + 2);
-    if (x.x == h) return 4 * b;
-    if (x.y == h) return 4 * b + 1;
-    if (y.x == h) return 4 * b + 2;
-    if (y.y == h) return 4 * b + 3;
-    if (x.x == KEY_EMPTY || x.y == KEY_EMPTY || y.x == KEY_EMPTY || y.y == KEY_EMPTY)
-      return SLOT_NONE;
+    uint64_t v[BUCKET];
+    ld_bucket(t.keys, b, v);
+    uint32_t sl = SLOT_NONE;
+    const int r = bucket_scan(v, b, h, &sl, free_slot);
+    if (r >= 0) return sl;
     b = (b + 1) & t.bmask;
   }
   *err = 1;
   return SLOT_NONE;
 }
 
-// Slot holding h, or SLOT_NONE; *free_slot = the first EMPTY or TOMB slot of
-// h's probe sequence (where an insert of h would go), with FREE_TOMB set when
-// that slot held a tombstone, or SLOT_NONE.
-constexpr uint32_t FREE_TOMB = 0x80000000u;
 __device__ __forceinline__ uint32_t table_find_free(const TableView& t, uint64_t h, int* err,
                                                     uint32_t* free_slot) {
-  uint32_t b = home_bucket(h, t.bmask);
-  uint32_t fr = SLOT_NONE;
-  for (uint32_t it = 0; it <= t.bmask; it++) {
-    const ulonglong2 x = ld_keys2(t.keys + 4 * (size_t)b);
-    const ulonglong2 y = ld_keys2(t.keys + 4 * (size_t)b + 2);
-    const uint64_t v[4] = {x.x, x.y, y.x, y.y};
-    bool empty = false;
-#pragma unroll
-    for (int q = 0; q < 4; q++) {
-      if (v[q] == h) {
-        *free_slot = fr;
-        return 4 * b + q;
-      }
-      if (v[q] < 2 && fr == SLOT_NONE) fr = (4 * b + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
-      empty |= v[q] == KEY_EMPTY;
-    }
-    if (empty) {
-      *free_slot = fr;
-      return SLOT_NONE;
-    }
-    b = (b + 1) & t.bmask;
-  }
-  *err = 1;
   *free_slot = SLOT_NONE;
-  return SLOT_NONE;
+  return table_find_free_from(t, h, home_bucket(h, t.bmask), err, free_slot);
+}
+
+__device__ __forceinline__ uint32_t table_find(const TableView& t, uint64_t h, int* err) {
+  uint32_t fr;
+  return table_find_free(t, h, err, &fr);
 }
 
 // Claims the first EMPTY or TOMB slot of h's probe sequence (h known absent;
@@ -272,15 +297,18 @@ __device__ __forceinline__ uint32_t table_insert(const TableView& t, uint64_t h,
                                                  int* err) {
   uint32_t b = home_bucket(h, t.bmask);
   for (uint32_t it = 0; it <= t.bmask; it++) {
+    uint64_t v[BUCKET];
+    ld_bucket(t.keys, b, v);
 #pragma unroll
-    for (int q = 0; q < 4; q++) {
-      unsigned long long* p = reinterpret_cast<unsigned long long*>(t.keys + 4 * (size_t)b + q);
-      unsigned long long cur = __ldcg(p);
+    for (int q = 0; q < BUCKET; q++) {
+      unsigned long long cur = v[q];
+      unsigned long long* p =
+          reinterpret_cast<unsigned long long*>(t.keys + (size_t)BUCKET * b + q);
       while (cur == KEY_EMPTY || cur == KEY_TOMB) {
         const unsigned long long prev = atomicCAS(p, cur, (unsigned long long)h);
         if (prev == cur) {
           *was_tomb = cur == KEY_TOMB;
-          return 4 * b + q;
+          return (uint32_t)BUCKET * b + q;
         }
         cur = prev;
       }
@@ -348,7 +376,7 @@ __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* met
     grp_bar<NT>();
     return;
   }
-  const size_t nslots = 4 * ((size_t)t.bmask + 1);
+  const size_t nslots = (size_t)BUCKET * ((size_t)t.bmask + 1);
   for (size_t s = threadIdx.x; s < nslots; s += NT) {
     t.keys[s] = KEY_EMPTY;
     t.stamp[s] = STAMP_NONE;

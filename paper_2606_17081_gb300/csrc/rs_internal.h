@@ -23,13 +23,13 @@ struct CacheMeta {
   uint32_t tombs;   // tombstoned slots
 };
 
-// Geometry of one worker's table: 4 * nbuckets slots (>= 2 K) and a log ring
+// Geometry of one worker's table: 8 * nbuckets slots (>= 4 K) and a log ring
 // of R entries (>= 4 K).
 struct TableGeom {
   uint32_t K;
   uint32_t bmask;      // nbuckets - 1
   uint32_t rmask;      // R - 1
-  size_t slots;        // 4 * nbuckets
+  size_t slots;        // 8 * nbuckets
   size_t R;
 };
 
@@ -64,6 +64,9 @@ struct SimBuffers {
   CacheMeta* meta_out;      // [nsim][W]
   rs_replica_result* res;   // [nsim]
   rs_records rec;           // every field non-NULL except possibly cost
+  float* dstat;             // [rows][6]: two lowest costs, draw position (see k_decision_stats)
+  const double* wco_tab;    // [(nbmax+1)(nbmax+2)] w_c * (m / nbt), or NULL
+  int wco_dim;              // nbmax + 2 (row length of wco_tab)
 };
 
 struct SimLaunch {
@@ -90,6 +93,9 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
                               int64_t* nbmax_out, cudaStream_t st);
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st);
+cudaError_t launch_wco_table(double* tab, int nbmax, double w_c, cudaStream_t st);
+cudaError_t launch_decision_stats(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
+                                  cudaStream_t st);
 
 // PoA of Eq. (12): one "problem" per replica.
 struct PoaProblem {

@@ -29,12 +29,12 @@ constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (w
 constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
 constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
 constexpr int PROBE_CAP = 2048;          // W * nb up to which the probe captures every slot
-constexpr int PROBE_ILP = 4;             // lookups a thread keeps in flight
+constexpr int PROBE_ILP = 2;             // lookups a thread keeps in flight
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct SimLayout {
-  size_t ftab, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
+  size_t ftab, wwco, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
   size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
   size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen;
@@ -57,6 +57,7 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   L.field = o;                 \
   o += (bytes);
   TAKE(ftab, 8 * (size_t)(nft > 0 ? nft : 1), 16)
+  TAKE(wwco, 8 * (size_t)W, 8)
   TAKE(f_oitl, 8 * C, 8)
   TAKE(f_a, 8 * C, 8)
   TAKE(f_o, 8 * C, 8)
@@ -105,10 +106,11 @@ size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap) {
 // One request as the loop sees it (two live at once: i and i+1).
 struct ReqState {
   int64_t off0;
+  double oitl;     // O * itl
   int64_t blk;     // ceil((L + O) / 16): active blocks while unfinished
   double a;        // arrival
   double rel;      // client release time
-  int nb, nbt, O, phase;
+  int nb, nbt, O, phase, full;
   float tau, omega;
 };
 
@@ -121,7 +123,7 @@ struct SimScalars {
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, full;
+  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild;
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
@@ -136,7 +138,7 @@ struct SimCtx {
   const SimBuffers* b;
   const SimLaunch* L;
   int sid;
-  double *f_a, *f_o, *ftab, *f_oitl;
+  double *f_a, *f_o, *ftab, *f_oitl, *wwco;
   uint64_t* h_k;
   uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
@@ -519,8 +521,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   int err = 0;
   for (int base = 0; base < total; base += NT_SIM * PROBE_ILP) {   // uniform
     int jj[PROBE_ILP], kk[PROBE_ILP];
-    uint64_t hv[PROBE_ILP];
-    ulonglong2 x[PROBE_ILP], y[PROBE_ILP];
+    uint64_t v[PROBE_ILP][BUCKET];
     uint32_t bk[PROBE_ILP];
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
@@ -530,11 +531,9 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
         const int j = it / nb;
         jj[r] = j;
         kk[r] = it - j * nb;
-        hv[r] = hbuf[kk[r]];
         const TableView t = c.table(j);
-        bk[r] = home_bucket(hv[r], t.bmask);
-        x[r] = ld_keys2(t.keys + 4 * (size_t)bk[r]);
-        y[r] = ld_keys2(t.keys + 4 * (size_t)bk[r] + 2);
+        bk[r] = home_bucket(hbuf[kk[r]], t.bmask);
+        ld_bucket(t.keys, bk[r], v[r]);
       }
     }
 #pragma unroll
@@ -542,22 +541,12 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
       const int it = base + r * NT_SIM + threadIdx.x;
       int miss = 0x7FFFFFFF;
       if (jj[r] >= 0) {
-        const uint64_t v[4] = {x[r].x, x[r].y, y[r].x, y[r].y};
+        const uint64_t h = hbuf[kk[r]];
         uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
-        bool done = false;
-#pragma unroll
-        for (int q = 0; q < 4; q++) {
-          if (!done && v[q] == hv[r]) { sl = 4 * bk[r] + q; done = true; }
-          if (!done && v[q] < 2 && fr == SLOT_NONE)
-            fr = (4 * bk[r] + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
-        }
-        const bool empty = v[0] == KEY_EMPTY || v[1] == KEY_EMPTY || v[2] == KEY_EMPTY ||
-                           v[3] == KEY_EMPTY;
-        if (!done && !empty) {
+        if (bucket_scan(v[r], bk[r], h, &sl, &fr) < 0) {
           // bucket full of other keys: continue along the probe sequence
-          uint32_t fr2;
-          sl = table_find_free(c.table(jj[r]), hv[r], &err, &fr2);
-          if (fr == SLOT_NONE) fr = fr2;
+          const TableView t = c.table(jj[r]);
+          sl = table_find_free_from(t, h, (bk[r] + 1) & t.bmask, &err, &fr);
         }
         c.pslot[it] = sl;
         c.pfree[it] = fr;
@@ -575,14 +564,15 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
 }
 
 // Cache update of the chosen worker (update group, warps 0-6).
-__device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb) {
+__device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb,
+                                              bool full) {
   SimScalars& S = *c.S;
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
   CacheMeta* meta = &c.wmeta[j];
   if (threadIdx.x == 0) {
     const uint64_t span = (uint64_t)meta->T - meta->head + (uint64_t)nb;
-    S.rebuild = span > g.R || meta->tombs > g.slots / 4 || (uint64_t)meta->T + nb > STAMP_LIMIT;
+    S.rebuild = span > g.R || meta->tombs > g.slots / 8 || (uint64_t)meta->T + nb > STAMP_LIMIT;
   }
   for (int k = threadIdx.x; k < nb; k += NT_UPD)   // release the duplicate detector
     if (c.dclaim[k] >= 0) c.sc.dupset[c.dclaim[k]] = 0ull;
@@ -595,7 +585,7 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
     if (threadIdx.x == 0) S.rebuilds++;
   }
-  if (S.full && !S.rebuild)
+  if (full && !S.rebuild)
     cache_lookup_captured<NT_UPD>(tv, c.pslot + (size_t)j * nb, c.pfree + (size_t)j * nb, nb,
                                   c.sc, &S.us);
   else
@@ -606,6 +596,8 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     S.inserted += S.us.n_ins;
     S.evicted += S.us.n_victims;
     S.slow += S.us.slow;
+    update_reset(&S.us);   // for the next request
+    S.us.err = 0;
   }
 }
 
@@ -619,9 +611,8 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   c.f_worker[f] = js;
   c.f_blk[f] = (int32_t)q.blk;
   c.f_a[f] = q.a;
-  const double o = q.nbt > 0 ? __ddiv_rn((double)c.wm[js], (double)q.nbt) : 0.0;
-  c.f_o[f] = __dmul_rn(mc.w_c, o);
-  c.f_oitl[f] = __dmul_rn((double)q.O, mc.itl);
+  c.f_o[f] = c.wwco[js];
+  c.f_oitl[f] = q.oitl;
   c.wA[js] += q.blk;
   S.in_flight++;
   S.hit_blocks += c.wm[js];
@@ -640,18 +631,33 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   S.n_routed++;
 }
 
-// Reads request i's scalars (control thread).
-__device__ __forceinline__ void load_request(const SimCtx& c, ReqState& q, int64_t i) {
-  const int64_t o0 = c.d->offsets[i], o1 = c.d->offsets[i + 1];
-  const int O = c.d->out_len[i];
-  const int64_t L = o1 - o0;
-  q.off0 = o0;
-  q.rel = c.d->release[i];
-  q.O = O;
+// Request i's scalars as read from the trace (control thread).
+struct RawReq {
+  int64_t o0, o1;
+  double rel;
+  int O;
+};
+
+__device__ __forceinline__ RawReq read_request(const SimCtx& c, int64_t i) {
+  RawReq r;
+  r.o0 = c.d->offsets[i];
+  r.o1 = c.d->offsets[i + 1];
+  r.rel = c.d->release[i];
+  r.O = c.d->out_len[i];
+  return r;
+}
+
+__device__ __forceinline__ void load_request(const SimCtx& c, ReqState& q, const RawReq& r) {
+  const int64_t L = r.o1 - r.o0;
+  q.off0 = r.o0;
+  q.rel = r.rel;
+  q.O = r.O;
+  q.oitl = __dmul_rn((double)r.O, c.L->mc.itl);
   q.nb = (L >> 4) > 0x7FFFFFFF ? 0x7FFFFFFF : (int)(L >> 4);
   q.nbt = (int)((L + 15) >> 4);
-  q.blk = (L + O + 15) >> 4;
+  q.blk = (L + r.O + 15) >> 4;
   q.phase = 0;
+  q.full = (int64_t)c.L->mc.W * (L >> 4) <= PROBE_CAP;
 }
 
 // Algorithm 1: the router parameters of the current regime (control thread).
@@ -666,6 +672,16 @@ __device__ __forceinline__ void regime_params(const SimCtx& c, ReqState& q) {
   }
   q.tau = tau;
   q.omega = om;
+}
+
+// Probe state of a request (lanes of the control warp).
+__device__ __forceinline__ void probe_setup(SimCtx& c, const ReqState& q, int lane) {
+  const int W = c.L->mc.W;
+  for (int j = lane; j < W; j += 32) {
+    c.wm[j] = q.nb;
+    c.wopen[j] = j;
+  }
+  if (lane == 0) c.S->nopen = W;
 }
 
 // Block hashes of a request into a staging buffer (lanes of one warp).
@@ -695,6 +711,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   c.sid = sid;
   c.ftab = reinterpret_cast<double*>(smem + lay.ftab);
   c.f_oitl = reinterpret_cast<double*>(smem + lay.f_oitl);
+  c.wwco = reinterpret_cast<double*>(smem + lay.wwco);
   c.f_a = reinterpret_cast<double*>(smem + lay.f_a);
   c.f_o = reinterpret_cast<double*>(smem + lay.f_o);
   c.h_k = reinterpret_cast<uint64_t*>(smem + lay.h_k);
@@ -769,11 +786,17 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   // ---- prologue: request 0's arrival and hashes
   if (n > 0) {
     if (threadIdx.x == CTL) {
-      load_request(c, S.q[0], 0);
+      load_request(c, S.q[0], read_request(c, 0));
       S.evres = events_advance(c, S.q[0]);
+      if (S.evres == 0) regime_params(c, S.q[0]);
+      update_reset(&S.us);
+      S.us.err = 0;
     }
     __syncthreads();
-    if (warp == NT_SIM / 32 - 1) stage_hashes(c, S.q[0], c.hbuf0, lane);
+    if (warp == NT_SIM / 32 - 1) {
+      stage_hashes(c, S.q[0], c.hbuf0, lane);
+      probe_setup(c, S.q[0], lane);
+    }
   }
   for (int64_t i = 0; i < n; i++) {
     const int p = (int)(i & 1);
@@ -782,7 +805,10 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       __syncthreads();
       if (S.evres == 0) break;
       tick_cta(c);
-      if (threadIdx.x == CTL) S.evres = events_advance(c, S.q[p]);
+      if (threadIdx.x == CTL) {
+        S.evres = events_advance(c, S.q[p]);
+        if (S.evres == 0) regime_params(c, S.q[p]);
+      }
     }
     if (S.status != RS_OK) break;
     const int nb = S.q[p].nb;
@@ -791,22 +817,11 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       break;
     }
     const int nbt = S.q[p].nbt;
+    const bool full = S.q[p].full;
     const uint64_t* hb = c.hbuf(p);
     const int64_t row = d.rec_base + i;
-    for (int j = threadIdx.x; j < W; j += NT_SIM) {
-      c.wm[j] = nb;
-      c.wopen[j] = j;
-    }
-    if (threadIdx.x == 0) {
-      S.nopen = W;
-      S.full = W * nb <= PROBE_CAP;
-      update_reset(&S.us);
-      S.us.err = 0;
-    }
-    if (threadIdx.x == CTL) regime_params(c, S.q[p]);
-    __syncthreads();
     // ---- cached prefix on every worker
-    if (W * nb <= PROBE_CAP) probe_full(c, hb, nb);
+    if (full) probe_full(c, hb, nb);
     else probe_prefixes(c, hb, nb);
     // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
     if (warp == 0) {
@@ -821,37 +836,45 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       __syncwarp();
       if (lane == 0) {
         const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
-        int nbd = 0;
-        S.jstar = select_worker(c.wcost, W, tau, u24, &nbd);
-        if (tau > 0.0f) {
-          S.sampled++;
-          S.near_bd += nbd;
-        }
+        float* ds = b.dstat + row * 6;
+        S.jstar = select_worker(c.wcost, W, tau, u24, ds + 2);
+        if (tau > 0.0f) S.sampled++;
+        else ds[3] = -1.0f;   // no draw
       }
     } else if (warp == 1 && lane == 0) {
-      // statistics of the decision, beside the choice: work done by the probe,
-      // and whether the two lowest Eq. (1) costs tie within 1e-6 (recomputed
-      // from the probe results so as not to wait for warp 0)
+      // statistics of the decision, beside the choice: work done by the probe
       int64_t pb = 0;
       for (int j = 0; j < W; j++) pb += min(c.wm[j] + 1, nb);
       S.probe_blocks += pb;
       S.hashed_blocks += nb;
-      if (W >= 2) {
-        const float om = S.q[p].omega;
-        int bmin = 0;
-        float c1 = router_cost(om, (int64_t)nbt - c.wm[0], c.wA[0]);
-        for (int j = 1; j < W; j++) {
-          const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
-          if (cj < c1) { c1 = cj; bmin = j; }
+      // the two lowest Eq. (1) costs, for the near-tie statistic (counted
+      // after the run); recomputed from the probe results so as not to wait
+      // for warp 0
+      const float om = S.q[p].omega;
+      float c1 = router_cost(om, (int64_t)nbt - c.wm[0], c.wA[0]);
+      int bmin = 0;
+      for (int j = 1; j < W; j++) {
+        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+        if (cj < c1) { c1 = cj; bmin = j; }
+      }
+      float c2 = __int_as_float(0x7F800000);
+      for (int j = 0; j < W; j++) {
+        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+        if (j != bmin && cj < c2) c2 = cj;
+      }
+      b.dstat[row * 6] = c1;
+      b.dstat[row * 6 + 1] = c2;
+    } else if (warp == NT_SIM / 32 - 1) {
+      // w_c * o_ij for every worker (the chosen one's enters its latency)
+      for (int j = lane; j < W; j += 32) {
+        double w;
+        if (b.wco_tab) {
+          w = b.wco_tab[(size_t)c.wm[j] * b.wco_dim + nbt];
+        } else {
+          const double o = nbt > 0 ? __ddiv_rn((double)c.wm[j], (double)nbt) : 0.0;
+          w = __dmul_rn(mc.w_c, o);
         }
-        float c2 = __int_as_float(0x7F800000);
-        for (int j = 0; j < W; j++) {
-          const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
-          if (j != bmin && cj < c2) c2 = cj;
-        }
-        const double diff = (double)c2 - (double)c1;
-        if (diff <= 1e-6 * fabs((double)c2)) S.near_ties++;
-        if (c2 == c1) S.exact_ties++;
+        c.wwco[j] = w;
       }
     } else if (warp >= 2 && warp < NT_SIM / 32 - 1) {
       // two blocks of one prompt with the same chained hash (a 64-bit
@@ -864,18 +887,25 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
     const int js = S.jstar;
     if (warp < NT_SIM / 32 - 1) {
       // ---- the chosen worker's LRU cache (warps 0-6)
-      update_chosen(c, hb, js, nb);
+      update_chosen(c, hb, js, nb, full);
     } else {
       // ---- control warp: request i's load and latency; request i+1's arrival
       ReqState& nq = S.q[p ^ 1];
       if (lane == 0) {
+        // the next request's loads go out first; their latency overlaps the bookkeeping
+        RawReq raw;
+        if (i + 1 < n) raw = read_request(c, i + 1);
         book_request(c, S.q[p], i);
-        if (i + 1 < n) load_request(c, nq, i + 1);
+        if (i + 1 < n) load_request(c, nq, raw);
       }
       __syncwarp();
       if (i + 1 < n) {
         stage_hashes(c, nq, c.hbuf(p ^ 1), lane);
-        if (lane == 0) S.evres = events_advance(c, nq);
+        probe_setup(c, nq, lane);
+        if (lane == 0) {
+          S.evres = events_advance(c, nq);
+          if (S.evres == 0) regime_params(c, nq);
+        }
       }
     }
   }
@@ -956,6 +986,79 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
     b.res[sid] = r;
   }
   for (int j = threadIdx.x; j < W; j += NT_SIM) b.meta_out[(size_t)sid * W + j] = c.wmeta[j];
+}
+
+// w_c * (m / nbt) for every cached-prefix length m <= nbmax and prompt
+// length nbt <= nbmax + 1 blocks, rounded as the latency of Eq. (9) uses it.
+__global__ void k_wco_table(double* tab, int nbmax, double w_c) {
+  const int dim = nbmax + 2;
+  const int64_t total = (int64_t)(nbmax + 1) * dim;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int m = (int)(e / dim), nbt = (int)(e % dim);
+    const double o = nbt > 0 ? __ddiv_rn((double)m, (double)nbt) : 0.0;
+    tab[e] = __dmul_rn(w_c, o);
+  }
+}
+
+cudaError_t launch_wco_table(double* tab, int nbmax, double w_c, cudaStream_t st) {
+  k_wco_table<<<152 * 4, 256, 0, st>>>(tab, nbmax, w_c);
+  return cudaGetLastError();
+}
+
+// Decision statistics of every replica from the per-request records of the
+// simulation: top-two Eq. (1) costs within 1e-6 relative (and equal), and
+// Eq. (2) draws within 1e-6 S of a cumulative-weight boundary.
+__global__ void __launch_bounds__(256) k_decision_stats(const SimDesc* __restrict__ descs,
+                                                        SimBuffers b, SimLaunch L) {
+  const SimDesc d = descs[blockIdx.x];
+  const int64_t n = b.res[blockIdx.x].n_routed;
+  long long near = 0, exact = 0, bd = 0;
+  for (int64_t q = threadIdx.x; q < n; q += blockDim.x) {
+    const float* ds = b.dstat + (d.rec_base + q) * 6;
+    if (L.mc.W >= 2) {
+      const float c1 = ds[0], c2 = ds[1];
+      const double diff = (double)c2 - (double)c1;
+      if (diff <= 1e-6 * fabs((double)c2)) near++;
+      if (c2 == c1) exact++;
+    }
+    if (ds[3] >= 0.0f) {
+      const double tg = (double)ds[2], S = (double)ds[3], eps = 1e-6 * S;
+      const float lo = ds[4], hi = ds[5];
+      if ((lo == lo && fabs(tg - (double)lo) <= eps) || (hi == hi && fabs(tg - (double)hi) <= eps))
+        bd++;
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    near += __shfl_xor_sync(FULL_MASK, near, o);
+    exact += __shfl_xor_sync(FULL_MASK, exact, o);
+    bd += __shfl_xor_sync(FULL_MASK, bd, o);
+  }
+  __shared__ long long red[3][8];
+  if ((threadIdx.x & 31) == 0) {
+    red[0][threadIdx.x >> 5] = near;
+    red[1][threadIdx.x >> 5] = exact;
+    red[2][threadIdx.x >> 5] = bd;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long a = 0, e = 0, z = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); w++) {
+      a += red[0][w];
+      e += red[1][w];
+      z += red[2][w];
+    }
+    b.res[blockIdx.x].near_ties = a;
+    b.res[blockIdx.x].exact_ties = e;
+    b.res[blockIdx.x].near_boundary = z;
+  }
+}
+
+cudaError_t launch_decision_stats(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
+                                  cudaStream_t st) {
+  if (L.nsim <= 0) return cudaSuccess;
+  k_decision_stats<<<L.nsim, 256, 0, st>>>(d_desc, b, L);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
