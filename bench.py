@@ -279,7 +279,9 @@ def cpu_baseline(p, traces, budget_s: float = 15.0) -> dict:
     cfg = O.OracleConfig(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
     done = dec = 0
     t0 = time.perf_counter()
-    order = [0, 5, 1, 6, 2, 7, 3, 8, 4, 9]   # selfish / load-balanced pairs over C
+    # selfish / load-balanced pairs over C first, then the rest of the 64 in order
+    first = [0, 5, 1, 6, 2, 7, 3, 8, 4, 9]
+    order = first + [k for k in range(len(p.replicas)) if k not in first]
     for k in order:
         r = p.replicas[k]
         o = O.simulate(cfg, traces[r.trace], r.C, policy=r.policy, controller=r.controller,
@@ -291,8 +293,9 @@ def cpu_baseline(p, traces, budget_s: float = 15.0) -> dict:
             break
     el = time.perf_counter() - t0
     return {"value": dec / el, "unit": "decisions/s", "cores": 1, "kind": "oracle",
-            "sample": f"{done} whole replicas (20000 requests each, replicas "
-                      f"{order[:done]} of the 64) incl. PoA, single thread, {el:.1f} s"}
+            "sample": f"{done} whole replicas of the {len(p.replicas)} (20000 requests each; "
+                      f"pairs 0/5, 1/6, ... first, then in order) incl. PoA, single thread, "
+                      f"{el:.1f} s"}
 
 
 def run_reference(args):

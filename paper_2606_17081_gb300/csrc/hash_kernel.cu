@@ -1,19 +1,32 @@
 // KV block hashing of prompts (K1), in two passes over all traces of a call.
 //
-// Content pass: one warp per request, lane l takes block k0 + l of a
-// 32-block chunk; the block's 64 bytes arrive as four 16-byte loads (five when
-// the request does not start on a 16-byte boundary) and fold into the content
-// hash g_k; the lane stores g_k ^ k at the block's output slot.  Fully
-// parallel, coalesced, HBM-bound (4 bytes per token in, 8 per block out).
+// Content pass (k_block_content): one warp per request, lane l takes blocks
+// l and l + 32 of each 64-block span; a block's 64 bytes arrive as four
+// 16-byte loads (five when the request does not start on a 16-byte boundary)
+// and fold into the content hash g_k; the lane stores g_k ^ k at the block's
+// output slot.  Fully parallel, coalesced, HBM-bound: 4 bytes per token in,
+// 8 bytes per block out.
 //
-// Chain pass: one thread per request folds its slots in order,
-// h_k = mix(h_{k-1} ^ g_k ^ k), in place; loads run four slots ahead.  One
-// 64-bit mix per block; the serial dependence is per request only.
+// Chain pass (k_block_chain): h_k = mix(h_{k-1} ^ g_k ^ k) is serial per
+// request, so each lane owns one request at a time and each round moves every
+// lane's request on by a chunk of 32 blocks: per request the warp reads the
+// chunk's 32 values with one coalesced 256-byte load into shared memory,
+// every lane folds its own row in order, and per request the warp writes the
+// 32 hashes back with one coalesced store.  Lanes whose requests are done
+// claim the next ones from a work counter (one atomic per warp for all of
+// them), so the warps stay busy until the counter runs out.  8 bytes per
+// block in and out.
 #include <climits>
 
 #include "rs_device.cuh"
 
 namespace rs {
+
+constexpr int CONTENT_NT = 256;              // content pass: threads per CTA
+constexpr int CHAIN_WARPS = 4;               // chain pass: warps per CTA
+constexpr int CHAIN_NT = 32 * CHAIN_WARPS;
+constexpr int CHAIN_ROW = 33;                // 32 staged blocks per request + 1 pad word
+constexpr int CHAIN_ILP = 8;                 // requests whose chunks are loaded together
 
 template <int S>
 __device__ __forceinline__ void take16(const uint32_t (&a)[20], uint32_t (&w)[16]) {
@@ -21,14 +34,27 @@ __device__ __forceinline__ void take16(const uint32_t (&a)[20], uint32_t (&w)[16
   for (int j = 0; j < 16; j++) w[j] = a[j + S];
 }
 
-__device__ __forceinline__ uint64_t hash_block(const int4* q, int shift) {
-  const int4 v0 = __ldg(q), v1 = __ldg(q + 1), v2 = __ldg(q + 2), v3 = __ldg(q + 3);
-  const int4 v4 = shift ? __ldg(q + 4) : make_int4(0, 0, 0, 0);
-  const uint32_t a[20] = {(uint32_t)v0.x, (uint32_t)v0.y, (uint32_t)v0.z, (uint32_t)v0.w,
-                          (uint32_t)v1.x, (uint32_t)v1.y, (uint32_t)v1.z, (uint32_t)v1.w,
-                          (uint32_t)v2.x, (uint32_t)v2.y, (uint32_t)v2.z, (uint32_t)v2.w,
-                          (uint32_t)v3.x, (uint32_t)v3.y, (uint32_t)v3.z, (uint32_t)v3.w,
-                          (uint32_t)v4.x, (uint32_t)v4.y, (uint32_t)v4.z, (uint32_t)v4.w};
+// The 64 bytes of one block starting `shift` int32 words into five int4.
+struct BlockBytes {
+  int4 v0, v1, v2, v3, v4;
+};
+
+__device__ __forceinline__ BlockBytes load_block(const int4* q, int shift) {
+  BlockBytes b;
+  b.v0 = __ldg(q);
+  b.v1 = __ldg(q + 1);
+  b.v2 = __ldg(q + 2);
+  b.v3 = __ldg(q + 3);
+  b.v4 = shift ? __ldg(q + 4) : make_int4(0, 0, 0, 0);
+  return b;
+}
+
+__device__ __forceinline__ uint64_t content_of(const BlockBytes& b, int shift) {
+  const uint32_t a[20] = {(uint32_t)b.v0.x, (uint32_t)b.v0.y, (uint32_t)b.v0.z, (uint32_t)b.v0.w,
+                          (uint32_t)b.v1.x, (uint32_t)b.v1.y, (uint32_t)b.v1.z, (uint32_t)b.v1.w,
+                          (uint32_t)b.v2.x, (uint32_t)b.v2.y, (uint32_t)b.v2.z, (uint32_t)b.v2.w,
+                          (uint32_t)b.v3.x, (uint32_t)b.v3.y, (uint32_t)b.v3.z, (uint32_t)b.v3.w,
+                          (uint32_t)b.v4.x, (uint32_t)b.v4.y, (uint32_t)b.v4.z, (uint32_t)b.v4.w};
   uint32_t w[16];
   switch (shift) {
     case 0: take16<0>(a, w); break;
@@ -39,22 +65,20 @@ __device__ __forceinline__ uint64_t hash_block(const int4* q, int shift) {
   return block_content16(w);
 }
 
-constexpr int HASH_NT = 256;
-
 __device__ __forceinline__ int find_job(const HashJob* jobs, int njobs, int64_t r) {
   int j = 0;
   while (j + 1 < njobs && r >= jobs[j + 1].req_base) j++;
   return j;
 }
 
-__global__ void __launch_bounds__(HASH_NT) k_block_content(const HashJob* __restrict__ jobs,
-                                                           int njobs, int64_t total_req) {
+__global__ void __launch_bounds__(CONTENT_NT) k_block_content(const HashJob* __restrict__ jobs,
+                                                              int njobs, int64_t total_req) {
   __shared__ HashJob s_jobs[HASH_MAX_JOBS];
-  for (int j = threadIdx.x; j < njobs; j += HASH_NT) s_jobs[j] = jobs[j];
+  for (int j = threadIdx.x; j < njobs; j += CONTENT_NT) s_jobs[j] = jobs[j];
   __syncthreads();
   const int lane = threadIdx.x & 31;
-  const int64_t warp0 = ((int64_t)blockIdx.x * HASH_NT + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * HASH_NT) >> 5;
+  const int64_t warp0 = ((int64_t)blockIdx.x * CONTENT_NT + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * CONTENT_NT) >> 5;
   for (int64_t r = warp0; r < total_req; r += nwarps) {
     const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
     const int64_t i = r - J.req_base;
@@ -63,39 +87,113 @@ __global__ void __launch_bounds__(HASH_NT) k_block_content(const HashJob* __rest
     const int shift = (int)(o0 & 3);
     const int4* q = reinterpret_cast<const int4*>(J.tokens) + (o0 >> 2);
     uint64_t* out = J.out + (o0 >> 4);
-    for (int64_t k = lane; k < nb; k += 32) out[k] = hash_block(q + 4 * k, shift) ^ (uint64_t)k;
+    for (int64_t k0 = 0; k0 < nb; k0 += 64) {
+      // both blocks' loads go out before either is folded
+      const int64_t ka = k0 + lane, kb = ka + 32;
+      const bool va = ka < nb, vb = kb < nb;
+      BlockBytes ba, bb;
+      if (va) ba = load_block(q + 4 * ka, shift);
+      if (vb) bb = load_block(q + 4 * kb, shift);
+      if (va) out[ka] = content_of(ba, shift) ^ (uint64_t)ka;
+      if (vb) out[kb] = content_of(bb, shift) ^ (uint64_t)kb;
+    }
   }
 }
 
-__global__ void __launch_bounds__(HASH_NT) k_block_chain(const HashJob* __restrict__ jobs,
-                                                         int njobs, int64_t total_req,
-                                                         uint64_t seed,
-                                                         int64_t* __restrict__ nbmax) {
+__global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restrict__ jobs,
+                                                          int njobs, int64_t total_req,
+                                                          uint64_t seed,
+                                                          int64_t* __restrict__ nbmax,
+                                                          unsigned long long* __restrict__ work) {
   __shared__ HashJob s_jobs[HASH_MAX_JOBS];
-  __shared__ int64_t s_max[HASH_NT / 32];
-  for (int j = threadIdx.x; j < njobs; j += HASH_NT) s_jobs[j] = jobs[j];
+  __shared__ uint64_t s_stage[CHAIN_WARPS][32 * CHAIN_ROW];
+  __shared__ int64_t s_max[CHAIN_WARPS];
+  for (int j = threadIdx.x; j < njobs; j += CHAIN_NT) s_jobs[j] = jobs[j];
   __syncthreads();
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const unsigned lt_mask = (1u << lane) - 1u;
+  uint64_t* stage = s_stage[wid];
+  uint64_t* row = stage + lane * CHAIN_ROW;
   int64_t local_max = 0;
-  const int64_t stride = (int64_t)gridDim.x * HASH_NT;
-  for (int64_t r = (int64_t)blockIdx.x * HASH_NT + threadIdx.x; r < total_req; r += stride) {
-    const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
-    const int64_t i = r - J.req_base;
-    const int64_t o0 = J.offsets[i];
-    const int64_t nb = (J.offsets[i + 1] - o0) >> 4;
-    local_max = nb > local_max ? nb : local_max;
-    uint64_t* out = J.out + (o0 >> 4);
-    uint64_t h = seed;
-    int64_t k = 0;
-    for (; k + 4 <= nb; k += 4) {
-      const uint64_t x0 = out[k], x1 = out[k + 1], x2 = out[k + 2], x3 = out[k + 3];
-      h = chain_step(h, x0); out[k] = h;
-      h = chain_step(h, x1); out[k + 1] = h;
-      h = chain_step(h, x2); out[k + 2] = h;
-      h = chain_step(h, x3); out[k + 3] = h;
+  bool exhausted = false;   // the work counter has passed the last request (warp-uniform)
+  // this lane's request: blocks [c0, nb) of the hashes at oaddr, chain value h
+  bool has = false;
+  unsigned long long oaddr = 0;
+  int64_t nb = 0, c0 = 0;
+  uint64_t h = seed;
+  for (;;) {
+    // ---- lanes without a request claim the next ones, one atomic per warp
+    unsigned need = __ballot_sync(FULL_MASK, !has);
+    while (need && !exhausted) {
+      const int cnt = __popc(need);
+      unsigned long long b = 0;
+      if (lane == 0) b = atomicAdd(work, (unsigned long long)cnt);
+      b = __shfl_sync(FULL_MASK, b, 0);
+      if ((int64_t)b + cnt >= total_req) exhausted = true;
+      const int64_t r = (int64_t)b + __popc(need & lt_mask);
+      if (!has && r < total_req) {
+        const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
+        const int64_t i = r - J.req_base;
+        const int64_t o0 = __ldg(J.offsets + i);
+        nb = (__ldg(J.offsets + i + 1) - o0) >> 4;
+        oaddr = (unsigned long long)(J.out + (o0 >> 4));
+        c0 = 0;
+        h = seed;
+        local_max = nb > local_max ? nb : local_max;
+        has = nb > 0;   // a prompt without a full block has nothing to chain
+      }
+      need = __ballot_sync(FULL_MASK, !has);
     }
-    for (; k < nb; k++) {
-      h = chain_step(h, out[k]);
-      out[k] = h;
+    const unsigned busy = __ballot_sync(FULL_MASK, has);
+    if (!busy) break;
+    // ---- 1. every busy lane's chunk into its row, CHAIN_ILP requests at a time
+    unsigned act = busy;
+    while (act) {
+      int rq[CHAIN_ILP];
+      bool vq[CHAIN_ILP];
+      uint64_t gq[CHAIN_ILP];
+#pragma unroll
+      for (int u = 0; u < CHAIN_ILP; u++) {
+        rq[u] = act ? __ffs(act) - 1 : -1;
+        act &= act - 1;   // no-op once empty
+      }
+#pragma unroll
+      for (int u = 0; u < CHAIN_ILP; u++) {
+        const int src = rq[u] < 0 ? 0 : rq[u];
+        const int64_t nbu = __shfl_sync(FULL_MASK, nb, src);
+        const int64_t k = __shfl_sync(FULL_MASK, c0, src) + lane;
+        const uint64_t* ou = reinterpret_cast<const uint64_t*>(__shfl_sync(FULL_MASK, oaddr, src));
+        vq[u] = rq[u] >= 0 && k < nbu;
+        if (vq[u]) gq[u] = ou[k];
+      }
+#pragma unroll
+      for (int u = 0; u < CHAIN_ILP; u++)
+        if (vq[u]) stage[rq[u] * CHAIN_ROW + lane] = gq[u];
+    }
+    __syncwarp();
+    // ---- 2. each lane chains its own request through the chunk
+    const int64_t left = nb - c0;
+    const int m = !has ? 0 : (left < 32 ? (int)left : 32);
+#pragma unroll 4
+    for (int j = 0; j < m; j++) {
+      h = chain_step(h, row[j]);
+      row[j] = h;
+    }
+    __syncwarp();
+    // ---- 3. coalesced stores, one request at a time
+    act = busy;
+    while (act) {
+      const int ra = __ffs(act) - 1;
+      act &= act - 1;
+      const int64_t nba = __shfl_sync(FULL_MASK, nb, ra);
+      const int64_t k = __shfl_sync(FULL_MASK, c0, ra) + lane;
+      uint64_t* oa = reinterpret_cast<uint64_t*>(__shfl_sync(FULL_MASK, oaddr, ra));
+      if (k < nba) oa[k] = stage[ra * CHAIN_ROW + lane];
+    }
+    __syncwarp();
+    if (has) {
+      c0 += 32;
+      if (c0 >= nb) has = false;
     }
   }
   if (nbmax) {
@@ -104,28 +202,37 @@ __global__ void __launch_bounds__(HASH_NT) k_block_chain(const HashJob* __restri
       const int64_t v = __shfl_xor_sync(FULL_MASK, local_max, o);
       local_max = v > local_max ? v : local_max;
     }
-    if ((threadIdx.x & 31) == 0) s_max[threadIdx.x >> 5] = local_max;
+    if (lane == 0) s_max[wid] = local_max;
     __syncthreads();
     if (threadIdx.x == 0) {
-      int64_t m = 0;
-      for (int w = 0; w < HASH_NT / 32; w++) m = s_max[w] > m ? s_max[w] : m;
-      if (m > 0) atomicMax(reinterpret_cast<unsigned long long*>(nbmax), (unsigned long long)m);
+      int64_t mx = 0;
+      for (int w = 0; w < CHAIN_WARPS; w++) mx = s_max[w] > mx ? s_max[w] : mx;
+      if (mx > 0) atomicMax(reinterpret_cast<unsigned long long*>(nbmax), (unsigned long long)mx);
     }
   }
 }
 
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
-                              int64_t* nbmax_out, cudaStream_t st) {
+                              int64_t* nbmax_out, unsigned long long* work, cudaStream_t st) {
   if (total_req <= 0) return cudaSuccess;
-  if (njobs < 1 || njobs > HASH_MAX_JOBS) return cudaErrorInvalidValue;
-  int64_t wb = (total_req + 7) / 8;              // 8 warps per CTA, one request each
-  if (wb > 152 * 16) wb = 152 * 16;
-  k_block_content<<<(unsigned)wb, HASH_NT, 0, st>>>(jobs_dev, njobs, total_req);
-  cudaError_t e = cudaGetLastError();
+  if (njobs < 1 || njobs > HASH_MAX_JOBS || !work) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  int64_t tb = (total_req + HASH_NT - 1) / HASH_NT;
-  if (tb > 152 * 8) tb = 152 * 8;
-  k_block_chain<<<(unsigned)tb, HASH_NT, 0, st>>>(jobs_dev, njobs, total_req, seed, nbmax_out);
+  // content: one warp per request, grid-strided
+  int64_t cb = (total_req + CONTENT_NT / 32 - 1) / (CONTENT_NT / 32);
+  if (cb > (int64_t)sms * 16) cb = (int64_t)sms * 16;
+  k_block_content<<<(unsigned)cb, CONTENT_NT, 0, st>>>(jobs_dev, njobs, total_req);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // chain: one wave of resident CTAs; the work counter hands out the requests
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_block_chain, CHAIN_NT, 0);
+  if (e != cudaSuccess) return e;
+  int64_t nblk = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+  const int64_t need = (total_req + CHAIN_NT - 1) / CHAIN_NT;
+  if (nblk > need) nblk = need;
+  k_block_chain<<<(unsigned)nblk, CHAIN_NT, 0, st>>>(jobs_dev, njobs, total_req, seed, nbmax_out,
+                                                     work);
   return cudaGetLastError();
 }
 

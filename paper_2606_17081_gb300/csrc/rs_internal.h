@@ -89,8 +89,10 @@ struct HashJob {
   int64_t req_base;
 };
 constexpr int HASH_MAX_JOBS = 64;
+// `work` points to a zeroed counter (one per launch) from which the kernel's
+// warps take their groups of requests.
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
-                              int64_t* nbmax_out, cudaStream_t st);
+                              int64_t* nbmax_out, unsigned long long* work, cudaStream_t st);
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st);
 cudaError_t launch_wco_table(double* tab, int nbmax, double w_c, cudaStream_t st);
