@@ -49,6 +49,18 @@ def _dist():
     return ws, rank, local
 
 
+def _max_over_ranks(values, device):
+    """Element-wise maximum of `values` over all ranks (the step time of the
+    slowest rank); the identity when torch.distributed is not initialised."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
 def _plan(rank: int, n_req=None):
     from paper_2606_17081_gb300 import workloads as wk
     p = wk.plan(WORKLOAD, n_req=n_req)
@@ -128,6 +140,27 @@ def _table_bytes(K: int) -> int:
     while ring < 4 * K:
         ring <<= 1
     return slots * 12 + ring * 4
+
+
+# DRAM bytes (read + write) of one full-size k_sim launch of this workload,
+# from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
+# with the SHA-256 of the simulation kernel's sources it was taken with.
+SIM_TRAFFIC = {"bytes": 32236985088 + 8341278976,
+               "sources_sha256": "d1226cb2c5fbd82b4d58dffc5e3d51502e7787108fcc490bfd4d4a2afea6e45d",
+               "summary": "profiles/k_sim_p2d.md"}
+
+
+def _sim_traffic(full_size: bool):
+    """The captured DRAM traffic per k_sim launch, or None when the kernel
+    changed since the capture (or the workload is not the full-size one)."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("sim_kernel.cu", "rs_device.cuh", "rs_internal.h"):
+        with open(os.path.join(ROOT, "paper_2606_17081_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if not full_size or h.hexdigest() != SIM_TRAFFIC["sources_sha256"]:
+        return None
+    return float(SIM_TRAFFIC["bytes"])
 
 
 def _alg_bytes(results, W: int) -> float:
@@ -210,10 +243,7 @@ def run_gpu(args):
     torch.cuda.synchronize()
     barrier()
     e2e_s = time.perf_counter() - t0
-    if ws > 1:
-        tt = torch.tensor([ms, e2e_s], dtype=torch.float64, device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms, e2e_s = float(tt[0]), float(tt[1])
+    ms, e2e_s = _max_over_ranks([ms, e2e_s], "cuda")
     if rank != 0:
         if ws > 1:
             dist.destroy_process_group()
@@ -255,7 +285,8 @@ def run_gpu(args):
         "roofline": {"kernel": "k_sim (replica simulation, one CTA per replica)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
-                     "alg_bytes_per_launch": alg, "traffic": None,
+                     "alg_bytes_per_launch": alg, "traffic": _sim_traffic(args.n_req is None),
+                     "traffic_source": SIM_TRAFFIC["summary"],
                      "note": "latency-bound event loop: 64 replicas on 152 SMs"},
         "hash_roofline": {"kernel": "k_block_hash", "bound": "hbm", "achieved": hash_gbs,
                           "peak": peak, "unit": "GB/s", "frac": hash_gbs / peak,

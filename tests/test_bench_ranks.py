@@ -1,0 +1,76 @@
+"""The multi-rank logic of bench.py, run as two gloo ranks on the CPU.
+
+Replicas are independent, so under torchrun every rank simulates its own
+replica grid (weak scaling) and the ranks meet only to take the slowest rank's
+time.  Checked here: each rank draws its own traces and routing seeds, the
+grids have the same shape, the timing reduction is the maximum over ranks, and
+a rank other than 0 prints nothing.
+"""
+import contextlib
+import io
+import json
+import os
+import socket
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank: int, world: int, port: int, out_dir: str):
+    sys.path.insert(0, ROOT)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import torch.distributed as dist
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        p = bench._plan(rank, n_req=50)
+        # rank r's step time is r + 1 ms, its end-to-end time 10 - r s
+        ms, e2e = bench._max_over_ranks([rank + 1.0, 10.0 - rank], "cpu")
+        buf = io.StringIO()
+        with contextlib.redirect_stdout(buf):
+            if rank != 0:
+                bench.run_reference(type("A", (), {"steps": 1, "warmup": 0})())
+        rec = {"trace_seeds": p.trace_seeds, "seeds": [r.seed for r in p.replicas],
+               "shape": [(r.C, r.policy, r.omega, r.tau, r.n_req, r.trace) for r in p.replicas],
+               "max": [ms, e2e], "printed": buf.getvalue()}
+        with open(os.path.join(out_dir, f"rank{rank}.json"), "w") as f:
+            json.dump(rec, f)
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_shard_replicas_and_take_max_time(tmp_path):
+    mp = pytest.importorskip("torch.multiprocessing")
+    world = 2
+    port = _free_port()
+    ctx = mp.get_context("spawn")
+    procs = [ctx.Process(target=_rank_main, args=(r, world, port, str(tmp_path)))
+             for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=180)
+    for p in procs:
+        if p.is_alive():
+            p.kill()
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    r0 = json.loads((tmp_path / "rank0.json").read_text())
+    r1 = json.loads((tmp_path / "rank1.json").read_text())
+    # same grid shape, disjoint traces and routing seeds
+    assert r0["shape"] == r1["shape"]
+    assert not set(r0["trace_seeds"]) & set(r1["trace_seeds"])
+    assert not set(r0["seeds"]) & set(r1["seeds"])
+    # the reported times are the slowest rank's
+    assert r0["max"] == r1["max"] == [2.0, 10.0]
+    # the reference arm prints only on rank 0
+    assert r1["printed"] == ""
