@@ -723,7 +723,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   CK(cudaEventRecord(ctx->ev[2], ctx->st), "event");
   if (!(flags & RS_SIM_NO_POA)) {
     if ((r = run_poa(ctx, rec, probs, rows, win_slots, sb.res)) != RS_OK) return r;
-    launches += 2;
+    launches += 3;
   }
   CK(cudaEventRecord(ctx->ev[3], ctx->st), "event");
   CK(cudaMemcpyAsync(results_host, sb.res, nsim * sizeof(rs_replica_result), cudaMemcpyDeviceToHost,

@@ -5,7 +5,7 @@
 // c_ij = a n_ij + b + d/(C - n_ij)^2 - w_c o_ij of the §6.4 matrix; a stable
 // bucket sort of the requests by window (request order kept inside a window).
 //
-// k_poa_solve (one CTA per replica, one warp per window): OPT of the window =
+// k_poa_solve (a few CTAs per replica, one warp per window): OPT of the window =
 // minimum-cost assignment of its requests to W workers of capacity
 // max(C_j, ceil(n/W)) each (the replicated-column square matrix of §6.4).
 // Every request first takes its cheapest worker; that is optimal unless a
@@ -13,7 +13,13 @@
 // (what stays is optimal for its own subset: every row sits at its minimum)
 // and put back one at a time along a shortest augmenting path (successive
 // shortest paths), found by Bellman-Ford on the W worker nodes with edge
-// weights min over the requests at j of (c_qk - c_qj).
+// weights min over the requests at j of (c_qk - c_qj).  The edge weights are
+// kept across augmentations: a request that moves in lowers its worker's
+// weights in O(W); only a worker that lost the request behind one of its
+// minima is rescanned.
+//
+// k_poa_total (one warp per replica): the whole-run PoA, sum of observed
+// latency over sum of OPT across the replica's windows.
 #include "rs_device.cuh"
 
 namespace rs {
@@ -152,9 +158,41 @@ struct PoaWarpShared {
   int counts[POA_WMAX];
   double wmin[POA_WMAX][POA_WMAX];
   int wrow[POA_WMAX][POA_WMAX];
+  int mv_row[POA_WMAX + 1], mv_to[POA_WMAX + 1];   // requests moved by the last augmentation
+  int dirty[POA_WMAX];                             // workers whose edge weights need a rescan
+  int nmv;
   double num, opt;
   int err;
 };
+
+// Edge weights out of worker j: for every k, the cheapest move of a request now
+// at j to k, min over those requests of c_qk - c_qj (ties: lowest row).
+__device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffers& b,
+                                               int64_t scratch_base, int64_t base, int64_t m,
+                                               int W, int j, int lane) {
+  double lm[POA_WMAX];
+  int lr[POA_WMAX];
+  for (int k = 0; k < W; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
+  for (int64_t r = lane; r < m; r += 32) {
+    if (b.asg[base + r] != j) continue;
+    const double* cr = b.cost + (scratch_base + b.order[base + r]) * W;
+    const double cj = cr[j];
+    for (int k = 0; k < W; k++) {
+      const double v = __dsub_rn(cr[k], cj);
+      if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
+    }
+  }
+  for (int k = 0; k < W; k++) {
+    double v = lm[k];
+    int rr = lr[k];
+    for (int o = 16; o > 0; o >>= 1) {
+      const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
+      const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
+      if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
+    }
+    if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
+  }
+}
 
 struct PoaSolveShared {
   PoaWarpShared w[NT_POA / 32];
@@ -170,21 +208,13 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
   __shared__ PoaSolveShared P;
   const PoaProblem pr = probs[blockIdx.x];
   const int64_t nw = b.nwin[blockIdx.x];
-  if (nw < 0) {
-    if (threadIdx.x == 0) {
-      b.total[blockIdx.x] = __longlong_as_double(0x7FF8000000000000ll);
-      if (b.res) {
-        b.res[blockIdx.x].poa_total = __longlong_as_double(0x7FF8000000000000ll);
-        b.res[blockIdx.x].n_windows = nw;
-      }
-    }
-    return;
-  }
+  if (nw < 0) return;   // k_poa_total reports it
   const int W = mc.W;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   PoaWarpShared& S = P.w[warp];
   const int64_t* wst = b.wstart + pr.win_base + blockIdx.x;
-  for (int64_t w = warp; w < nw; w += NT_POA / 32) {
+  const int64_t nwarps = (int64_t)gridDim.y * (NT_POA / 32);
+  for (int64_t w = (int64_t)blockIdx.y * (NT_POA / 32) + warp; w < nw; w += nwarps) {
     const int64_t s0 = wst[w];
     const int64_t m = wst[w + 1] - s0;
     const int64_t base = pr.scratch_base + s0;   // window rows in order[], asg[]
@@ -233,35 +263,11 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       }
       __syncwarp();
       const int64_t nrem = (int64_t)S.num;
+      for (int j = 0; j < W; j++) poa_edges_from(S, b, pr.scratch_base, base, m, W, j, lane);
+      __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
         const double* c0 = b.cost + (pr.scratch_base + b.order[base + r0]) * W;
-        // edge weights j -> k: cheapest move of a request now at j to k
-        for (int j = 0; j < W; j++) {
-          double lm[POA_WMAX];
-          int lr[POA_WMAX];
-          for (int k = 0; k < W; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
-          for (int64_t r = lane; r < m; r += 32) {
-            if (b.asg[base + r] != j) continue;
-            const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
-            const double cj = cr[j];
-            for (int k = 0; k < W; k++) {
-              const double v = __dsub_rn(cr[k], cj);
-              if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
-            }
-          }
-          for (int k = 0; k < W; k++) {
-            double v = lm[k];
-            int rr = lr[k];
-            for (int o = 16; o > 0; o >>= 1) {
-              const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
-              const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
-              if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
-            }
-            if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
-          }
-        }
-        __syncwarp();
         if (lane == 0) {
           double dist[POA_WMAX];
           int pred[POA_WMAX];
@@ -281,21 +287,56 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
           int tgt = -1;
           for (int k = 0; k < W; k++)
             if (S.counts[k] < capw && (tgt < 0 || dist[k] < dist[tgt])) tgt = k;
+          int nmv = 0;
+          for (int j = 0; j < W; j++) S.dirty[j] = 0;
           if (tgt < 0) {
             S.err = 1;
           } else {
+            // walk the path back from its end: each edge j -> k moves the
+            // request behind S.wrow[j][k] from j to k
             int k = tgt, steps = 0;
             while (pred[k] >= 0 && steps <= W) {
               const int j = pred[k];
-              b.asg[base + S.wrow[j][k]] = k;
+              const int r = S.wrow[j][k];
+              S.mv_row[nmv] = r;
+              S.mv_to[nmv++] = k;
+              // j loses r: its weights need a rescan where r was the minimum
+              for (int k2 = 0; k2 < W; k2++) S.dirty[j] |= S.wrow[j][k2] == r;
               k = j;
               steps++;
             }
-            if (steps > W) S.err = 1;
-            b.asg[base + r0] = k;
-            S.counts[tgt]++;
+            if (steps > W) {
+              S.err = 1;
+              nmv = 0;
+            } else {
+              for (int t = 0; t < nmv; t++) b.asg[base + S.mv_row[t]] = S.mv_to[t];
+              b.asg[base + r0] = k;
+              S.mv_row[nmv] = (int)r0;
+              S.mv_to[nmv++] = k;
+              S.counts[tgt]++;
+            }
           }
+          // requests that moved in lower their new worker's weights
+          for (int t = 0; t < nmv; t++) {
+            const int r = S.mv_row[t], to = S.mv_to[t];
+            const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
+            const double ct = cr[to];
+            for (int k2 = 0; k2 < W; k2++) {
+              if (k2 == to) continue;
+              const double v = __dsub_rn(cr[k2], ct);
+              const int wr = S.wrow[to][k2];
+              if (wr < 0 || v < S.wmin[to][k2] || (v == S.wmin[to][k2] && r < wr)) {
+                S.wmin[to][k2] = v;
+                S.wrow[to][k2] = r;
+              }
+            }
+          }
+          S.nmv = nmv;
         }
+        __syncwarp();
+        if (S.err) break;
+        for (int j = 0; j < W; j++)
+          if (S.dirty[j]) poa_edges_from(S, b, pr.scratch_base, base, m, W, j, lane);
         __syncwarp();
       }
     }
@@ -313,19 +354,30 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
     }
     __syncwarp();
   }
-  __syncthreads();
-  if (threadIdx.x == 0) {
+}
+
+// Whole-run PoA of every replica: one warp per replica, windows summed in
+// order by lane 0 (the same order as a sequential sum).
+__global__ void __launch_bounds__(NT_POA) k_poa_total(int nprob, PoaBuffers b,
+                                                      const PoaProblem* __restrict__ probs) {
+  const int lane = threadIdx.x & 31;
+  const int p = (int)(((int64_t)blockIdx.x * NT_POA + threadIdx.x) >> 5);
+  if (p >= nprob || lane != 0) return;
+  const PoaProblem pr = probs[p];
+  const int64_t nw = b.nwin[p];
+  double tot = __longlong_as_double(0x7FF8000000000000ll);
+  if (nw >= 0) {
     double tn = 0.0, to = 0.0;
     for (int64_t w = 0; w < nw; w++) {
       tn += b.wnum[pr.win_base + w];
       to += b.wopt[pr.win_base + w];
     }
-    const double tot = to > 0.0 ? tn / to : 0.0;
-    b.total[blockIdx.x] = tot;
-    if (b.res) {
-      b.res[blockIdx.x].poa_total = tot;
-      b.res[blockIdx.x].n_windows = nw;
-    }
+    tot = to > 0.0 ? tn / to : 0.0;
+  }
+  b.total[p] = tot;
+  if (b.res) {
+    b.res[p].poa_total = tot;
+    b.res[p].n_windows = nw;
   }
 }
 
@@ -335,7 +387,15 @@ cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
   k_poa_prep<<<nprob, NT_POA, 0, st>>>(d_prob, b, mc);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_poa_solve<<<nprob, NT_POA, 0, st>>>(d_prob, b, mc);
+  // a few CTAs per replica so that a handful of replicas still fill the GPU
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int split = (4 * sms + nprob - 1) / nprob;
+  split = split < 1 ? 1 : (split > 16 ? 16 : split);
+  k_poa_solve<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  k_poa_total<<<(nprob + NT_POA / 32 - 1) / (NT_POA / 32), NT_POA, 0, st>>>(nprob, b, d_prob);
   return cudaGetLastError();
 }
 
