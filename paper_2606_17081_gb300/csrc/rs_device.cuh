@@ -47,6 +47,19 @@ __device__ __forceinline__ uint64_t chain_step(uint64_t prev, uint64_t gk) {
   return h < 2 ? h + 2 : h;
 }
 
+// ---------------------------------------------------------------- async copies
+
+// 8-byte global -> shared copy that completes in the background (both
+// addresses 8-byte aligned); cp_async_wait_all waits for this thread's copies.
+__device__ __forceinline__ void cp_async8(void* smem_dst, const void* gmem_src) {
+  const unsigned d = (unsigned)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;\n" ::: "memory");
+}
+
 // ---------------------------------------------------------------- Philox4x32-10
 
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
@@ -336,7 +349,7 @@ struct UpdateScratch {
 };
 
 struct UpdateShared {   // small shared scalars of the update
-  int n_absent, n_ins, reclaimed, n_victims, slow, err, dup;
+  int n_absent, n_ins, reclaimed, n_victims, n_tomb, slow, err, dup;
   uint32_t pmin, gathered;
 };
 
@@ -425,6 +438,7 @@ __device__ __forceinline__ void update_reset(UpdateShared* us) {
   us->n_ins = 0;
   us->reclaimed = 0;
   us->n_victims = 0;
+  us->n_tomb = 0;
   us->slow = 0;
   us->dup = 0;
   us->pmin = STAMP_NONE;
@@ -506,6 +520,11 @@ __device__ __forceinline__ void cache_lookup_captured(const TableView& t, const 
 
 // Gathers live log entries starting at meta->head until `want` are held
 // (or the log ends).  Continues from us->gathered entries already held.
+// Beside each entry's stamp, the first entries' buckets are read too (same
+// round trip): an entry whose bucket holds an EMPTY key is marked
+// VSLOT_EMPTY_OK, and evicting it may leave an EMPTY instead of a tombstone.
+constexpr uint32_t VSLOT_EMPTY_OK = 0x80000000u;
+
 template <int NT>
 __device__ __forceinline__ void gather_live(const TableView& t, const CacheMeta* meta, uint32_t* pos,
                             uint32_t want, UpdateScratch& sc, UpdateShared* us, int* warp_tot) {
@@ -514,16 +533,25 @@ __device__ __forceinline__ void gather_live(const TableView& t, const CacheMeta*
   uint32_t p0 = *pos;
   while (have < want && p0 < T) {
     const uint32_t p = p0 + threadIdx.x;
-    bool live = false;
+    bool live = false, empty_ok = false;
     uint32_t x = 0;
     if (p < T) {
       x = t.log[p & t.rmask];
+      // buckets of the entries likely to become victims (dead entries
+      // interleave, hence the margin)
+      const bool look = threadIdx.x < 2 * (want - have) + 32;
+      uint64_t v[BUCKET];
+      if (look) ld_bucket(t.keys, x / BUCKET, v);
       live = __ldcg(t.stamp + x) == p;
+      if (look) {
+#pragma unroll
+        for (int q = 0; q < BUCKET; q++) empty_ok |= v[q] == KEY_EMPTY;
+      }
     }
     int tot;
     const int r = cta_rank<NT>(live, warp_tot, &tot);
     if (live && have + r < want) {
-      sc.vslot[have + r] = x;
+      sc.vslot[have + r] = x | (empty_ok ? VSLOT_EMPTY_OK : 0u);
       sc.vt[have + r] = p;
     }
     have = min(want, have + (uint32_t)tot);
@@ -632,12 +660,22 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
     grp_bar<NT>();
   }
   const int E = us->n_victims;
-  // evictions first (tombstones), then inserts, then stamps and log
+  // evictions first, then inserts, then stamps and log.  A lookup scans whole
+  // buckets and stops at the first bucket holding an EMPTY key; a bucket that
+  // holds one has held one since the last rebuild (slots only become EMPTY
+  // here, and only in such buckets), so no key has overflowed past it and the
+  // evicted key may become EMPTY.  Elsewhere it becomes a tombstone.
+  int ntomb = 0;
   for (int v = threadIdx.x; v < E; v += NT) {
-    const uint32_t x = sc.vslot[sc.victim[v]];
-    t.keys[x] = KEY_TOMB;
+    const uint32_t xv = sc.vslot[sc.victim[v]];
+    const uint32_t x = xv & ~VSLOT_EMPTY_OK;
+    const bool tomb = (xv & VSLOT_EMPTY_OK) == 0u;
+    t.keys[x] = tomb ? KEY_TOMB : KEY_EMPTY;
     t.stamp[x] = STAMP_NONE;
+    ntomb += tomb;
   }
+  ntomb = __reduce_add_sync(FULL_MASK, (unsigned)ntomb);
+  if ((threadIdx.x & 31) == 0 && ntomb) atomicAdd(&us->n_tomb, ntomb);
   grp_bar<NT>();
   const uint32_t T = meta->T;
   int nins = 0, recl = 0, err = 0;
@@ -675,7 +713,7 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
   if (err) us->err = RS_ERR_TIMEOUT;
   grp_bar<NT>();
   if (threadIdx.x == 0) {
-    meta->tombs = meta->tombs + (uint32_t)E - (uint32_t)us->reclaimed;
+    meta->tombs = meta->tombs + (uint32_t)us->n_tomb - (uint32_t)us->reclaimed;
     meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
     if (E > 0) meta->head = sc.vt[sc.victim[E - 1]] + 1;
     meta->T = T + (uint32_t)nb;

@@ -114,8 +114,16 @@ struct ReqState {
   float tau, omega;
 };
 
+// Request i's scalars as read from the trace (control thread).
+struct RawReq {
+  int64_t o0, o1;
+  double rel;
+  int O;
+};
+
 struct SimScalars {
   ReqState q[2];
+  RawReq nraw;                 // the request after the next one to arrive, as read
   double prev_arrival, min_ft, tick_t, lastL, ewma, sum_ttft, sum_e2e, makespan;
   int64_t next_tick, np;
   int64_t near_ties, exact_ties, sampled, near_bd, hit_blocks, inserted, evicted, slow, rebuilds;
@@ -615,7 +623,6 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   c.f_oitl[f] = q.oitl;
   c.wA[js] += q.blk;
   S.in_flight++;
-  S.hit_blocks += c.wm[js];
   const int64_t row = c.d->rec_base + i;
   c.b->rec.worker[row] = js;
   c.b->rec.arrival[row] = q.a;
@@ -630,13 +637,6 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   S.prev_arrival = q.a;
   S.n_routed++;
 }
-
-// Request i's scalars as read from the trace (control thread).
-struct RawReq {
-  int64_t o0, o1;
-  double rel;
-  int O;
-};
 
 __device__ __forceinline__ RawReq read_request(const SimCtx& c, int64_t i) {
   RawReq r;
@@ -787,6 +787,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   if (n > 0) {
     if (threadIdx.x == CTL) {
       load_request(c, S.q[0], read_request(c, 0));
+      if (n > 1) S.nraw = read_request(c, 1);
       S.evres = events_advance(c, S.q[0]);
       if (S.evres == 0) regime_params(c, S.q[0]);
       update_reset(&S.us);
@@ -838,6 +839,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
         const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
         float* ds = b.dstat + row * 6;
         S.jstar = select_worker(c.wcost, W, tau, u24, ds + 2);
+        S.hit_blocks += c.wm[S.jstar];
         if (tau > 0.0f) S.sampled++;
         else ds[3] = -1.0f;   // no draw
       }
@@ -891,22 +893,34 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
     } else {
       // ---- control warp: request i's load and latency; request i+1's arrival
       ReqState& nq = S.q[p ^ 1];
-      if (lane == 0) {
-        // the next request's loads go out first; their latency overlaps the bookkeeping
-        RawReq raw;
-        if (i + 1 < n) raw = read_request(c, i + 1);
-        book_request(c, S.q[p], i);
-        if (i + 1 < n) load_request(c, nq, raw);
+      const bool more = i + 1 < n;
+      if (more) {
+        // request i+1's hashes: asynchronous copies into the other staging
+        // buffer, waited for before the next barrier
+        const int64_t nbn = (S.nraw.o1 - S.nraw.o0) >> 4;
+        if (nbn <= (int64_t)L.g.K) {
+          const uint64_t* src = d.hashes + (S.nraw.o0 >> 4);
+          uint64_t* dst = c.hbuf(p ^ 1);
+          for (int k = lane; k < (int)nbn; k += 32) cp_async8(dst + k, src + k);
+        }
+        if (lane == 0) load_request(c, nq, S.nraw);
       }
       __syncwarp();
-      if (i + 1 < n) {
-        stage_hashes(c, nq, c.hbuf(p ^ 1), lane);
-        probe_setup(c, nq, lane);
-        if (lane == 0) {
+      if (more) probe_setup(c, nq, lane);
+      if (lane == 0) {
+        // the loads of the request after next go out first; their latency
+        // overlaps the bookkeeping and the events
+        RawReq raw2;
+        const bool more2 = i + 2 < n;
+        if (more2) raw2 = read_request(c, i + 2);
+        book_request(c, S.q[p], i);
+        if (more) {
           S.evres = events_advance(c, nq);
           if (S.evres == 0) regime_params(c, nq);
         }
+        if (more2) S.nraw = raw2;
       }
+      cp_async_wait_all();
     }
   }
   __syncthreads();
