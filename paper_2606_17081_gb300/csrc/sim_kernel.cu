@@ -473,10 +473,11 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
 // m_j: leading blocks of the prompt found in worker j's cache, for every j
 // (all threads).  Rounds of CH blocks per still-undecided worker; a worker is
 // decided once a miss is found below the round's end.
+template <int NT>
 __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
-  const int CH = max(32, ((4 * NT_SIM) / W) & ~31);
+  const int CH = max(32, ((4 * NT) / W) & ~31);
   int c0 = 0;
   int err = 0;
   unsigned cnt = 0;
@@ -484,9 +485,9 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
     const int nopen = S.nopen;
     const int len = min(CH, nb - c0);
     const int total = len > 0 ? nopen * len : 0;
-    const int rounds = (total + NT_SIM - 1) / NT_SIM;
+    const int rounds = (total + NT - 1) / NT;
     for (int q = 0; q < rounds; q++) {        // uniform trip count: warp reductions below
-      const int it = q * NT_SIM + threadIdx.x;
+      const int it = q * NT + threadIdx.x;
       int jj = -1, miss = 0x7FFFFFFF;
       if (it < total) {
         jj = c.wopen[it / len];
@@ -501,7 +502,7 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
       if (jj >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
         atomicMin(&c.wm[jj], m);
     }
-    __syncthreads();
+    grp_bar<NT>();
     c0 += CH;
     if (threadIdx.x == 0) {
       int no = 0;
@@ -510,7 +511,7 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
           if (c.wm[j] >= c0) c.wopen[no++] = j;
       S.nopen = no;
     }
-    __syncthreads();
+    grp_bar<NT>();
     if (S.nopen == 0) break;
   }
   cnt = __reduce_add_sync(FULL_MASK, cnt);
@@ -522,18 +523,19 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
 // PROBE_CAP): each thread issues the first-bucket loads of PROBE_ILP pairs
 // before resolving them, and the slot found (or the first free slot of the
 // probe path) is kept for the chosen worker's update.
+template <int NT>
 __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
   const int total = W * nb;
   int err = 0;
-  for (int base = 0; base < total; base += NT_SIM * PROBE_ILP) {   // uniform
+  for (int base = 0; base < total; base += NT * PROBE_ILP) {   // uniform
     int jj[PROBE_ILP], kk[PROBE_ILP];
     uint64_t v[PROBE_ILP][BUCKET];
     uint32_t bk[PROBE_ILP];
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
-      const int it = base + r * NT_SIM + threadIdx.x;
+      const int it = base + r * NT + threadIdx.x;
       jj[r] = -1;
       if (it < total) {
         const int j = it / nb;
@@ -546,7 +548,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
     }
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
-      const int it = base + r * NT_SIM + threadIdx.x;
+      const int it = base + r * NT + threadIdx.x;
       int miss = 0x7FFFFFFF;
       if (jj[r] >= 0) {
         const uint64_t h = hbuf[kk[r]];
@@ -568,7 +570,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   }
   if (threadIdx.x == 0) S.probes += (unsigned long long)total;
   if (err) S.status = RS_ERR_TIMEOUT;
-  __syncthreads();
+  grp_bar<NT>();
 }
 
 // Cache update of the chosen worker (update group, warps 0-6).
@@ -788,8 +790,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
     if (threadIdx.x == CTL) {
       load_request(c, S.q[0], read_request(c, 0));
       if (n > 1) S.nraw = read_request(c, 1);
-      S.evres = events_advance(c, S.q[0]);
-      if (S.evres == 0) regime_params(c, S.q[0]);
+      S.evres = 0;
       update_reset(&S.us);
       S.us.err = 0;
     }
@@ -801,16 +802,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   }
   for (int64_t i = 0; i < n; i++) {
     const int p = (int)(i & 1);
-    // ---- controller samples that need the CTA, before request i arrives
-    for (;;) {
-      __syncthreads();
-      if (S.evres == 0) break;
-      tick_cta(c);
-      if (threadIdx.x == CTL) {
-        S.evres = events_advance(c, S.q[p]);
-        if (S.evres == 0) regime_params(c, S.q[p]);
-      }
-    }
+    __syncthreads();
     if (S.status != RS_OK) break;
     const int nb = S.q[p].nb;
     if (nb > (int)L.g.K) {
@@ -821,9 +813,27 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
     const bool full = S.q[p].full;
     const uint64_t* hb = c.hbuf(p);
     const int64_t row = d.rec_base + i;
-    // ---- cached prefix on every worker
-    if (full) probe_full(c, hb, nb);
-    else probe_prefixes(c, hb, nb);
+    if (warp < NT_SIM / 32 - 1) {
+      // ---- cached prefix on every worker (warps 0-6)
+      if (full) probe_full<NT_UPD>(c, hb, nb);
+      else probe_prefixes<NT_UPD>(c, hb, nb);
+    } else if (lane == 0) {
+      // ---- control thread, at the same time: completions and controller
+      // samples up to request i's arrival (the probe needs none of them)
+      S.evres = events_advance(c, S.q[p]);
+      if (S.evres == 0) regime_params(c, S.q[p]);
+    }
+    __syncthreads();
+    // ---- controller samples whose window needs the CTA (P99 of Eq. (10))
+    while (S.evres != 0) {
+      tick_cta(c);
+      if (threadIdx.x == CTL) {
+        S.evres = events_advance(c, S.q[p]);
+        if (S.evres == 0) regime_params(c, S.q[p]);
+      }
+      __syncthreads();
+    }
+    if (S.status != RS_OK) break;
     // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
     if (warp == 0) {
       const float om = S.q[p].omega, tau = S.q[p].tau;
@@ -891,7 +901,8 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       // ---- the chosen worker's LRU cache (warps 0-6)
       update_chosen(c, hb, js, nb, full);
     } else {
-      // ---- control warp: request i's load and latency; request i+1's arrival
+      // ---- control warp: request i's load and latency; request i+1's
+      // scalars, probe state and block hashes
       ReqState& nq = S.q[p ^ 1];
       const bool more = i + 1 < n;
       if (more) {
@@ -914,10 +925,6 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
         const bool more2 = i + 2 < n;
         if (more2) raw2 = read_request(c, i + 2);
         book_request(c, S.q[p], i);
-        if (more) {
-          S.evres = events_advance(c, nq);
-          if (S.evres == 0) regime_params(c, nq);
-        }
         if (more2) S.nraw = raw2;
       }
       cp_async_wait_all();
