@@ -236,19 +236,28 @@ __device__ __forceinline__ uint32_t home_bucket(uint64_t h, uint32_t bmask) {
   return (uint32_t)(h ^ (h >> 32)) & bmask;
 }
 
-__device__ __forceinline__ ulonglong2 ld_keys2(const uint64_t* p) {
-  return __ldcg(reinterpret_cast<const ulonglong2*>(p));
+// Four keys (one 32-byte sector) in one 256-bit load through L2; p 32-byte
+// aligned (buckets are 64-byte aligned: the key arrays start on 256-byte
+// boundaries and every table holds a multiple of 8 slots).
+__device__ __forceinline__ void ld_keys4(const uint64_t* p, uint64_t& a, uint64_t& b, uint64_t& c,
+                                         uint64_t& d) {
+  unsigned long long x0, x1, x2, x3;
+  asm("ld.global.cg.v4.u64 {%0, %1, %2, %3}, [%4];"
+               : "=l"(x0), "=l"(x1), "=l"(x2), "=l"(x3)
+               : "l"(p));
+  a = x0;
+  b = x1;
+  c = x2;
+  d = x3;
 }
 
-// The BUCKET keys of bucket b (four independent 16-byte loads).
+// The BUCKET keys of bucket b: two independent 256-bit loads, one request
+// per 32-byte sector.
 __device__ __forceinline__ void ld_bucket(const uint64_t* keys, uint32_t b, uint64_t (&v)[BUCKET]) {
   const uint64_t* p = keys + (size_t)BUCKET * b;
-#pragma unroll
-  for (int q = 0; q < BUCKET / 2; q++) {
-    const ulonglong2 x = ld_keys2(p + 2 * q);
-    v[2 * q] = x.x;
-    v[2 * q + 1] = x.y;
-  }
+  static_assert(BUCKET == 8, "two 32-byte sectors per bucket");
+  ld_keys4(p, v[0], v[1], v[2], v[3]);
+  ld_keys4(p + 4, v[4], v[5], v[6], v[7]);
 }
 
 // Slot holding h, or SLOT_NONE; *free_slot = the first EMPTY or TOMB slot of
@@ -487,6 +496,22 @@ __device__ __forceinline__ void cache_lookup_all(const TableView& t, const uint6
       if (sc.owner[k] >= 0) sc.dupset[sc.owner[k]] = 0ull;
 }
 
+// Claims table slot x for one insert of this update in the shared-memory set
+// (keys x + 1; the set is empty between uses).  Returns the set position
+// claimed, or -1 when another block of the request claimed x first.
+__device__ __forceinline__ int32_t slot_claim(UpdateScratch& sc, uint32_t x) {
+  const unsigned long long key = (unsigned long long)x + 1ull;
+  uint32_t d = (x * 0x9E3779B1u) & sc.dupmask;
+  for (uint32_t it = 0; it <= sc.dupmask; it++) {
+    const unsigned long long prev = atomicCAS(
+        reinterpret_cast<unsigned long long*>(sc.dupset + d), 0ull, key);
+    if (prev == 0ull) return (int32_t)d;
+    if (prev == key) return -1;
+    d = (d + 1) & sc.dupmask;
+  }
+  return -1;
+}
+
 // The chosen worker's lookup from slots captured by the probe (no table
 // reads): stamps of present blocks, absent count, insert positions.
 template <int NT>
@@ -565,24 +590,88 @@ __device__ __forceinline__ void gather_live(const TableView& t, const CacheMeta*
   grp_bar<NT>();
 }
 
+// The chosen worker's update inputs from the probe's captured slots, in one
+// round of loads: the stamps of the present blocks and, for the nabs - free
+// victims this request needs, the first log entries after the head with
+// their stamps and buckets (as gather_live's first pass).  us must be reset.
+template <int NT>
+__device__ __forceinline__ void cache_prepare_captured(const TableView& t, const CacheMeta* meta,
+                                                       uint32_t K, const uint32_t* pslot,
+                                                       const uint32_t* pfree, int nb, int nabs,
+                                                       UpdateScratch& sc, UpdateShared* us,
+                                                       int* warp_tot, uint32_t* scan_pos) {
+  const uint32_t size = meta->size, T = meta->T, head = meta->head;
+  const uint32_t free_slots = K - size;
+  const uint32_t E0 = (uint32_t)nabs > free_slots ? (uint32_t)nabs - free_slots : 0u;
+  // the log entries go out first ...
+  const uint32_t p = head + threadIdx.x;
+  const bool gp = E0 > 0 && p < T;
+  uint32_t x = 0;
+  if (gp) x = t.log[p & t.rmask];
+  // ... then the present blocks' stamps, which do not depend on them
+  uint32_t pmin = STAMP_NONE;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const uint32_t sl = pslot[k];
+    sc.slot[k] = sl;
+    sc.fslot[k] = pfree[k];
+    sc.evk[k] = 0;
+    uint32_t st = STAMP_NONE;
+    if (sl != SLOT_NONE) {
+      st = __ldcg(t.stamp + sl);
+      pmin = min(pmin, st);
+    }
+    sc.pst[k] = st;
+  }
+  // stamps and buckets of the log entries
+  bool live = false, empty_ok = false;
+  if (gp) {
+    const bool look = threadIdx.x < 2 * E0 + 32;
+    uint64_t v[BUCKET];
+    if (look) ld_bucket(t.keys, x / BUCKET, v);
+    live = __ldcg(t.stamp + x) == p;
+    if (look) {
+#pragma unroll
+      for (int q = 0; q < BUCKET; q++) empty_ok |= v[q] == KEY_EMPTY;
+    }
+  }
+  pmin = __reduce_min_sync(FULL_MASK, pmin);
+  if ((threadIdx.x & 31) == 0 && pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  int tot;
+  const int r = cta_rank<NT>(live, warp_tot, &tot);
+  if (live && (uint32_t)r < E0) {
+    sc.vslot[r] = x | (empty_ok ? VSLOT_EMPTY_OK : 0u);
+    sc.vt[r] = p;
+  }
+  if (threadIdx.x == 0) {
+    us->n_absent = nabs;
+    us->gathered = min(E0, (uint32_t)tot);
+    *scan_pos = head + NT;
+  }
+  grp_bar<NT>();
+}
+
 // Applies one request's block list to the chosen worker's cache: exact LRU
 // semantics of touching blocks 0..nb-1 in order (hits -> most recent, misses
 // inserted, the least-recent entry evicted whenever the cache is full).
 // Returns through us: n_victims, n_ins; updates meta.  CTA-wide.
+// With `pregathered`, cache_prepare_captured has already gathered the first
+// entries (us->gathered, *scan_pos).
 template <int NT>
 __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta, uint32_t K, const uint64_t* hbuf,
                             int nb, UpdateScratch& sc, UpdateShared* us, int* warp_tot,
-                            uint32_t* scan_pos) {
+                            uint32_t* scan_pos, bool pregathered = false) {
   const uint32_t size = meta->size;
   const int nabs = us->n_absent;
   const uint32_t free_slots = K - size;
   const uint32_t E0 = (uint32_t)nabs > free_slots ? (uint32_t)nabs - free_slots : 0u;
-  if (threadIdx.x == 0) {
-    us->gathered = 0;
-    *scan_pos = meta->head;
+  if (!pregathered) {
+    if (threadIdx.x == 0) {
+      us->gathered = 0;
+      *scan_pos = meta->head;
+    }
+    grp_bar<NT>();
   }
-  grp_bar<NT>();
-  if (E0 > 0) gather_live<NT>(t, meta, scan_pos, E0, sc, us, warp_tot);
+  if (E0 > 0 && us->gathered < E0) gather_live<NT>(t, meta, scan_pos, E0, sc, us, warp_tot);
   if (E0 > 0 && us->gathered < E0) {   // fewer live entries than the size says
     if (threadIdx.x == 0) us->err = RS_ERR_TIMEOUT;
     grp_bar<NT>();
@@ -679,25 +768,40 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
   grp_bar<NT>();
   const uint32_t T = meta->T;
   int nins = 0, recl = 0, err = 0;
+  // inserts at the positions the lookup saw free: this CTA alone writes the
+  // table, so a shared-memory claim per slot settles blocks that saw the same
+  // position and the key is stored plainly; the others insert after the
+  // barrier, along their probe path
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    if (!sc.kind[k]) continue;
+    const uint32_t fr = sc.fslot[k];
+    uint32_t sl = SLOT_NONE;
+    int32_t cl = -1;
+    if (fr != SLOT_NONE) {
+      const uint32_t x = fr & ~FREE_TOMB;
+      cl = slot_claim(sc, x);
+      if (cl >= 0) {
+        t.keys[x] = hbuf[k];
+        sl = x;
+        recl += (fr & FREE_TOMB) != 0;
+      }
+    }
+    sc.slot[k] = sl;
+    sc.pst[k] = (uint32_t)cl;   // pst is not needed past the decision: the claim to release
+    nins++;
+  }
+  grp_bar<NT>();
   for (int k = threadIdx.x; k < nb; k += NT) {
     uint32_t sl = sc.slot[k];
     if (sc.kind[k]) {
-      int wt = 0;
-      const uint32_t fr = sc.fslot[k];
-      sl = SLOT_NONE;
-      if (fr != SLOT_NONE) {   // the position the lookup saw free: one CAS
-        const uint32_t x = fr & ~FREE_TOMB;
-        const unsigned long long want = (fr & FREE_TOMB) ? KEY_TOMB : KEY_EMPTY;
-        if (atomicCAS(reinterpret_cast<unsigned long long*>(t.keys + x), want,
-                      (unsigned long long)hbuf[k]) == want) {
-          sl = x;
-          wt = (fr & FREE_TOMB) != 0;
-        }
+      const int32_t cl = (int32_t)sc.pst[k];
+      if (cl >= 0) sc.dupset[cl] = 0ull;
+      if (sl == SLOT_NONE) {
+        int wt = 0;
+        sl = table_insert(t, hbuf[k], &wt, &err);
+        recl += wt;
+        sc.slot[k] = sl;
       }
-      if (sl == SLOT_NONE) sl = table_insert(t, hbuf[k], &wt, &err);
-      nins++;
-      recl += wt;
-      sc.slot[k] = sl;
     }
     if (sl != SLOT_NONE) {
       t.stamp[sl] = T + (uint32_t)k;

@@ -37,7 +37,7 @@ struct SimLayout {
   size_t ftab, wwco, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
   size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
-  size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen;
+  size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen, wabs;
   size_t kind, evk, touched;
   size_t total;
   uint32_t dupmask;
@@ -89,6 +89,7 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(wm, 4 * (size_t)W, 4)
   TAKE(wcost, 4 * (size_t)W, 4)
   TAKE(wopen, 4 * (size_t)W, 4)
+  TAKE(wabs, 4 * (size_t)W, 4)
   TAKE(kind, nb, 1)
   TAKE(evk, nb, 1)
   TAKE(touched, nv, 1)
@@ -131,7 +132,7 @@ struct SimScalars {
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild;
+  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, nabs;
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
@@ -151,7 +152,7 @@ struct SimCtx {
   uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
-  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *dclaim;
+  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs, *dclaim;
   uint32_t *pslot, *pfree;
   int64_t* wA;
   float* wcost;
@@ -564,8 +565,11 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
       }
       const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
       const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
-      if (jj[r] >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
+      const unsigned nab = __popc(__ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp);
+      if (jj[r] >= 0 && (__ffs(grp) - 1) == (int)(threadIdx.x & 31) && nab) {
         atomicMin(&c.wm[jj[r]], m);
+        atomicAdd(&c.wabs[jj[r]], (int)nab);   // absent blocks, for the update's victim count
+      }
     }
   }
   if (threadIdx.x == 0) S.probes += (unsigned long long)total;
@@ -580,13 +584,7 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
   CacheMeta* meta = &c.wmeta[j];
-  if (threadIdx.x == 0) {
-    const uint64_t span = (uint64_t)meta->T - meta->head + (uint64_t)nb;
-    S.rebuild = span > g.R || meta->tombs > g.slots / 8 || (uint64_t)meta->T + nb > STAMP_LIMIT;
-  }
-  for (int k = threadIdx.x; k < nb; k += NT_UPD)   // release the duplicate detector
-    if (c.dclaim[k] >= 0) c.sc.dupset[c.dclaim[k]] = 0ull;
-  grp_bar<NT_UPD>();
+  // (the duplicate detector was released and the rebuild decided at the choice)
   if (S.us.dup) {
     if (threadIdx.x == 0) S.status = RS_ERR_COLLISION;
     return;
@@ -595,12 +593,14 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
     if (threadIdx.x == 0) S.rebuilds++;
   }
-  if (full && !S.rebuild)
-    cache_lookup_captured<NT_UPD>(tv, c.pslot + (size_t)j * nb, c.pfree + (size_t)j * nb, nb,
-                                  c.sc, &S.us);
+  const bool captured = full && !S.rebuild;
+  if (captured)
+    cache_prepare_captured<NT_UPD>(tv, meta, g.K, c.pslot + (size_t)j * nb,
+                                   c.pfree + (size_t)j * nb, nb, S.nabs, c.sc, &S.us,
+                                   S.warp_tot, &S.scan_pos);
   else
     cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
-  cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos);
+  cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos, captured);
   if (threadIdx.x == 0) {
     if (S.us.err) S.status = S.us.err;
     S.inserted += S.us.n_ins;
@@ -682,6 +682,7 @@ __device__ __forceinline__ void probe_setup(SimCtx& c, const ReqState& q, int la
   for (int j = lane; j < W; j += 32) {
     c.wm[j] = q.nb;
     c.wopen[j] = j;
+    c.wabs[j] = 0;
   }
   if (lane == 0) c.S->nopen = W;
 }
@@ -731,6 +732,7 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
   c.wqt = reinterpret_cast<int32_t*>(smem + lay.wqt);
   c.wm = reinterpret_cast<int32_t*>(smem + lay.wm);
   c.wopen = reinterpret_cast<int32_t*>(smem + lay.wopen);
+  c.wabs = reinterpret_cast<int32_t*>(smem + lay.wabs);
   c.wA = reinterpret_cast<int64_t*>(smem + lay.wA);
   c.wcost = reinterpret_cast<float*>(smem + lay.wcost);
   c.sc.slot = reinterpret_cast<uint32_t*>(smem + lay.slot);
@@ -848,8 +850,17 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       if (lane == 0) {
         const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
         float* ds = b.dstat + row * 6;
-        S.jstar = select_worker(c.wcost, W, tau, u24, ds + 2);
-        S.hit_blocks += c.wm[S.jstar];
+        const int js = select_worker(c.wcost, W, tau, u24, ds + 2);
+        S.jstar = js;
+        S.hit_blocks += c.wm[js];
+        // the chosen worker's absent blocks, latched before the control warp
+        // resets the probe state for the next request
+        S.nabs = c.wabs[js];
+        // the chosen worker's table: rebuild first when its log span, its
+        // tombstones or its stamps would overflow
+        const CacheMeta* mt = &c.wmeta[js];
+        const uint64_t span = (uint64_t)mt->T - mt->head + (uint64_t)nb;
+        S.rebuild = span > L.g.R || mt->tombs > L.g.slots / 8 || (uint64_t)mt->T + nb > STAMP_LIMIT;
         if (tau > 0.0f) S.sampled++;
         else ds[3] = -1.0f;   // no draw
       }
@@ -894,6 +905,9 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       int dup = 0;
       for (int k = threadIdx.x - 64; k < nb; k += NT_SIM - 96) c.dclaim[k] = dup_claim(c.sc, hb[k], &dup);
       if (dup) S.us.dup = 1;
+      asm volatile("bar.sync 2, %0;" ::"n"(NT_SIM - 96) : "memory");   // warps 2-6: all claims made
+      for (int k = threadIdx.x - 64; k < nb; k += NT_SIM - 96)
+        if (c.dclaim[k] >= 0) c.sc.dupset[c.dclaim[k]] = 0ull;
     }
     __syncthreads();
     const int js = S.jstar;
