@@ -61,7 +61,14 @@ typedef enum {
 } rs_status;
 
 enum { RS_POLICY_DYNAMO = 0,   /* Eq. (1) cost with the replica's omega, tau */
-       RS_POLICY_LOADBAL = 1   /* coordinated: Eq. (1) with omega = 0, tau = 0 */ };
+       RS_POLICY_LOADBAL = 1,  /* coordinated: Eq. (1) with omega = 0, tau = 0 */
+       /* Static counterfactual policies of the routing-baselines discussion
+        * (§9): they ignore the cache state except through P2C's cost. */
+       RS_POLICY_ROUNDROBIN = 2,   /* request i -> worker i mod W */
+       RS_POLICY_RANDOM = 3,       /* uniform: floor(u W), u = (Philox x0 >> 8) 2^-24 */
+       RS_POLICY_P2C = 4           /* power of two choices: two distinct uniform workers
+                                      (x0, x1 of one Philox draw), the lower Eq. (1)
+                                      cost wins, ties to the lower index */ };
 
 enum { RS_MEM_DEVICE = 0, RS_MEM_HOST = 1 };
 
@@ -194,6 +201,9 @@ typedef struct {
   int64_t hashed_blocks;    /* sum of nb_i (full blocks) over routed requests */
   int64_t slow_path;        /* updates that needed the exact sequential path */
   int64_t rebuilds;         /* table/log compactions */
+  double poa_static;        /* the realized assignment under the frozen cost model of
+                               §6.4: sum over windows of sum_i c_{i, worker(i)} over
+                               the sum of OPTs (the static counterfactual of §9) */
 } rs_replica_result;
 
 /* Per-request records, device memory, each pointer may be NULL.  Replica r's
@@ -273,8 +283,8 @@ rs_status route_last_timing(const rs_ctx* ctx, rs_timing* out);
  *   poa_total_dev (double) and n_windows_dev (int64): one entry each;
  *   *n_windows_dev = -1 if the records span more than n + 2 windows.
  * Returns RS_ERR_CAPACITY (before any work) when n rows of W columns need
- * more than the static array: about n * (8 W + 60) + 2 KB bytes, i.e. up to
- * roughly 390 000 rows at W = 3.  The first call on a device takes the
+ * more than the static array: about n * (8 W + 68) + 2 KB bytes, i.e. up to
+ * roughly 360 000 rows at W = 3.  The first call on a device takes the
  * array's device address (cudaGetSymbolAddress) for that device; make that
  * first call before any stream capture.  All calls on a device share the one
  * array and every call rewrites what it reads, so calls that overlap on the

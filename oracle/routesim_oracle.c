@@ -555,7 +555,7 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   const int64_t n = rep->n_req;
   if (W < 1 || cfg->block < 2 || (cfg->block & 1) || cfg->K < 1 || cfg->cap < 2 || rep->C < 1 ||
       n < 0 || !(rep->tau >= 0.0f) || !(rep->omega >= 0.0f) ||
-      (rep->policy != ORC_POLICY_DYNAMO && rep->policy != ORC_POLICY_LOADBAL)) {
+      rep->policy < ORC_POLICY_DYNAMO || rep->policy > ORC_POLICY_P2C) {
     sum->status = ORC_ERR_INVALID;
     return ORC_ERR_INVALID;
   }
@@ -670,8 +670,30 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
       if (s.prefix) s.prefix[i * W + j] = (uint16_t)m[j];
       if (s.cost) s.cost[i * W + j] = c[j];
     }
-    uint32_t u24 = tau > 0.0f ? draw_u24(rep->seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
-    int32_t jstar = orc_select(c, W, tau, u24);
+    uint32_t u24 = 0u;
+    int32_t jstar;
+    if (rep->policy == ORC_POLICY_ROUNDROBIN) {
+      /* request i goes to worker i mod W */
+      jstar = (int32_t)(i % W);
+    } else if (rep->policy == ORC_POLICY_RANDOM || rep->policy == ORC_POLICY_P2C) {
+      /* uniform workers from one Philox block of this request */
+      uint32_t ctr[4] = {(uint32_t)i, (uint32_t)((uint64_t)i >> 32), 0u, TAG_SIM};
+      uint32_t key[2] = {(uint32_t)rep->seed, (uint32_t)(rep->seed >> 32)};
+      uint32_t x[4];
+      orc_philox4x32_10(ctr, key, x);
+      int32_t j1 = (int32_t)(((uint64_t)(x[0] >> 8) * (uint64_t)W) >> 24);
+      jstar = j1;
+      if (rep->policy == ORC_POLICY_P2C && W >= 2) {
+        /* a second worker, uniform over the other W - 1 */
+        int32_t j2 = (int32_t)(((uint64_t)(x[1] >> 8) * (uint64_t)(W - 1)) >> 24);
+        if (j2 >= j1) j2++;
+        int32_t lo = j1 < j2 ? j1 : j2, hi = j1 < j2 ? j2 : j1;
+        jstar = c[hi] < c[lo] ? hi : lo;   /* lower Eq. (1) cost, ties to the lower index */
+      }
+    } else {
+      if (tau > 0.0f) u24 = draw_u24(rep->seed, (uint64_t)i, 0u, TAG_SIM);
+      jstar = orc_select(c, W, tau, u24);
+    }
     if (W >= 2) {
       int32_t b = argmin_lowest(c, W);
       float c2 = INFINITY;
@@ -681,7 +703,7 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
       if (diff <= 1e-6 * fabs((double)c2)) sum->near_ties++;
       if (c2 == c[b]) sum->exact_ties++;
     }
-    if (tau > 0.0f) {
+    if (tau > 0.0f && (rep->policy == ORC_POLICY_DYNAMO || rep->policy == ORC_POLICY_LOADBAL)) {
       sum->sampled++;
       sum->near_boundary += near_boundary(c, W, tau, u24);
     }
@@ -978,6 +1000,32 @@ int64_t orc_poa(const orc_config* cfg, int64_t n, const int32_t* worker, const d
   }
   *poa_total = to > 0.0 ? tn / to : 0.0;
   free(start); free(rows); free(fill); free(cm); free(as);
+  return nw;
+}
+
+/* The static counterfactual of the routing-baselines discussion (§9): per
+ * window of Eq. (12), the frozen cost of the assignment that was made,
+ * sum over the window's requests of c_{i, worker(i)} with the §6.4 cost
+ * matrix.  Divided by the window's OPT (orc_poa) it compares the assignment
+ * itself, without queueing, with the optimum.  Returns the windows spanned. */
+int64_t orc_static_numer(const orc_config* cfg, int64_t n, const int32_t* worker,
+                         const double* completion, const int32_t* nbt, const uint16_t* n_frozen,
+                         const uint16_t* prefix, double* numer_static, int64_t n_win_cap) {
+  const int32_t W = cfg->W;
+  int64_t nw = 0;
+  for (int64_t q = 0; q < n; q++) {
+    if (worker[q] < 0) continue;
+    int64_t w = (int64_t)floor(completion[q] / cfg->poa_window);
+    if (w + 1 > nw) nw = w + 1;
+  }
+  if (nw > n_win_cap) return ORC_ERR_INVALID;
+  for (int64_t w = 0; w < nw; w++) numer_static[w] = 0.0;
+  for (int64_t q = 0; q < n; q++) {   /* request order inside each window */
+    if (worker[q] < 0) continue;
+    int64_t w = (int64_t)floor(completion[q] / cfg->poa_window);
+    int32_t j = worker[q];
+    numer_static[w] += frozen_cost(cfg, n_frozen[q * W + j], prefix[q * W + j], nbt[q]);
+  }
   return nw;
 }
 

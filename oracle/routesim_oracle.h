@@ -42,7 +42,9 @@ enum {
   ORC_ERR_COLLISION = -7   /* two blocks of one prompt share a chained hash */
 };
 
-enum { ORC_POLICY_DYNAMO = 0, ORC_POLICY_LOADBAL = 1 };
+enum { ORC_POLICY_DYNAMO = 0, ORC_POLICY_LOADBAL = 1,
+       /* static counterfactual policies (§9, routing baselines) */
+       ORC_POLICY_ROUNDROBIN = 2, ORC_POLICY_RANDOM = 3, ORC_POLICY_P2C = 4 };
 
 typedef struct {
   int32_t W;              /* decode workers (routing-game resources) */
@@ -139,6 +141,12 @@ int64_t orc_poa(const orc_config* cfg, int64_t n, const int32_t* worker, const d
                 const double* ttft, const int32_t* nbt, const uint16_t* n_frozen,
                 const uint16_t* prefix, int32_t method, double* numer, double* opt,
                 int64_t* count, int64_t n_win_cap, double* poa_total);
+
+/* Static counterfactual (§9): per window, sum of the frozen §6.4 costs of the
+ * realized assignment, c_{i, worker(i)}.  Returns windows spanned. */
+int64_t orc_static_numer(const orc_config* cfg, int64_t n, const int32_t* worker,
+                         const double* completion, const int32_t* nbt, const uint16_t* n_frozen,
+                         const uint16_t* prefix, double* numer_static, int64_t n_win_cap);
 
 /* Min-cost assignment of n rows to W groups of `capw` identical columns;
  * cost is row-major [n*W].  method 1 Hungarian, 2 min-cost flow, 3 brute force

@@ -19,6 +19,8 @@ _LIB = os.path.join(_HERE, "liboracle.so")
 
 OK, ERR_INVALID, ERR_OOM, ERR_CAPACITY, ERR_COLLISION = 0, -1, -2, -3, -7
 POLICY_DYNAMO, POLICY_LOADBAL = 0, 1
+# static counterfactual policies of the routing-baselines discussion (§9)
+POLICY_ROUNDROBIN, POLICY_RANDOM, POLICY_P2C = 2, 3, 4
 
 
 def build_oracle(force: bool = False) -> str:
@@ -114,6 +116,7 @@ def lib():
         L.orc_select.argtypes = [C.c_void_p, C.c_int32, C.c_float, C.c_uint32]
         L.orc_simulate.restype = C.c_int32
         L.orc_poa.restype = C.c_int64
+        L.orc_static_numer.restype = C.c_int64
         L.orc_assign.restype = C.c_double
         L.orc_assign.argtypes = [C.c_void_p, C.c_int64, C.c_int32, C.c_int64, C.c_int32,
                                  C.c_void_p]
@@ -243,6 +246,34 @@ def poa(cfg: OracleConfig, rec: dict, method: int = 0):
     if nw < 0:
         raise RuntimeError(f"orc_poa failed: {nw}")
     return numer[:nw], opt[:nw], cnt[:nw], float(total.value)
+
+
+def static_numer(cfg: OracleConfig, rec: dict):
+    """Per Eq. (12) window, the frozen §6.4 cost of the realized assignment
+    (the static counterfactual of §9): sum over the window of c_{i, worker(i)}."""
+    n = rec["worker"].size
+    wk = _c(rec["worker"], np.int32)
+    ct = _c(rec["completion"], np.float64)
+    nbt = _c(rec["nbt"], np.int32)
+    nf = _c(np.asarray(rec["n_frozen"]).reshape(-1), np.uint16)
+    pf = _c(np.asarray(rec["prefix"]).reshape(-1), np.uint16)
+    routed = ct[wk >= 0]
+    cap = int(np.floor(routed.max() / cfg.poa_window)) + 2 if routed.size else 1
+    out = np.zeros(cap)
+    cc = cfg.c()
+    nw = lib().orc_static_numer(C.byref(cc), C.c_int64(n), _p(wk), _p(ct), _p(nbt), _p(nf),
+                                _p(pf), _p(out), C.c_int64(cap))
+    if nw < 0:
+        raise RuntimeError(f"orc_static_numer failed: {nw}")
+    return out[:nw]
+
+
+def poa_static(cfg: OracleConfig, rec: dict) -> float:
+    """Sum of the realized assignment's frozen costs over the sum of window OPTs."""
+    _, opt, _, _ = poa(cfg, rec)
+    st = static_numer(cfg, rec)
+    to = float(np.sum(opt))
+    return float(np.sum(st)) / to if to > 0 else 0.0
 
 
 def assign(cost, capw: int, method: int = 1):

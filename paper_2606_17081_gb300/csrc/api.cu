@@ -39,7 +39,7 @@ struct rs_ctx {
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
-      p_nwin, p_prob;
+      p_nwin, p_prob, p_wstat, p_tstat;
   DevBuf h_tokens, h_offsets, h_release, h_outlen;
   int64_t* pinned = nullptr;   // small host staging for device -> host reads
   size_t pinned_n = 0;
@@ -266,7 +266,8 @@ void route_destroy(rs_ctx* ctx) {
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
                    &ctx->p_wnum, &ctx->p_wopt, &ctx->p_wcnt, &ctx->p_total, &ctx->p_nwin,
-                   &ctx->p_prob, &ctx->h_tokens, &ctx->h_offsets, &ctx->h_release, &ctx->h_outlen};
+                   &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->h_tokens, &ctx->h_offsets,
+                   &ctx->h_release, &ctx->h_outlen};
   for (DevBuf* b : all) release(*b);
   if (ctx->pinned) cudaFreeHost(ctx->pinned);
   for (auto& ev : ctx->ev)
@@ -478,6 +479,8 @@ static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, const std::vector<P
       (r = ensure(ctx, ctx->p_wfill, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wnum, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wopt, (size_t)win_slots * 8, "poa windows")) ||
+      (r = ensure(ctx, ctx->p_wstat, (size_t)win_slots * 8, "poa windows")) ||
+      (r = ensure(ctx, ctx->p_tstat, (size_t)np * 8, "poa totals")) ||
       (r = ensure(ctx, ctx->p_wcnt, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_total, (size_t)np * 8, "poa totals")) ||
       (r = ensure(ctx, ctx->p_nwin, (size_t)np * 8, "poa totals")) ||
@@ -495,9 +498,11 @@ static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, const std::vector<P
   b.wstart = P<int64_t>(ctx->p_wstart);
   b.wfill = P<int64_t>(ctx->p_wfill);
   b.wnum = P<double>(ctx->p_wnum);
+  b.wstat = P<double>(ctx->p_wstat);
   b.wopt = P<double>(ctx->p_wopt);
   b.wcnt = P<int64_t>(ctx->p_wcnt);
   b.total = P<double>(ctx->p_total);
+  b.total_static = P<double>(ctx->p_tstat);
   b.nwin = P<int64_t>(ctx->p_nwin);
   b.res = res_dev;
   CK(launch_poa(P<PoaProblem>(ctx->p_prob), np, b, ctx->mc, ctx->st), "poa launch");
@@ -533,7 +538,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     const rs_replica_params& p = params[r];
     if (p.trace < 0 || p.trace >= n_traces) return fail(ctx, RS_ERR_INVALID, "replica %d: bad trace", r);
     if (p.C < 1 || p.C > 65535) return fail(ctx, RS_ERR_INVALID, "replica %d: C out of range", r);
-    if (p.policy != RS_POLICY_DYNAMO && p.policy != RS_POLICY_LOADBAL)
+    if (p.policy < RS_POLICY_DYNAMO || p.policy > RS_POLICY_P2C)
       return fail(ctx, RS_ERR_INVALID, "replica %d: bad policy", r);
     if (!(p.omega >= 0.0f) || !(p.tau >= 0.0f) || !std::isfinite(p.omega) || !std::isfinite(p.tau))
       return fail(ctx, RS_ERR_INVALID, "replica %d: omega/tau must be finite and >= 0", r);

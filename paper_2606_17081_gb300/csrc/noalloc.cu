@@ -27,7 +27,8 @@ size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // Carve-up of the static array for n rows of W workers (byte offsets).
 struct NoallocLayout {
-  size_t prob, total, nwin, cost, order, asg, wkey, wstart, wfill, wnum, wopt, wcnt, end;
+  size_t prob, total, nwin, cost, order, asg, wkey, wstart, wfill, wnum, wopt, wcnt, wstat,
+      tstat, end;
 };
 
 NoallocLayout layout(int64_t n, int W) {
@@ -47,6 +48,8 @@ NoallocLayout layout(int64_t n, int W) {
   L.wnum = o; o = up256(o + win * 8);
   L.wopt = o; o = up256(o + win * 8);
   L.wcnt = o; o = up256(o + win * 8);
+  L.wstat = o; o = up256(o + win * 8);
+  L.tstat = o; o = up256(o + 8);
   L.end = o;
   return L;
 }
@@ -138,6 +141,8 @@ extern "C" rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records
   b.wnum = reinterpret_cast<double*>(s + L.wnum);
   b.wopt = reinterpret_cast<double*>(s + L.wopt);
   b.wcnt = reinterpret_cast<int64_t*>(s + L.wcnt);
+  b.wstat = reinterpret_cast<double*>(s + L.wstat);
+  b.total_static = reinterpret_cast<double*>(s + L.tstat);
   b.total = reinterpret_cast<double*>(s + L.total);
   b.nwin = reinterpret_cast<int64_t*>(s + L.nwin);
   b.res = nullptr;

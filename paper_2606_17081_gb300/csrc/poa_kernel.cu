@@ -19,7 +19,8 @@
 // minima is rescanned.
 //
 // k_poa_total (one warp per replica): the whole-run PoA, sum of observed
-// latency over sum of OPT across the replica's windows.
+// latency over sum of OPT across the replica's windows; and the static
+// counterfactual of §9, the realized assignment's frozen cost over OPT.
 #include "rs_device.cuh"
 
 namespace rs {
@@ -222,6 +223,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       if (lane == 0) {
         b.wnum[pr.win_base + w] = 0.0;
         b.wopt[pr.win_base + w] = 0.0;
+        b.wstat[pr.win_base + w] = 0.0;
         b.wcnt[pr.win_base + w] = 0;
       }
       continue;
@@ -231,10 +233,11 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
     if (lane < W) S.counts[lane] = 0;
     if (lane == 0) S.err = 0;
     __syncwarp();
-    double num = 0.0;
+    double num = 0.0, nst = 0.0;
     for (int64_t r = lane; r < m; r += 32) {
       const int q = b.order[base + r];
       const double* cr = b.cost + (pr.scratch_base + q) * W;
+      nst += cr[b.rec.worker[pr.rec_base + q]];   // the realized assignment's frozen cost
       int best = 0;
       double bc = cr[0];
       for (int j = 1; j < W; j++)
@@ -244,6 +247,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       num += b.rec.ttft[pr.rec_base + q];
     }
     num = warp_sum(num);
+    nst = warp_sum(nst);
     __syncwarp();
     int over = 0;
     for (int j = 0; j < W; j++) over |= S.counts[j] > capw;
@@ -349,6 +353,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
     opt = warp_sum(opt);
     if (lane == 0) {
       b.wnum[pr.win_base + w] = num;
+      b.wstat[pr.win_base + w] = nst;
       b.wopt[pr.win_base + w] = S.err ? __longlong_as_double(0x7FF8000000000000ll) : opt;
       b.wcnt[pr.win_base + w] = m;
     }
@@ -365,18 +370,22 @@ __global__ void __launch_bounds__(NT_POA) k_poa_total(int nprob, PoaBuffers b,
   if (p >= nprob || lane != 0) return;
   const PoaProblem pr = probs[p];
   const int64_t nw = b.nwin[p];
-  double tot = __longlong_as_double(0x7FF8000000000000ll);
+  double tot = __longlong_as_double(0x7FF8000000000000ll), tst = tot;
   if (nw >= 0) {
-    double tn = 0.0, to = 0.0;
+    double tn = 0.0, to = 0.0, ts = 0.0;
     for (int64_t w = 0; w < nw; w++) {
       tn += b.wnum[pr.win_base + w];
       to += b.wopt[pr.win_base + w];
+      ts += b.wstat[pr.win_base + w];
     }
     tot = to > 0.0 ? tn / to : 0.0;
+    tst = to > 0.0 ? ts / to : 0.0;
   }
   b.total[p] = tot;
+  if (b.total_static) b.total_static[p] = tst;
   if (b.res) {
     b.res[p].poa_total = tot;
+    b.res[p].poa_static = tst;
     b.res[p].n_windows = nw;
   }
 }

@@ -86,6 +86,24 @@ __device__ __forceinline__ uint32_t draw_u24(uint64_t seed, uint64_t ordinal, ui
   return philox4x32_10(c, k).x >> 8;
 }
 
+// The worker a static policy sends request `ordinal` to (round robin, uniform
+// random, power of two choices; §9's routing baselines).  c: Eq. (1) costs
+// (P2C only).  Random draws take words x0 and x1 of the request's Philox
+// block, counter (ordinal, stream, tag) as draw_u24.
+__device__ __forceinline__ int static_policy_worker(int policy, const float* c, int W,
+                                                    uint64_t seed, uint64_t ordinal,
+                                                    uint32_t stream, uint32_t tag) {
+  if (policy == RS_POLICY_ROUNDROBIN) return (int)(ordinal % (uint64_t)W);
+  const uint4 x = philox4x32_10(make_uint4((uint32_t)ordinal, (uint32_t)(ordinal >> 32), stream, tag),
+                                make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+  const int j1 = (int)(((uint64_t)(x.x >> 8) * (uint64_t)W) >> 24);
+  if (policy == RS_POLICY_RANDOM || W < 2) return j1;
+  int j2 = (int)(((uint64_t)(x.y >> 8) * (uint64_t)(W - 1)) >> 24);   // uniform over the others
+  if (j2 >= j1) j2++;
+  const int lo = j1 < j2 ? j1 : j2, hi = j1 < j2 ? j2 : j1;
+  return c[hi] < c[lo] ? hi : lo;   // lower cost, ties to the lower index
+}
+
 // ---------------------------------------------------------------- exp of Eq. (2)
 
 // Cody-Waite reduction by ln2 (split in an 8-trailing-zero high part and a

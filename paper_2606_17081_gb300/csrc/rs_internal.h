@@ -118,8 +118,10 @@ struct PoaBuffers {
   int64_t* wfill;           // [win slots]
   double* wnum;             // [win slots]
   double* wopt;             // [win slots]
+  double* wstat;            // [win slots] frozen cost of the realized assignment
   int64_t* wcnt;            // [win slots]
   double* total;            // [problems]: PoA total
+  double* total_static;     // [problems]: realized assignment's frozen cost / OPT
   int64_t* nwin;            // [problems]: windows spanned (or -1 on overflow)
   rs_replica_result* res;   // optional [problems] (poa_total, n_windows filled)
 };

@@ -848,9 +848,12 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
       }
       __syncwarp();
       if (lane == 0) {
-        const uint32_t u24 = tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
+        const bool eq2 = d.policy == RS_POLICY_DYNAMO || d.policy == RS_POLICY_LOADBAL;
+        const uint32_t u24 = eq2 && tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
         float* ds = b.dstat + row * 6;
-        const int js = select_worker(c.wcost, W, tau, u24, ds + 2);
+        const int js = eq2 ? select_worker(c.wcost, W, tau, u24, ds + 2)
+                           : static_policy_worker(d.policy, c.wcost, W, d.seed, (uint64_t)i, 0u,
+                                                  TAG_SIM);
         S.jstar = js;
         S.hit_blocks += c.wm[js];
         // the chosen worker's absent blocks, latched before the control warp
@@ -861,8 +864,8 @@ __global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ d
         const CacheMeta* mt = &c.wmeta[js];
         const uint64_t span = (uint64_t)mt->T - mt->head + (uint64_t)nb;
         S.rebuild = span > L.g.R || mt->tombs > L.g.slots / 8 || (uint64_t)mt->T + nb > STAMP_LIMIT;
-        if (tau > 0.0f) S.sampled++;
-        else ds[3] = -1.0f;   // no draw
+        if (eq2 && tau > 0.0f) S.sampled++;
+        else ds[3] = -1.0f;   // no Eq. (2) draw
       }
     } else if (warp == 1 && lane == 0) {
       // statistics of the decision, beside the choice: work done by the probe

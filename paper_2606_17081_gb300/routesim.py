@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libroutesim.so")
 RS_OK, RS_ERR_INVALID, RS_ERR_OOM, RS_ERR_CAPACITY = 0, -1, -2, -3
 RS_ERR_CUDA, RS_ERR_TIMEOUT, RS_ERR_STATE, RS_ERR_COLLISION = -4, -5, -6, -7
 RS_POLICY_DYNAMO, RS_POLICY_LOADBAL = 0, 1
+RS_POLICY_ROUNDROBIN, RS_POLICY_RANDOM, RS_POLICY_P2C = 2, 3, 4
 RS_MEM_DEVICE, RS_MEM_HOST = 0, 1
 RS_SIM_NO_POA = 1
 
@@ -57,7 +58,7 @@ class rs_replica_result(C.Structure):
                 ("reserved0", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
                 ("final_ewma", C.c_double), ("probes", C.c_int64),
                 ("probe_blocks", C.c_int64), ("hashed_blocks", C.c_int64),
-                ("slow_path", C.c_int64), ("rebuilds", C.c_int64)]
+                ("slow_path", C.c_int64), ("rebuilds", C.c_int64), ("poa_static", C.c_double)]
 
     def as_dict(self) -> dict:
         return {f: (list(getattr(self, f)) if f == "ticks_in_regime" else getattr(self, f))

@@ -27,6 +27,10 @@ BLOCK = 16
 
 POLICY_DYNAMO = 0    # router cost of Eq. (1): omega * prefill blocks + active blocks
 POLICY_LOADBAL = 1   # coordinated: the same cost with omega = 0, tau = 0
+# static counterfactual policies (the routing-baselines discussion, §9)
+POLICY_ROUNDROBIN = 2   # request i -> worker i mod W
+POLICY_RANDOM = 3       # uniform worker from a Philox draw
+POLICY_P2C = 4          # two distinct uniform workers, the lower Eq. (1) cost
 
 
 @dataclass(frozen=True)

@@ -282,3 +282,33 @@ def test_route_release_rejects_bad_worker():
         rs.route_release(ctx.h, 0, wd, bd, 3)
     assert e.value.status == rs.RS_ERR_INVALID
     assert np.array_equal(rs.route_active(ctx.h, 0, 2), [0, 0])
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("W", [3, 5])
+def test_static_policies_and_static_poa(W):
+    # round robin, uniform random and power of two choices (the routing
+    # baselines of §9), below and above saturation (C = 256 > 63 W for W = 3)
+    spec = wk.TraceSpec(n_req=2500, n_groups=16, prefix_min=64, prefix_max=512,
+                        len_median=512, len_max=4096, out_median=128, out_max=1024)
+    tr = wk.make_trace(spec, 11)
+    reps = []
+    for k, (pol, om) in enumerate([(wk.POLICY_ROUNDROBIN, 1.0), (wk.POLICY_RANDOM, 1.0),
+                                   (wk.POLICY_P2C, 0.0), (wk.POLICY_P2C, 1.0)]):
+        for C in (8, 64, 256):
+            reps.append(wk.Replica(0, C, pol, 0, om, 0.0, 100 + k, tr.n_req))
+    ctx = rs.Context(W=W, K=8192)
+    st, g = gpu_run(ctx, [tr], reps)
+    assert st == 0
+    cfg = oracle_cfg(ctx)
+    for k, r in enumerate(reps):
+        o = oracle_run(cfg, tr, r)
+        assert_replica_equal(g[k], o, W)
+        tot = O.poa(cfg, o)[3]
+        sp = O.poa_static(cfg, o)
+        res = g[k]["result"]
+        assert abs(res["poa_total"] - tot) <= 1e-9 * tot
+        assert abs(res["poa_static"] - sp) <= 1e-9 * sp
+    if W == 3:   # queueing at C = 256: the observed estimate exceeds the static one
+        sat = [g[k]["result"] for k, r in enumerate(reps) if r.C == 256]
+        assert all(x["poa_total"] > x["poa_static"] for x in sat)
