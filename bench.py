@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 32236985088 + 8341278976,
-               "sources_sha256": "d1226cb2c5fbd82b4d58dffc5e3d51502e7787108fcc490bfd4d4a2afea6e45d",
+SIM_TRAFFIC = {"bytes": 32089563648 + 6073165056,
+               "sources_sha256": "95ce82398c6e5fe905df72d7de604e089549b0d502e6afa97f9423d67c14a997",
                "summary": "profiles/k_sim_p2d.md"}
 
 
