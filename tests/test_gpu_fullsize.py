@@ -20,7 +20,8 @@ if not torch.cuda.is_available():
 def _check(p, sample, poa=True):
     traces = p.traces()
     ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
-    st, g = gpu_run(ctx, traces, p.replicas, with_cost=False)
+    st, g = gpu_run(ctx, traces, p.replicas, with_cost=False,
+                    flags=0 if poa else rs.RS_SIM_NO_POA)
     assert st == 0
     cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
     for k in sample:
@@ -48,3 +49,18 @@ def test_p5d_grid_reduced():
 def test_grid_reduced():
     p = wk.plan("grid", n_req=1500, replicas=list(range(0, 8192, 173)))
     _check(p, range(len(p.replicas)))
+
+
+def test_large_shape_w64_reduced():
+    # the W = 64 workload's prompt shape (median 2048 tokens, up to 32768, i.e.
+    # 2048 blocks; 1024 prefix groups): the chunked probe, 64 lanes of costs,
+    # PoA off (the solver takes W <= 16).  Smaller caches so that the oracle
+    # finishes in seconds, and C = 512: with 2048-block prompts a replica's
+    # shared memory holds at most about 512 requests in flight
+    p = wk.plan("large", n_req=2000, replicas=[0, 8])
+    p.K = 1 << 14
+    for r in p.replicas:
+        r.C = 512
+    g = _check(p, range(len(p.replicas)), poa=False)
+    assert all(x["result"]["status"] == 0 for x in g)
+    assert max(x["result"]["hashed_blocks"] for x in g) > 0
