@@ -14,8 +14,10 @@
 // every lane folds its own row in order, and per request the warp writes the
 // 32 hashes back with one coalesced store.  Lanes whose requests are done
 // claim the next ones from a work counter (one atomic per warp for all of
-// them), so the warps stay busy until the counter runs out.  8 bytes per
-// block in and out.
+// them), so the warps stay busy until the counter runs out.  The content pass
+// lists the long prompts (HASH_LONG_NB blocks and more), and the counter hands
+// those out first: their chains, serial and up to hundreds of blocks long,
+// overlap the bulk instead of trailing it.  8 bytes per block in and out.
 #include <climits>
 
 #include "rs_device.cuh"
@@ -27,6 +29,7 @@ constexpr int CHAIN_WARPS = 4;               // chain pass: warps per CTA
 constexpr int CHAIN_NT = 32 * CHAIN_WARPS;
 constexpr int CHAIN_ROW = 33;                // 32 staged blocks per request + 1 pad word
 constexpr int CHAIN_ILP = 8;                 // requests whose chunks are loaded together
+constexpr int64_t HASH_LONG_NB = 96;         // prompts of this many blocks are chained first
 
 template <int S>
 __device__ __forceinline__ void take16(const uint32_t (&a)[20], uint32_t (&w)[16]) {
@@ -72,7 +75,9 @@ __device__ __forceinline__ int find_job(const HashJob* jobs, int njobs, int64_t 
 }
 
 __global__ void __launch_bounds__(CONTENT_NT) k_block_content(const HashJob* __restrict__ jobs,
-                                                              int njobs, int64_t total_req) {
+                                                              int njobs, int64_t total_req,
+                                                              HashSched* __restrict__ sched,
+                                                              int64_t* __restrict__ long_list) {
   __shared__ HashJob s_jobs[HASH_MAX_JOBS];
   for (int j = threadIdx.x; j < njobs; j += CONTENT_NT) s_jobs[j] = jobs[j];
   __syncthreads();
@@ -87,6 +92,8 @@ __global__ void __launch_bounds__(CONTENT_NT) k_block_content(const HashJob* __r
     const int shift = (int)(o0 & 3);
     const int4* q = reinterpret_cast<const int4*>(J.tokens) + (o0 >> 2);
     uint64_t* out = J.out + (o0 >> 4);
+    if (lane == 0 && nb >= HASH_LONG_NB)   // its chain goes first in the chain pass
+      long_list[atomicAdd(&sched->nlong, 1ull)] = r;
     for (int64_t k0 = 0; k0 < nb; k0 += 64) {
       // both blocks' loads go out before either is folded
       const int64_t ka = k0 + lane, kb = ka + 32;
@@ -104,7 +111,8 @@ __global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restr
                                                           int njobs, int64_t total_req,
                                                           uint64_t seed,
                                                           int64_t* __restrict__ nbmax,
-                                                          unsigned long long* __restrict__ work) {
+                                                          HashSched* __restrict__ sched,
+                                                          const int64_t* __restrict__ long_list) {
   __shared__ HashJob s_jobs[HASH_MAX_JOBS];
   __shared__ uint64_t s_stage[CHAIN_WARPS][32 * CHAIN_ROW];
   __shared__ int64_t s_max[CHAIN_WARPS];
@@ -115,7 +123,11 @@ __global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restr
   uint64_t* stage = s_stage[wid];
   uint64_t* row = stage + lane * CHAIN_ROW;
   int64_t local_max = 0;
-  bool exhausted = false;   // the work counter has passed the last request (warp-uniform)
+  // indices 0 .. nlong-1 of the work counter are the long prompts, then come
+  // all requests in order (long ones skipped: they are chained already)
+  const int64_t nlong = (int64_t)sched->nlong;
+  const int64_t nidx = nlong + total_req;
+  bool exhausted = false;   // the work counter has passed the last index (warp-uniform)
   // this lane's request: blocks [c0, nb) of the hashes at oaddr, chain value h
   bool has = false;
   unsigned long long oaddr = 0;
@@ -127,11 +139,13 @@ __global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restr
     while (need && !exhausted) {
       const int cnt = __popc(need);
       unsigned long long b = 0;
-      if (lane == 0) b = atomicAdd(work, (unsigned long long)cnt);
+      if (lane == 0) b = atomicAdd(&sched->work, (unsigned long long)cnt);
       b = __shfl_sync(FULL_MASK, b, 0);
-      if ((int64_t)b + cnt >= total_req) exhausted = true;
-      const int64_t r = (int64_t)b + __popc(need & lt_mask);
-      if (!has && r < total_req) {
+      if ((int64_t)b + cnt >= nidx) exhausted = true;
+      const int64_t v = (int64_t)b + __popc(need & lt_mask);
+      const bool listed = v < nlong;
+      const int64_t r = listed ? long_list[v] : v - nlong;
+      if (!has && v < nidx) {
         const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
         const int64_t i = r - J.req_base;
         const int64_t o0 = __ldg(J.offsets + i);
@@ -140,7 +154,9 @@ __global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restr
         c0 = 0;
         h = seed;
         local_max = nb > local_max ? nb : local_max;
-        has = nb > 0;   // a prompt without a full block has nothing to chain
+        // a prompt without a full block has nothing to chain; a long one
+        // reached in order was chained from the list
+        has = nb > 0 && (listed || nb < HASH_LONG_NB);
       }
       need = __ballot_sync(FULL_MASK, !has);
     }
@@ -213,9 +229,10 @@ __global__ void __launch_bounds__(CHAIN_NT) k_block_chain(const HashJob* __restr
 }
 
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
-                              int64_t* nbmax_out, unsigned long long* work, cudaStream_t st) {
+                              int64_t* nbmax_out, HashSched* sched, int64_t* long_list,
+                              cudaStream_t st) {
   if (total_req <= 0) return cudaSuccess;
-  if (njobs < 1 || njobs > HASH_MAX_JOBS || !work) return cudaErrorInvalidValue;
+  if (njobs < 1 || njobs > HASH_MAX_JOBS || !sched || !long_list) return cudaErrorInvalidValue;
   int dev = 0, sms = 0, per_sm = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -223,7 +240,8 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
   // content: one warp per request, grid-strided
   int64_t cb = (total_req + CONTENT_NT / 32 - 1) / (CONTENT_NT / 32);
   if (cb > (int64_t)sms * 16) cb = (int64_t)sms * 16;
-  k_block_content<<<(unsigned)cb, CONTENT_NT, 0, st>>>(jobs_dev, njobs, total_req);
+  k_block_content<<<(unsigned)cb, CONTENT_NT, 0, st>>>(jobs_dev, njobs, total_req, sched,
+                                                       long_list);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // chain: one wave of resident CTAs; the work counter hands out the requests
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_block_chain, CHAIN_NT, 0);
@@ -232,7 +250,7 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
   const int64_t need = (total_req + CHAIN_NT - 1) / CHAIN_NT;
   if (nblk > need) nblk = need;
   k_block_chain<<<(unsigned)nblk, CHAIN_NT, 0, st>>>(jobs_dev, njobs, total_req, seed, nbmax_out,
-                                                     work);
+                                                     sched, long_list);
   return cudaGetLastError();
 }
 
