@@ -783,13 +783,14 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
   }
   ntomb = __reduce_add_sync(FULL_MASK, (unsigned)ntomb);
   if ((threadIdx.x & 31) == 0 && ntomb) atomicAdd(&us->n_tomb, ntomb);
-  grp_bar<NT>();
   const uint32_t T = meta->T;
   int nins = 0, recl = 0, err = 0;
   // inserts at the positions the lookup saw free: this CTA alone writes the
   // table, so a shared-memory claim per slot settles blocks that saw the same
   // position and the key is stored plainly; the others insert after the
-  // barrier, along their probe path
+  // barrier, along their probe path.  No barrier from the evictions is
+  // needed: a position seen free is not a victim (victims hold keys), and the
+  // stamps and the probing inserts come after the barrier below.
   for (int k = threadIdx.x; k < nb; k += NT) {
     if (!sc.kind[k]) continue;
     const uint32_t fr = sc.fslot[k];
@@ -834,13 +835,13 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
   }
   if (err) us->err = RS_ERR_TIMEOUT;
   grp_bar<NT>();
+  // (the caller's next barrier orders this with any later reader of meta)
   if (threadIdx.x == 0) {
     meta->tombs = meta->tombs + (uint32_t)us->n_tomb - (uint32_t)us->reclaimed;
     meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
     if (E > 0) meta->head = sc.vt[sc.victim[E - 1]] + 1;
     meta->T = T + (uint32_t)nb;
   }
-  grp_bar<NT>();
 }
 
 }  // namespace rs
