@@ -695,7 +695,11 @@ __device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q,
   for (int k = lane; k < q.nb; k += 32) dst[k] = __ldg(src + k);
 }
 
-__global__ void __launch_bounds__(NT_SIM, 2) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
+// MINB = CTAs the launch keeps resident per SM: 2 (128 registers) when there
+// are more replicas than SMs, 1 (no register cap to speak of, no spills) when
+// every replica has an SM to itself.
+template <int MINB>
+__global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ SimScalars S;
@@ -1103,10 +1107,19 @@ cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaun
                        cudaStream_t st) {
   if (L.nsim <= 0) return cudaSuccess;
   const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap);
-  cudaError_t e = cudaFuncSetAttribute(k_sim, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  k_sim<<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
+  if (L.nsim <= sms) {   // one replica per SM: the kernel may use every register
+    e = cudaFuncSetAttribute(k_sim<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_sim<1><<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
+  } else {
+    e = cudaFuncSetAttribute(k_sim<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_sim<2><<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
+  }
   return cudaGetLastError();
 }
 
