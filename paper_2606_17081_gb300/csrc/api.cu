@@ -36,7 +36,7 @@ struct rs_ctx {
   DevBuf r_keys, r_stamp, r_log, r_tmp, r_meta, r_active, r_ord, r_status, r_hash, r_stats;
   // simulation scratch (grow-only)
   DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, hwork, hlong, dstat,
-      wco;
+      wco, slots;
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -262,7 +262,7 @@ void route_destroy(rs_ctx* ctx) {
   DevBuf* all[] = {&ctx->r_keys, &ctx->r_stamp, &ctx->r_log, &ctx->r_tmp, &ctx->r_meta,
                    &ctx->r_active, &ctx->r_ord, &ctx->r_status, &ctx->r_hash, &ctx->r_stats,
                    &ctx->keys, &ctx->stamp, &ctx->log, &ctx->tmp, &ctx->pend, &ctx->meta_out,
-                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->hwork, &ctx->hlong, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
+                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->hwork, &ctx->hlong, &ctx->slots, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
                    &ctx->rec_arrival, &ctx->rec_start, &ctx->rec_first, &ctx->rec_completion,
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
@@ -648,13 +648,20 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   CK(cudaStreamSynchronize(ctx->st), "sync");
   int64_t nbmax = std::max<int64_t>(1, ctx->pinned[0]);
   if (nbmax > (int64_t)g.K) nbmax = g.K;   // longer prompts stop their replica with RS_ERR_CAPACITY
-  const size_t smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap);
   int maxsmem = 0;
   cudaDeviceGetAttribute(&maxsmem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device);
-  if (smem + sizeof(int) * 2048 > (size_t)maxsmem)
+  const size_t smem_room = (size_t)maxsmem > sizeof(int) * 2048 ? maxsmem - sizeof(int) * 2048 : 0;
+  // per-request slot arrays in shared memory when they fit, else in global memory
+  bool slots_global = false;
+  size_t smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, false);
+  if (smem > smem_room) {
+    slots_global = true;
+    smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, true);
+  }
+  if (smem > smem_room)
     return fail(ctx, RS_ERR_CAPACITY,
-                "prompt of %lld blocks and C = %d need %zu bytes of shared memory per replica",
-                (long long)nbmax, cmax, smem);
+                "prompt of %lld blocks needs %zu bytes of shared memory per replica",
+                (long long)nbmax, smem);
   // ---- scratch
   const size_t nsim = n_replicas;
   const size_t nsl = nsim * W * g.slots;
@@ -668,6 +675,9 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       (r = ensure(ctx, ctx->desc, nsim * sizeof(SimDesc), "replica descriptors")) ||
       (r = ensure(ctx, ctx->dstat, (size_t)std::max<int64_t>(rows, 1) * 6 * sizeof(float),
                   "decision statistics")))
+    return r;
+  if (slots_global &&
+      (r = ensure(ctx, ctx->slots, nsim * sim_slot_bytes(cmax), "request slots")) != RS_OK)
     return r;
   // w_c * (m / nbt) table for prompts up to nbmax blocks (none beyond 2048)
   const bool use_tab = nbmax <= 2048;
@@ -719,10 +729,12 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   sb.dstat = P<float>(ctx->dstat);
   sb.wco_tab = use_tab ? P<double>(ctx->wco) : nullptr;
   sb.wco_dim = (int)nbmax + 2;
+  sb.slotmem = slots_global ? P<unsigned char>(ctx->slots) : nullptr;
   SimLaunch L;
   L.nsim = (int)nsim;
   L.nbmax = (int)nbmax;
   L.cmax = cmax;
+  L.slots_global = slots_global ? 1 : 0;
   L.g = g;
   L.mc = ctx->mc;
   L.mc.write_cost = want_cost ? 1 : 0;

@@ -67,17 +67,22 @@ struct SimBuffers {
   float* dstat;             // [rows][6]: two lowest costs, draw position (see k_decision_stats)
   const double* wco_tab;    // [(nbmax+1)(nbmax+2)] w_c * (m / nbt), or NULL
   int wco_dim;              // nbmax + 2 (row length of wco_tab)
+  unsigned char* slotmem;   // [nsim][sim_slot_bytes(cmax)] when SimLaunch::slots_global
 };
 
 struct SimLaunch {
   int nsim;
   int nbmax;                // max full blocks of any routed prompt
   int cmax;                 // max concurrency over replicas
+  int slots_global;         // 1: per-request slot arrays in SimBuffers::slotmem
   TableGeom g;
   ModelConsts mc;
 };
 
-size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap);
+// Dynamic shared memory of one replica CTA; with slots_global the per-request
+// slot arrays are in global memory instead (sim_slot_bytes per replica).
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global);
+size_t sim_slot_bytes(int cmax);
 
 // One trace for the block-hash kernels: requests req_base .. req_base+n_req-1
 // of the launch's global request numbering.

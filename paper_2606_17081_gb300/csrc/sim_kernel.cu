@@ -40,12 +40,18 @@ struct SimLayout {
   size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen, wabs;
   size_t kind, evk, touched;
   size_t total;
+  size_t slot_bytes;   // per-replica global bytes of the slot arrays (0: in shared memory)
   uint32_t dupmask;
 };
 
-__host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax, int nft) {
+// slots_global: the per-request slot arrays (times, links, the event heap;
+// 56 bytes per request in flight) live in global memory, for concurrencies
+// whose slots do not fit in shared memory; their offsets are then relative to
+// the replica's global slot area.
+__host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax, int nft,
+                                                     bool slots_global = false) {
   SimLayout L;
-  size_t o = 0;
+  size_t o = 0, og = 0;
   const size_t nb = (size_t)(nbmax > 0 ? nbmax : 1);
   const size_t nv = 2 * nb;
   const size_t C = (size_t)(cmax > 0 ? cmax : 1);
@@ -56,22 +62,30 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   o = align_up(o, al);         \
   L.field = o;                 \
   o += (bytes);
+#define TAKES(field, bytes, al)  /* a slot array */ \
+  if (slots_global) {                               \
+    og = align_up(og, al);                          \
+    L.field = og;                                   \
+    og += (bytes);                                  \
+  } else {                                          \
+    TAKE(field, bytes, al)                          \
+  }
   TAKE(ftab, 8 * (size_t)(nft > 0 ? nft : 1), 16)
   TAKE(wwco, 8 * (size_t)W, 8)
-  TAKE(f_oitl, 8 * C, 8)
-  TAKE(f_a, 8 * C, 8)
-  TAKE(f_o, 8 * C, 8)
-  TAKE(h_k, 8 * C, 8)
+  TAKES(f_oitl, 8 * C, 8)
+  TAKES(f_a, 8 * C, 8)
+  TAKES(f_o, 8 * C, 8)
+  TAKES(h_k, 8 * C, 8)
   TAKE(hbuf0, 8 * nb, 16)
   TAKE(hbuf1, 8 * nb, 16)
   TAKE(dupset, 8 * dup, 16)
   TAKE(wA, 8 * (size_t)W, 8)
-  TAKE(f_req, 4 * C, 4)
-  TAKE(f_worker, 4 * C, 4)
-  TAKE(f_blk, 4 * C, 4)
-  TAKE(f_next, 4 * C, 4)
-  TAKE(h_f, 4 * C, 4)
-  TAKE(freestk, 4 * C, 4)
+  TAKES(f_req, 4 * C, 4)
+  TAKES(f_worker, 4 * C, 4)
+  TAKES(f_blk, 4 * C, 4)
+  TAKES(f_next, 4 * C, 4)
+  TAKES(h_f, 4 * C, 4)
+  TAKES(freestk, 4 * C, 4)
   TAKE(owner, 4 * nv, 4)
   TAKE(victim, 4 * nv, 4)
   TAKE(slot, 4 * nb, 4)
@@ -93,15 +107,21 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(kind, nb, 1)
   TAKE(evk, nb, 1)
   TAKE(touched, nv, 1)
+#undef TAKES
 #undef TAKE
   L.total = align_up(o, 16);
+  L.slot_bytes = slots_global ? align_up(og, 256) : 0;
   return L;
 }
 
 __host__ __device__ inline int ftab_size(int cap) { return cap < FTAB_MAX ? cap : FTAB_MAX; }
 
-size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap) {
-  return make_sim_layout(W, nbmax, cmax, ftab_size(cap)).total;
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global) {
+  return make_sim_layout(W, nbmax, cmax, ftab_size(cap), slots_global).total;
+}
+
+size_t sim_slot_bytes(int cmax) {
+  return make_sim_layout(1, 1, cmax, 1, true).slot_bytes;
 }
 
 // One request as the loop sees it (two live at once: i and i+1).
@@ -698,7 +718,9 @@ __device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q,
 // MINB = CTAs the launch keeps resident per SM: 2 (128 registers) when there
 // are more replicas than SMs, 1 (no register cap to speak of, no spills) when
 // every replica has an SM to itself.
-template <int MINB>
+// SG: the per-request slot arrays are in global memory (a compile-time
+// choice, so that in the common case the compiler knows they are shared).
+template <int MINB, bool SG>
 __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
   extern __shared__ __align__(16) unsigned char smem[];
@@ -708,7 +730,13 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   const int W = L.mc.W;
   const ModelConsts& mc = L.mc;
   const int nft = ftab_size(mc.cap);
-  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax, nft);
+  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax, nft, SG);
+  // the slot arrays: shared memory, or this replica's global slot area
+  unsigned char* slotbase;
+  if constexpr (SG)
+    slotbase = b.slotmem + (size_t)sid * make_sim_layout(1, 1, L.cmax, 1, true).slot_bytes;
+  else
+    slotbase = smem;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   SimCtx c;
   c.S = &S;
@@ -717,19 +745,19 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.L = &L;
   c.sid = sid;
   c.ftab = reinterpret_cast<double*>(smem + lay.ftab);
-  c.f_oitl = reinterpret_cast<double*>(smem + lay.f_oitl);
+  c.f_oitl = reinterpret_cast<double*>(slotbase + lay.f_oitl);
   c.wwco = reinterpret_cast<double*>(smem + lay.wwco);
-  c.f_a = reinterpret_cast<double*>(smem + lay.f_a);
-  c.f_o = reinterpret_cast<double*>(smem + lay.f_o);
-  c.h_k = reinterpret_cast<uint64_t*>(smem + lay.h_k);
+  c.f_a = reinterpret_cast<double*>(slotbase + lay.f_a);
+  c.f_o = reinterpret_cast<double*>(slotbase + lay.f_o);
+  c.h_k = reinterpret_cast<uint64_t*>(slotbase + lay.h_k);
   c.hbuf0 = reinterpret_cast<uint64_t*>(smem + lay.hbuf0);
   c.hbuf1 = reinterpret_cast<uint64_t*>(smem + lay.hbuf1);
-  c.f_req = reinterpret_cast<int32_t*>(smem + lay.f_req);
-  c.f_worker = reinterpret_cast<int32_t*>(smem + lay.f_worker);
-  c.f_blk = reinterpret_cast<int32_t*>(smem + lay.f_blk);
-  c.f_next = reinterpret_cast<int32_t*>(smem + lay.f_next);
-  c.h_f = reinterpret_cast<int32_t*>(smem + lay.h_f);
-  c.freestk = reinterpret_cast<int32_t*>(smem + lay.freestk);
+  c.f_req = reinterpret_cast<int32_t*>(slotbase + lay.f_req);
+  c.f_worker = reinterpret_cast<int32_t*>(slotbase + lay.f_worker);
+  c.f_blk = reinterpret_cast<int32_t*>(slotbase + lay.f_blk);
+  c.f_next = reinterpret_cast<int32_t*>(slotbase + lay.f_next);
+  c.h_f = reinterpret_cast<int32_t*>(slotbase + lay.h_f);
+  c.freestk = reinterpret_cast<int32_t*>(slotbase + lay.freestk);
   c.wmeta = reinterpret_cast<CacheMeta*>(smem + lay.wmeta);
   c.winserv = reinterpret_cast<int32_t*>(smem + lay.winserv);
   c.wqh = reinterpret_cast<int32_t*>(smem + lay.wqh);
@@ -1106,20 +1134,19 @@ cudaError_t launch_decision_stats(const SimDesc* d_desc, const SimBuffers& b, co
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st) {
   if (L.nsim <= 0) return cudaSuccess;
-  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap);
+  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap, L.slots_global != 0);
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  if (L.nsim <= sms) {   // one replica per SM: the kernel may use every register
-    e = cudaFuncSetAttribute(k_sim<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    k_sim<1><<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
-  } else {
-    e = cudaFuncSetAttribute(k_sim<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    k_sim<2><<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
-  }
+  // one replica per SM: the kernel may use every register
+  const bool one = L.nsim <= sms;
+  void (*kern)(const SimDesc*, SimBuffers, SimLaunch) =
+      one ? (L.slots_global ? k_sim<1, true> : k_sim<1, false>)
+          : (L.slots_global ? k_sim<2, true> : k_sim<2, false>);
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  kern<<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);
   return cudaGetLastError();
 }
 

@@ -53,14 +53,14 @@ def test_grid_reduced():
 
 def test_large_shape_w64_reduced():
     # the W = 64 workload's prompt shape (median 2048 tokens, up to 32768, i.e.
-    # 2048 blocks; 1024 prefix groups): the chunked probe, 64 lanes of costs,
-    # PoA off (the solver takes W <= 16).  Smaller caches so that the oracle
-    # finishes in seconds, and C = 512: with 2048-block prompts a replica's
-    # shared memory holds at most about 512 requests in flight
-    p = wk.plan("large", n_req=2000, replicas=[0, 8])
+    # 2048 blocks; 1024 prefix groups) and its concurrency C = 4096: the
+    # chunked probe, 64 lanes of costs, the per-request slots and event heap in
+    # global memory (4096 in flight do not fit beside 2048-block prompts in
+    # shared memory), PoA off (the solver takes W <= 16).  Smaller caches and
+    # fewer requests so that the oracle finishes in seconds.
+    p = wk.plan("large", n_req=6000, replicas=[0, 8])
     p.K = 1 << 14
-    for r in p.replicas:
-        r.C = 512
+    assert all(r.C == 4096 for r in p.replicas)
     g = _check(p, range(len(p.replicas)), poa=False)
     assert all(x["result"]["status"] == 0 for x in g)
     assert max(x["result"]["hashed_blocks"] for x in g) > 0
