@@ -176,6 +176,11 @@ typedef struct {
   float omega, tau;     /* Below-regime router parameters (>= 0) */
   uint64_t seed;        /* Philox key of this replica's sampling stream */
   int64_t n_req;        /* 0 .. trace n_req */
+  /* Load-spike schedule (Experiment 3, §7.7): the client holds C requests in
+   * flight before c_t1, c_mid on [c_t1, c_t2) and c_end from c_t2 on (s of
+   * simulated time).  c_mid = 0: C throughout (the times are ignored). */
+  double c_t1, c_t2;
+  int32_t c_mid, c_end;
 } rs_replica_params;
 
 typedef struct {
@@ -201,6 +206,7 @@ typedef struct {
   int64_t hashed_blocks;    /* sum of nb_i (full blocks) over routed requests */
   int64_t slow_path;        /* updates that needed the exact sequential path */
   int64_t rebuilds;         /* table/log compactions */
+  double first_switch_t;    /* time of the first controller regime switch, -1 if none */
   double poa_static;        /* the realized assignment under the frozen cost model of
                                §6.4: sum over windows of sum_i c_{i, worker(i)} over
                                the sum of OPTs (the static counterfactual of §9) */

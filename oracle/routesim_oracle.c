@@ -529,7 +529,9 @@ static void controller_tick(sim_t* s) {
   }
   s->npending = keep;
   double L = nw > 0 ? p99_nearest_rank(s->window, nw) : 0.0;
+  int64_t sw0 = s->ctl.switches;
   ctl_sample(&s->ctl, cfg, nw > 0, L);
+  if (sw0 == 0 && s->ctl.switches > 0) s->sum->first_switch_t = tt;
   if (s->ctl.regime > s->sum->max_regime) s->sum->max_regime = s->ctl.regime;
   if (s->tick_ewma && s->sum->ticks < s->max_ticks) {
     s->tick_ewma[s->sum->ticks] = s->ctl.have_ewma ? s->ctl.ewma : -1.0;
@@ -545,17 +547,36 @@ static double next_tick_time(const sim_t* s) {
   return s->rep->controller ? (double)s->next_tick * s->cfg->dt : INFINITY;
 }
 
+/* Concurrency of the load-spike schedule at time t (Experiment 3). */
+static int64_t conc_at(const orc_replica* r, double t) {
+  if (r->c_mid <= 0) return r->C;
+  if (t < r->c_t1) return r->C;
+  if (t < r->c_t2) return r->c_mid;
+  return r->c_end;
+}
+
+/* The next time after t at which the schedule's concurrency changes. */
+static double next_step_time(const orc_replica* r, double t) {
+  if (r->c_mid <= 0) return INFINITY;
+  if (t < r->c_t1) return r->c_t1;
+  if (t < r->c_t2) return r->c_t2;
+  return INFINITY;
+}
+
 int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t* offsets,
                      const double* release, const int32_t* out_len, const orc_replica* rep,
                      orc_records* rec, orc_summary* sum, uint64_t* cache_keys,
                      int64_t* cache_sizes, double* tick_ewma, int32_t* tick_regime,
                      int64_t max_ticks) {
   memset(sum, 0, sizeof *sum);
+  sum->first_switch_t = -1.0;
   const int32_t W = cfg->W;
   const int64_t n = rep->n_req;
   if (W < 1 || cfg->block < 2 || (cfg->block & 1) || cfg->K < 1 || cfg->cap < 2 || rep->C < 1 ||
       n < 0 || !(rep->tau >= 0.0f) || !(rep->omega >= 0.0f) ||
-      rep->policy < ORC_POLICY_DYNAMO || rep->policy > ORC_POLICY_P2C) {
+      rep->policy < ORC_POLICY_DYNAMO || rep->policy > ORC_POLICY_P2C ||
+      (rep->c_mid > 0 && (rep->c_end < 1 || !(rep->c_t1 >= 0.0) || !(rep->c_t2 >= rep->c_t1))) ||
+      rep->c_mid < 0) {
     sum->status = ORC_ERR_INVALID;
     return ORC_ERR_INVALID;
   }
@@ -612,20 +633,24 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   double prev_arrival = 0.0;
 
   for (int64_t i = 0; i < n; i++) {
-    /* closed-loop client (§7.4): request i waits for a free semaphore slot */
+    /* closed-loop client (§7.4): request i waits until fewer than C(t)
+     * requests are in flight; completions, controller samples and steps of
+     * the load-spike schedule are taken in time order (ties in that order) */
     double T = prev_arrival;
-    if (s.in_flight >= rep->C) {
-      for (;;) {
-        double tc = s.heap[0].t;
-        if (next_tick_time(&s) < tc) {
-          controller_tick(&s);
-          if (s.err) { status = s.err; goto done; }
-          continue;
-        }
+    while (s.in_flight >= conc_at(rep, T)) {
+      double tc = s.nheap > 0 ? s.heap[0].t : INFINITY;
+      double tt = next_tick_time(&s);
+      double ts = next_step_time(rep, T);
+      if (tc == INFINITY && ts == INFINITY) { status = ORC_ERR_TIMEOUT; goto done; }
+      if (tc <= tt && tc <= ts) {
         cev e = heap_pop(s.heap, &s.nheap);
         complete(&s, e.q, e.t);
         if (e.t > T) T = e.t;
-        break;
+      } else if (tt <= ts) {
+        controller_tick(&s);
+        if (s.err) { status = s.err; goto done; }
+      } else {
+        T = ts;   /* the schedule steps to its next concurrency */
       }
     }
     double a = release[i] > T ? release[i] : T;

@@ -39,6 +39,7 @@ enum {
   ORC_ERR_INVALID = -1,
   ORC_ERR_OOM = -2,
   ORC_ERR_CAPACITY = -3,   /* a prompt has more full blocks than a cache holds */
+  ORC_ERR_TIMEOUT = -5,    /* inconsistent event state (cannot happen) */
   ORC_ERR_COLLISION = -7   /* two blocks of one prompt share a chained hash */
 };
 
@@ -72,6 +73,10 @@ typedef struct {
   float omega, tau;       /* static router parameters (Below regime) */
   uint64_t seed;          /* Philox key of the sampling stream */
   int64_t n_req;          /* requests routed (prefix of the trace) */
+  /* load-spike schedule (Experiment 3): C before c_t1, c_mid on [c_t1, c_t2),
+   * c_end from c_t2 on; c_mid = 0 keeps C */
+  double c_t1, c_t2;
+  int32_t c_mid, c_end;
 } orc_replica;
 
 typedef struct {
@@ -84,6 +89,7 @@ typedef struct {
   int32_t final_regime, max_regime;
   int64_t ticks_in_regime[3];
   double final_ewma;
+  double first_switch_t;   /* first regime switch, -1 if none */
 } orc_summary;
 
 /* Per-request outputs; every pointer may be NULL.  Arrays of n (or n*W). */

@@ -47,7 +47,8 @@ class _Config(C.Structure):
 class _Replica(C.Structure):
     _fields_ = [("C", C.c_int32), ("policy", C.c_int32), ("controller", C.c_int32),
                 ("omega", C.c_float), ("tau", C.c_float), ("seed", C.c_uint64),
-                ("n_req", C.c_int64)]
+                ("n_req", C.c_int64), ("c_t1", C.c_double), ("c_t2", C.c_double),
+                ("c_mid", C.c_int32), ("c_end", C.c_int32)]
 
 
 class _Summary(C.Structure):
@@ -58,7 +59,7 @@ class _Summary(C.Structure):
                 ("evicted_blocks", C.c_int64), ("ticks", C.c_int64),
                 ("regime_switches", C.c_int64), ("final_regime", C.c_int32),
                 ("max_regime", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
-                ("final_ewma", C.c_double)]
+                ("final_ewma", C.c_double), ("first_switch_t", C.c_double)]
 
 
 class _Records(C.Structure):
@@ -180,8 +181,11 @@ def hash_blocks(tokens, offsets, block: int = 16, seed: int = 0) -> np.ndarray:
 
 def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
              controller: int = 0, omega: float = 1.0, tau: float = 0.0, seed: int = 0,
-             n_req=None, want_cache: bool = False, max_ticks: int = 0) -> dict:
-    """Run one replica.  `trace` has tokens/offsets/release/out_len arrays."""
+             n_req=None, want_cache: bool = False, max_ticks: int = 0,
+             schedule=None) -> dict:
+    """Run one replica.  `trace` has tokens/offsets/release/out_len arrays.
+    schedule: None or (c_t1, c_t2, c_mid, c_end), the load-spike concurrency
+    of Experiment 3 (C before c_t1, c_mid until c_t2, c_end after)."""
     n = trace.n_req if n_req is None else int(n_req)
     W = cfg.W
     t = _c(trace.tokens, np.int32)
@@ -198,7 +202,9 @@ def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
     rec = _Records(*[_p(r[k]).value for k in ("worker", "arrival", "start", "first_token",
                                                 "completion", "ttft", "nbt", "n_frozen",
                                                 "prefix", "cost")])
-    rep = _Replica(C_, policy, controller, omega, tau, seed, n)
+    st = schedule if schedule is not None else (0.0, 0.0, 0, 0)
+    rep = _Replica(C_, policy, controller, omega, tau, seed, n, float(st[0]), float(st[1]),
+                   int(st[2]), int(st[3]))
     s = _Summary()
     keys = np.zeros(W * cfg.K, np.uint64) if want_cache else None
     sizes = np.zeros(W, np.int64) if want_cache else None

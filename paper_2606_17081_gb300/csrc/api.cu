@@ -546,6 +546,10 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     const rs_replica_params& p = params[r];
     if (p.trace < 0 || p.trace >= n_traces) return fail(ctx, RS_ERR_INVALID, "replica %d: bad trace", r);
     if (p.C < 1 || p.C > 65535) return fail(ctx, RS_ERR_INVALID, "replica %d: C out of range", r);
+    if (p.c_mid < 0 || p.c_mid > 65535 ||
+        (p.c_mid > 0 && (p.c_end < 1 || p.c_end > 65535 || !(p.c_t1 >= 0.0) ||
+                         !(p.c_t2 >= p.c_t1))))
+      return fail(ctx, RS_ERR_INVALID, "replica %d: bad load-spike schedule", r);
     if (p.policy < RS_POLICY_DYNAMO || p.policy > RS_POLICY_P2C)
       return fail(ctx, RS_ERR_INVALID, "replica %d: bad policy", r);
     if (!(p.omega >= 0.0f) || !(p.tau >= 0.0f) || !std::isfinite(p.omega) || !std::isfinite(p.tau))
@@ -554,6 +558,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       return fail(ctx, RS_ERR_INVALID, "replica %d: n_req out of range", r);
     rows += p.n_req;
     cmax = std::max(cmax, p.C);
+    if (p.c_mid > 0) cmax = std::max(cmax, std::max(p.c_mid, p.c_end));
     if (p.controller) pend_cap = std::max(pend_cap, p.n_req);
     win_slots += p.n_req + 2;
     used[p.trace] = 1;
@@ -700,6 +705,10 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     d.n_req = p.n_req;
     d.rec_base = rb;
     d.C = p.C;
+    d.c_t1 = p.c_t1;
+    d.c_t2 = p.c_t2;
+    d.c_mid = p.c_mid > 0 ? p.c_mid : 0;
+    d.c_end = p.c_mid > 0 ? p.c_end : 0;
     d.policy = p.policy;
     d.controller = p.controller ? 1 : 0;
     d.reserved = 0;

@@ -46,6 +46,8 @@ struct SimDesc {
   int32_t C, policy, controller, reserved;
   float omega, tau;
   uint64_t seed;
+  double c_t1, c_t2;        // load-spike schedule: C, then c_mid on [c_t1, c_t2),
+  int32_t c_mid, c_end;     // then c_end (c_mid = 0: C throughout)
 };
 
 struct ModelConsts {

@@ -131,7 +131,8 @@ struct ReqState {
   int64_t blk;     // ceil((L + O) / 16): active blocks while unfinished
   double a;        // arrival
   double rel;      // client release time
-  int nb, nbt, O, phase, full;
+  double twait;    // while waiting for a free client slot: the time reached
+  int nb, nbt, O, phase, full;   // phase 0 new, 2 waiting for a slot, 1 arrival known
   float tau, omega;
 };
 
@@ -145,7 +146,7 @@ struct RawReq {
 struct SimScalars {
   ReqState q[2];
   RawReq nraw;                 // the request after the next one to arrive, as read
-  double prev_arrival, min_ft, tick_t, lastL, ewma, sum_ttft, sum_e2e, makespan;
+  double prev_arrival, min_ft, tick_t, lastL, ewma, sum_ttft, sum_e2e, makespan, first_switch_t;
   int64_t next_tick, np;
   int64_t near_ties, exact_ties, sampled, near_bd, hit_blocks, inserted, evicted, slow, rebuilds;
   int64_t ticks, switches, tir[3], n_routed, probe_blocks, hashed_blocks;
@@ -300,6 +301,7 @@ __device__ __forceinline__ void complete(SimCtx& c, int f, double t) {
 __device__ __forceinline__ void ctl_sample(SimCtx& c, bool has_window, double Lw) {
   SimScalars& S = *c.S;
   const ModelConsts& mc = c.L->mc;
+  const int64_t sw0 = S.switches;
   double L = 0.0;
   if (has_window) {
     L = Lw;
@@ -335,6 +337,7 @@ __device__ __forceinline__ void ctl_sample(SimCtx& c, bool has_window, double Lw
     }
     if (S.regime > S.max_regime) S.max_regime = S.regime;
   }
+  if (sw0 == 0 && S.switches > 0) S.first_switch_t = S.tick_t;   // this sample's time
   S.tir[S.regime]++;
   S.ticks++;
   S.next_tick++;
@@ -352,30 +355,43 @@ __device__ __forceinline__ uint64_t tick_key(const SimCtx& c) {
 __device__ __forceinline__ int events_advance(SimCtx& c, ReqState& q) {
   SimScalars& S = *c.S;
   if (q.phase == 0) {
-    double T = S.prev_arrival;
-    if (S.in_flight >= c.d->C) {
-      for (;;) {
-        if (S.status != RS_OK) return 0;
-        if (S.nheap == 0) {   // cannot happen: every request in flight is in service or queued
-          S.status = RS_ERR_TIMEOUT;
-          return 0;
-        }
-        const uint64_t kc = c.h_k[0];
-        const uint64_t kt = tick_key(c);
-        if (kt < kc) {
-          if (tkey(S.min_ft) >= kt) { ctl_sample(c, false, 0.0); continue; }
-          return 1;
-        }
+    q.twait = S.prev_arrival;
+    q.phase = 2;
+  }
+  if (q.phase == 2) {
+    // closed-loop client (§7.4): wait until fewer than C(t) requests are in
+    // flight; completions, controller samples and steps of the load-spike
+    // schedule in time order (ties in that order)
+    const SimDesc& d = *c.d;
+    for (;;) {
+      const uint64_t kw = tkey(q.twait);
+      const bool mid = d.c_mid > 0 && kw >= tkey(d.c_t1);
+      const bool end = d.c_mid > 0 && kw >= tkey(d.c_t2);
+      const int conc = end ? d.c_end : (mid ? d.c_mid : d.C);
+      if (S.in_flight < conc) break;
+      if (S.status != RS_OK) return 0;
+      const uint64_t kc = S.nheap > 0 ? c.h_k[0] : KEY_INF;
+      const uint64_t kt = tick_key(c);
+      const uint64_t ks = d.c_mid <= 0 || end ? KEY_INF : tkey(mid ? d.c_t2 : d.c_t1);
+      if (kc == KEY_INF && ks == KEY_INF) {   // cannot happen: a request in flight is in service
+        S.status = RS_ERR_TIMEOUT;
+        return 0;
+      }
+      if (kc <= kt && kc <= ks) {
         uint64_t k;
         int f;
         heap_pop(c, &k, &f);
         const double t = tval(k);
         complete(c, f, t);
-        if (k > tkey(T)) T = t;
-        break;
+        if (k > kw) q.twait = t;
+      } else if (kt <= ks) {
+        if (tkey(S.min_ft) >= kt) { ctl_sample(c, false, 0.0); continue; }
+        return 1;
+      } else {
+        q.twait = mid ? d.c_t2 : d.c_t1;   // the schedule steps
       }
     }
-    q.a = tkey(q.rel) > tkey(T) ? q.rel : T;
+    q.a = tkey(q.rel) > tkey(q.twait) ? q.rel : q.twait;
     q.phase = 1;
   }
   const uint64_t ka = tkey(q.a);
@@ -800,7 +816,9 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       reinterpret_cast<uint4*>(st)[s] = make_uint4(STAMP_NONE, STAMP_NONE, STAMP_NONE, STAMP_NONE);
     for (uint32_t s = threadIdx.x; s <= lay.dupmask; s += NT_SIM) c.sc.dupset[s] = 0ull;
     for (int q = 1 + threadIdx.x; q < nft; q += NT_SIM) c.ftab[q] = latency_f(mc, q);
-    for (int p = threadIdx.x; p < d.C; p += NT_SIM) c.freestk[p] = d.C - 1 - p;
+    // request slots: as many as the schedule ever holds in flight
+    const int cslots = max(d.C, max(d.c_mid, d.c_end));
+    for (int p = threadIdx.x; p < cslots; p += NT_SIM) c.freestk[p] = cslots - 1 - p;
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
       c.wmeta[j] = CacheMeta{0u, 0u, 0u, 0u};
       c.winserv[j] = 0;
@@ -813,7 +831,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       S.min_ft = __longlong_as_double(0x7FF0000000000000ll);
       S.next_tick = 1;
       S.tick_t = mc.dt;
-      S.nfree = d.C;
+      S.nfree = max(d.C, max(d.c_mid, d.c_end));
+      S.first_switch_t = -1.0;
     }
     __syncthreads();
   }
@@ -1053,6 +1072,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     r.hashed_blocks = S.hashed_blocks;
     r.slow_path = S.slow;
     r.rebuilds = S.rebuilds;
+    r.first_switch_t = S.first_switch_t;
     b.res[sid] = r;
   }
   for (int j = threadIdx.x; j < W; j += NT_SIM) b.meta_out[(size_t)sid * W + j] = c.wmeta[j];

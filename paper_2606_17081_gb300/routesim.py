@@ -44,7 +44,8 @@ class rs_trace(C.Structure):
 class rs_replica_params(C.Structure):
     _fields_ = [("trace", C.c_int32), ("C", C.c_int32), ("policy", C.c_int32),
                 ("controller", C.c_int32), ("omega", C.c_float), ("tau", C.c_float),
-                ("seed", C.c_uint64), ("n_req", C.c_int64)]
+                ("seed", C.c_uint64), ("n_req", C.c_int64), ("c_t1", C.c_double),
+                ("c_t2", C.c_double), ("c_mid", C.c_int32), ("c_end", C.c_int32)]
 
 
 class rs_replica_result(C.Structure):
@@ -58,7 +59,8 @@ class rs_replica_result(C.Structure):
                 ("reserved0", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
                 ("final_ewma", C.c_double), ("probes", C.c_int64),
                 ("probe_blocks", C.c_int64), ("hashed_blocks", C.c_int64),
-                ("slow_path", C.c_int64), ("rebuilds", C.c_int64), ("poa_static", C.c_double)]
+                ("slow_path", C.c_int64), ("rebuilds", C.c_int64),
+                ("first_switch_t", C.c_double), ("poa_static", C.c_double)]
 
     def as_dict(self) -> dict:
         return {f: (list(getattr(self, f)) if f == "ticks_in_regime" else getattr(self, f))
@@ -276,7 +278,9 @@ def host_trace(trace, pinned: bool = True) -> TraceBuffers:
 
 
 def replica_params(r) -> rs_replica_params:
-    return rs_replica_params(r.trace, r.C, r.policy, r.controller, r.omega, r.tau, r.seed, r.n_req)
+    return rs_replica_params(r.trace, r.C, r.policy, r.controller, r.omega, r.tau, r.seed, r.n_req,
+                             float(getattr(r, "c_t1", 0.0)), float(getattr(r, "c_t2", 0.0)),
+                             int(getattr(r, "c_mid", 0)), int(getattr(r, "c_end", 0)))
 
 
 def device_records(rows: int, W: int, device="cuda", with_cost: bool = False):

@@ -130,6 +130,12 @@ class Replica:
     tau: float
     seed: int             # Philox key for temperature sampling
     n_req: int            # requests of the trace this replica routes
+    # load-spike schedule (Experiment 3): C before c_t1, c_mid on [c_t1, c_t2),
+    # c_end after; c_mid = 0 keeps C throughout
+    c_t1: float = 0.0
+    c_t2: float = 0.0
+    c_mid: int = 0
+    c_end: int = 0
 
 
 @dataclass
@@ -203,6 +209,18 @@ def plan(name: str, n_req: Optional[int] = None, replicas: Optional[list] = None
             reps.append(Replica(ts, C, POLICY_DYNAMO, 0, Ws[cell % 6], Ts[cell // 36], rs, spec.n_req))
             reps.append(Replica(ts, C, POLICY_LOADBAL, 0, 0.0, 0.0, rs, spec.n_req))
         p = Plan(name, W=6, K=32768, spec=spec, trace_seeds=list(range(8)), replicas=reps)
+    elif name == "spike":
+        # Experiment 3's three-phase load spike, C = 32 -> 128 -> 32 for
+        # 120 / 180 / 120 s, on the 70B 1P/2D topology (2 decode workers):
+        # static routing (tau = 0, omega = 1 throughout) against the adaptive
+        # controller, three seeds each; the requests outlast the 420 s.
+        spec = P2D_SPEC
+        reps = []
+        for sd in range(3):
+            for ctl in (0, 1):
+                reps.append(Replica(sd, 32, POLICY_DYNAMO, ctl, 1.0, 0.0, sd, 9000,
+                                    c_t1=120.0, c_t2=300.0, c_mid=128, c_end=32))
+        p = Plan(name, W=2, K=65536, spec=spec, trace_seeds=list(range(3)), replicas=reps)
     elif name == "large":
         spec = LARGE_SPEC
         reps = []

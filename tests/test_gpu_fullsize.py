@@ -64,3 +64,17 @@ def test_large_shape_w64_reduced():
     g = _check(p, range(len(p.replicas)), poa=False)
     assert all(x["result"]["status"] == 0 for x in g)
     assert max(x["result"]["hashed_blocks"] for x in g) > 0
+
+
+def test_load_spike_static_and_adaptive():
+    # Experiment 3's load spike (C = 32 -> 128 -> 32 for 120 / 180 / 120 s, two
+    # decode workers), static and adaptive replicas over three seeds, all in
+    # one launch; the first regime switch times must agree too
+    p = wk.plan("spike")
+    g = _check(p, range(len(p.replicas)))
+    for k, r in enumerate(p.replicas):
+        fs = g[k]["result"]["first_switch_t"]
+        if r.controller:
+            assert fs > r.c_t1          # the adaptive replicas switch during the spike
+        else:
+            assert fs == -1.0
