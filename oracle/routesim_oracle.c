@@ -11,10 +11,11 @@
  * Readings fixed where the paper is silent (each also listed in the design
  * notes of the repository):
  *  - KV blocks hold `block` tokens; only full blocks are hashed and cached.
- *  - Block hash: content g_k = fold of the block's 64-bit little-endian token
- *    pairs through the SplitMix64 finalizer, start 0x9E3779B97F4A7C15 ^ block;
- *    chain h_k = mix(h_{k-1} ^ g_k ^ k), h_{-1} = seed; values 0 and 1 are
- *    reserved and mapped to 2 and 3.
+ *  - Block hash: content g_k = the block's 64-bit little-endian token pairs
+ *    folded by one multiply-xorshift each from 0x9E3779B97F4A7C15 ^ block,
+ *    then the SplitMix64 finalizer; prefix H_k = H_{k-1} P + g_k mod 2^64 with
+ *    H_{-1} = seed, P = 0x94D049BB133111EB; stored h_k = mix(H_k ^ k); values 0
+ *    and 1 are reserved and mapped to 2 and 3.
  *  - b^prefill of Eq. (1) = ceil(L/block) - m_ij, with m_ij the number of
  *    leading blocks found in worker j's cache (first-miss prefix); the overlap
  *    o_ij of Eq. (7) is m_ij / ceil(L/block).
@@ -46,26 +47,32 @@ uint64_t orc_mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
+/* Content of one block: its little-endian 64-bit token pairs folded in
+ * order, one multiply-xorshift each (x = (x ^ w) M, then x ^= x >> 32; M
+ * odd, so each step is a bijection of x and of w), then the SplitMix64
+ * finalizer. */
 static uint64_t block_content(const int32_t* t, int32_t block) {
   uint64_t x = 0x9E3779B97F4A7C15ULL ^ (uint64_t)block;
   for (int32_t q = 0; q < block / 2; q++) {
     uint64_t w = (uint64_t)(uint32_t)t[2 * q] | ((uint64_t)(uint32_t)t[2 * q + 1] << 32);
-    x = orc_mix64(x ^ w);
+    x = (x ^ w) * 0xBF58476D1CE4E5B9ULL;
+    x ^= x >> 32;
   }
-  return x;
+  return orc_mix64(x);
 }
 
-static uint64_t chain_step(uint64_t prev, uint64_t g, int64_t k) {
-  uint64_t h = orc_mix64(prev ^ g ^ (uint64_t)k);
-  if (h < 2) h += 2;
-  return h;
-}
+/* Prefix hash of blocks 0..k (Horner): H_{-1} = seed, H_k = H_{k-1} P + g_k
+ * (mod 2^64, P odd); the stored hash is mix(H_k ^ k), with the values 0 and 1
+ * (the table's empty and tombstone keys) mapped to 2 and 3. */
+#define PREFIX_P 0x94D049BB133111EBULL
 
 static void hash_request(const int32_t* t, int64_t nb, int32_t block, uint64_t seed,
                          uint64_t* out) {
-  uint64_t h = seed;
+  uint64_t H = seed;
   for (int64_t k = 0; k < nb; k++) {
-    h = chain_step(h, block_content(t + k * block, block), k);
+    H = H * PREFIX_P + block_content(t + k * block, block);
+    uint64_t h = orc_mix64(H ^ (uint64_t)k);
+    if (h < 2) h += 2;
     out[k] = h;
   }
 }

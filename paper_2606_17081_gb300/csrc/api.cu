@@ -35,8 +35,7 @@ struct rs_ctx {
   int32_t ninst = 0;
   DevBuf r_keys, r_stamp, r_log, r_tmp, r_meta, r_active, r_ord, r_status, r_hash, r_stats;
   // simulation scratch (grow-only)
-  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, hwork, hlong, dstat,
-      wco, slots;
+  DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, dstat, wco, slots;
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -262,7 +261,7 @@ void route_destroy(rs_ctx* ctx) {
   DevBuf* all[] = {&ctx->r_keys, &ctx->r_stamp, &ctx->r_log, &ctx->r_tmp, &ctx->r_meta,
                    &ctx->r_active, &ctx->r_ord, &ctx->r_status, &ctx->r_hash, &ctx->r_stats,
                    &ctx->keys, &ctx->stamp, &ctx->log, &ctx->tmp, &ctx->pend, &ctx->meta_out,
-                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->hwork, &ctx->hlong, &ctx->slots, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
+                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->slots, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
                    &ctx->rec_arrival, &ctx->rec_start, &ctx->rec_first, &ctx->rec_completion,
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
@@ -294,17 +293,8 @@ rs_status route_hash_blocks(rs_ctx* ctx, const int32_t* tokens_dev, const int64_
 // Hashes every job (trace) in launches of up to HASH_MAX_JOBS traces.
 static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbmax_dev) {
   if (jobs.empty()) return RS_OK;
-  const size_t nlaunch = (jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS;
   rs_status r = ensure(ctx, ctx->hjobs, sizeof(HashJob) * jobs.size(), "hash jobs");
-  int64_t most = 0;   // requests of the largest launch
-  for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
-    const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
-    most = std::max<int64_t>(most, jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - jobs[g0].req_base);
-  }
-  if (r == RS_OK) r = ensure(ctx, ctx->hwork, sizeof(HashSched) * nlaunch, "hash scheduling");
-  if (r == RS_OK) r = ensure(ctx, ctx->hlong, 8 * (size_t)std::max<int64_t>(most, 1), "hash long list");
   if (r != RS_OK) return r;
-  CK(cudaMemsetAsync(ctx->hwork.p, 0, sizeof(HashSched) * nlaunch, ctx->st), "memset");
   CK(cudaMemcpyAsync(ctx->hjobs.p, jobs.data(), sizeof(HashJob) * jobs.size(),
                      cudaMemcpyHostToDevice, ctx->st),
      "copy hash jobs");
@@ -320,8 +310,7 @@ static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbm
                          cudaMemcpyHostToDevice, ctx->st),
          "copy hash jobs");
     CK(launch_block_hash(P<HashJob>(ctx->hjobs) + g0, (int)grp.size(), total, ctx->cfg.hash_seed,
-                         nbmax_dev, P<HashSched>(ctx->hwork) + g0 / HASH_MAX_JOBS,
-                         P<int64_t>(ctx->hlong), ctx->st),
+                         nbmax_dev, ctx->st),
        "block hash launch");
   }
   return RS_OK;
@@ -646,7 +635,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       hashed_tokens += tot[t];
     }
     if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->stats))) != RS_OK) return r;
-    launches += 2 * (((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS);
+    launches += ((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS;
   }
   CK(cudaEventRecord(ctx->ev[1], ctx->st), "event");
   CK(cudaMemcpyAsync(ctx->pinned, ctx->stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");

@@ -34,16 +34,26 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
 }
 
 // content hash g of one 16-token block given as 16 words
+// Content hash of one 16-token block: its 64-bit little-endian token pairs
+// folded in order by one multiply-xorshift each, then the SplitMix64
+// finalizer.
 __device__ __forceinline__ uint64_t block_content16(const uint32_t (&w)[16]) {
   uint64_t x = 0x9E3779B97F4A7C15ull ^ 16ull;
 #pragma unroll
-  for (int q = 0; q < 8; q++) x = mix64(x ^ ((uint64_t)w[2 * q] | ((uint64_t)w[2 * q + 1] << 32)));
-  return x;
+  for (int q = 0; q < 8; q++) {
+    x = (x ^ ((uint64_t)w[2 * q] | ((uint64_t)w[2 * q + 1] << 32))) * 0xBF58476D1CE4E5B9ull;
+    x ^= x >> 32;
+  }
+  return mix64(x);
 }
 
-__device__ __forceinline__ uint64_t chain_step(uint64_t prev, uint64_t gk) {
-  // gk already carries the block index: g_k ^ k
-  uint64_t h = mix64(prev ^ gk);
+// Prefix hash of blocks 0..k: H_k = H_{k-1} P + g_k (mod 2^64), H_{-1} = the
+// hash seed; the stored hash is mix(H_k ^ k), 0 and 1 (the table's empty and
+// tombstone keys) mapped to 2 and 3.
+constexpr uint64_t PREFIX_P = 0x94D049BB133111EBull;
+
+__device__ __forceinline__ uint64_t prefix_output(uint64_t H, uint64_t k) {
+  const uint64_t h = mix64(H ^ k);
   return h < 2 ? h + 2 : h;
 }
 

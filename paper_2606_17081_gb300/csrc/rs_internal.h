@@ -96,16 +96,8 @@ struct HashJob {
   int64_t req_base;
 };
 constexpr int HASH_MAX_JOBS = 64;
-// Scheduling state of one hash launch (zeroed before it): the content pass
-// lists the long prompts, the chain pass hands them out first.
-struct HashSched {
-  unsigned long long work;    // chain pass: next index to hand out
-  unsigned long long nlong;   // prompts in the long list
-};
-// long_list: room for total_req request numbers.
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
-                              int64_t* nbmax_out, HashSched* sched, int64_t* long_list,
-                              cudaStream_t st);
+                              int64_t* nbmax_out, cudaStream_t st);
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st);
 cudaError_t launch_wco_table(double* tab, int nbmax, double w_c, cudaStream_t st);
