@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 32089563648 + 6073165056,
-               "sources_sha256": "95ce82398c6e5fe905df72d7de604e089549b0d502e6afa97f9423d67c14a997",
+SIM_TRAFFIC = {"bytes": 31854879744 + 6050301440,
+               "sources_sha256": "918833786b08d37faf7246658648fea1a0bcd57d4ccb62eda83a2e51780efdd2",
                "summary": "profiles/k_sim_p2d.md"}
 
 
