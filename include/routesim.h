@@ -277,7 +277,7 @@ rs_status route_last_timing(const rs_ctx* ctx, rs_timing* out);
  * cudaFree would synchronise the device.
  *
  * Same result as poa_estimate (Eq. (12) per window of completion time) for
- * caller records of one replica (device pointers, n rows, cfg->W <= 16
+ * caller records of one replica (device pointers, n rows, cfg->W <= 64
  * columns), computed in a fixed static device array of RS_NOALLOC_POA_BYTES
  * bytes that every GPU loading the library holds until the process exits.
  * No context is needed; nothing is allocated (no cudaMalloc, cudaFree or

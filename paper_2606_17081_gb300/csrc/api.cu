@@ -781,8 +781,8 @@ rs_status poa_estimate(rs_ctx* ctx, const rs_records* records, int64_t n, double
   const rs_records& u = *records;
   if (n > 0 && (!u.worker || !u.completion || !u.ttft || !u.nbt || !u.n_frozen || !u.prefix))
     return fail(ctx, RS_ERR_INVALID, "records need worker, completion, ttft, nbt, n_frozen, prefix");
-  if (ctx->cfg.W > POA_WMAX)
-    return fail(ctx, RS_ERR_INVALID, "the PoA estimator supports W <= %d", POA_WMAX);
+  if (ctx->cfg.W > POA_WMAX_WIDE)
+    return fail(ctx, RS_ERR_INVALID, "the PoA estimator supports W <= %d", POA_WMAX_WIDE);
   std::vector<PoaProblem> probs(1);
   probs[0].rec_base = 0;
   probs[0].n = n;

@@ -88,7 +88,7 @@ extern "C" rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records
                                           double* poa_total_dev, int64_t* n_windows_dev,
                                           void* cuda_stream) {
   if (!cfg || !records || !poa_total_dev || !n_windows_dev) return RS_ERR_INVALID;
-  if (cfg->W < 1 || cfg->W > POA_WMAX || cfg->cap < 2 || cfg->cap > 65535 ||
+  if (cfg->W < 1 || cfg->W > POA_WMAX_WIDE || cfg->cap < 2 || cfg->cap > 65535 ||
       !(cfg->poa_window > 0.0))
     return RS_ERR_INVALID;
   if (n < 0 || max_windows < 0) return RS_ERR_INVALID;

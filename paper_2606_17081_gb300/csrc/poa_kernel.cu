@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restric
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
     P.maxw = -1;
-    P.overflow = W > POA_WMAX;
+    P.overflow = W > POA_WMAX_WIDE;
     P.carry = 0;
   }
   if (lane == 0) P.wn[warp] = 0;
@@ -361,6 +361,234 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
   }
 }
 
+// The same OPT for W > POA_WMAX workers, one warp per CTA with its window's
+// W x W edge weights in shared memory.  Lane l owns the target workers
+// k = l, l + 32: it keeps column k of the weights (one pass over the rows
+// updates every source at once) and relaxes dist[k] in Bellman-Ford, all
+// targets of a round in parallel (rounds until nothing changes, at most W), so
+// that no step costs O(W^2) on one lane.
+struct PoaWide {
+  double* wmin;   // [W][W]
+  double* dist;   // [W]
+  int* wrow;      // [W][W]
+  int* pred;      // [W]
+  int* counts;    // [W]
+  int* dirty;     // [W]
+  int* mv_row;    // [W + 1]
+  int* mv_to;     // [W + 1]
+};
+
+__host__ __device__ inline size_t poa_wide_smem(int W) {
+  const size_t w = (size_t)W;
+  return w * w * 12 + w * 12 + w * 8 + 2 * (w + 1) * 4;
+}
+
+// Recompute the weights out of every source j with dirty[j] (all of them when
+// all is set): min over the requests at j of c_qk - c_qj, ties to the lowest row.
+__device__ __forceinline__ void wide_rescan(const PoaWide& S, const PoaBuffers& b,
+                                            int64_t scratch_base, int64_t base, int64_t m,
+                                            int W, int lane, bool all) {
+  const double inf = __longlong_as_double(0x7FF0000000000000ll);
+  for (int k = lane; k < W; k += 32)
+    for (int j = 0; j < W; j++)
+      if (all || S.dirty[j]) { S.wmin[j * W + k] = inf; S.wrow[j * W + k] = -1; }
+  for (int64_t r = 0; r < m; r++) {
+    const int j = b.asg[base + r];
+    if (j < 0 || !(all || S.dirty[j])) continue;
+    const double* cr = b.cost + (scratch_base + b.order[base + r]) * W;
+    const double cj = cr[j];
+    for (int k = lane; k < W; k += 32) {
+      const double v = __dsub_rn(cr[k], cj);
+      if (k != j && v < S.wmin[j * W + k]) { S.wmin[j * W + k] = v; S.wrow[j * W + k] = (int)r; }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restrict__ probs,
+                                                       PoaBuffers b, ModelConsts mc) {
+  extern __shared__ __align__(16) unsigned char wsm[];
+  const int W = mc.W;
+  PoaWide S;
+  {
+    unsigned char* q = wsm;
+    S.wmin = reinterpret_cast<double*>(q); q += (size_t)W * W * 8;
+    S.dist = reinterpret_cast<double*>(q); q += (size_t)W * 8;
+    S.wrow = reinterpret_cast<int*>(q); q += (size_t)W * W * 4;
+    S.pred = reinterpret_cast<int*>(q); q += (size_t)W * 4;
+    S.counts = reinterpret_cast<int*>(q); q += (size_t)W * 4;
+    S.dirty = reinterpret_cast<int*>(q); q += (size_t)W * 4;
+    S.mv_row = reinterpret_cast<int*>(q); q += (size_t)(W + 1) * 4;
+    S.mv_to = reinterpret_cast<int*>(q);
+  }
+  __shared__ int s_err, s_nmv;
+  __shared__ long long s_nrem;
+  const PoaProblem pr = probs[blockIdx.x];
+  const int64_t nw = b.nwin[blockIdx.x];
+  if (nw < 0) return;
+  const int lane = threadIdx.x;
+  const int64_t* wst = b.wstart + pr.win_base + blockIdx.x;
+  for (int64_t w = blockIdx.y; w < nw; w += gridDim.y) {
+    const int64_t s0 = wst[w];
+    const int64_t m = wst[w + 1] - s0;
+    const int64_t base = pr.scratch_base + s0;
+    if (m == 0) {
+      if (lane == 0) {
+        b.wnum[pr.win_base + w] = 0.0;
+        b.wopt[pr.win_base + w] = 0.0;
+        b.wstat[pr.win_base + w] = 0.0;
+        b.wcnt[pr.win_base + w] = 0;
+      }
+      continue;
+    }
+    int64_t capw = (m + W - 1) / W;
+    if (capw < mc.cap) capw = mc.cap;
+    for (int j = lane; j < W; j += 32) S.counts[j] = 0;
+    if (lane == 0) s_err = 0;
+    __syncwarp();
+    double num = 0.0, nst = 0.0;
+    for (int64_t r = lane; r < m; r += 32) {
+      const int q = b.order[base + r];
+      const double* cr = b.cost + (pr.scratch_base + q) * W;
+      nst += cr[b.rec.worker[pr.rec_base + q]];
+      int best = 0;
+      double bc = cr[0];
+      for (int j = 1; j < W; j++)
+        if (cr[j] < bc) { bc = cr[j]; best = j; }
+      b.asg[base + r] = best;
+      atomicAdd(&S.counts[best], 1);
+      num += b.rec.ttft[pr.rec_base + q];
+    }
+    num = warp_sum(num);
+    nst = warp_sum(nst);
+    __syncwarp();
+    int over = 0;
+    for (int j = lane; j < W; j += 32) over |= S.counts[j] > capw;
+    if (__any_sync(FULL_MASK, over)) {
+      if (lane == 0) {   // take out the excess, latest rows first
+        long long nrem = 0;
+        for (int64_t r = m - 1; r >= 0; r--) {
+          const int j = b.asg[base + r];
+          if (S.counts[j] > capw) {
+            S.counts[j]--;
+            b.asg[base + r] = -1;
+            b.wkey[base + nrem++] = (int32_t)r;
+          }
+        }
+        s_nrem = nrem;
+      }
+      __syncwarp();
+      const int64_t nrem = s_nrem;
+      wide_rescan(S, b, pr.scratch_base, base, m, W, lane, true);
+      __syncwarp();
+      for (int64_t e = 0; e < nrem; e++) {
+        const int64_t r0 = b.wkey[base + e];
+        const double* c0 = b.cost + (pr.scratch_base + b.order[base + r0]) * W;
+        for (int k = lane; k < W; k += 32) { S.dist[k] = c0[k]; S.pred[k] = -1; }
+        __syncwarp();
+        // Jacobi rounds: every target reads the previous round's distances.
+        // Only gains above 1e-12 count (exact cycles are >= 0; rounding-level
+        // negative ones must not loop the predecessors).
+        for (int it = 0; it < W; it++) {
+          double nd0 = 0.0, nd1 = 0.0;
+          int np0 = -1, np1 = -1, ch = 0;
+          const int k0 = lane, k1 = lane + 32;
+          if (k0 < W) { nd0 = S.dist[k0]; np0 = S.pred[k0]; }
+          if (k1 < W) { nd1 = S.dist[k1]; np1 = S.pred[k1]; }
+          for (int j = 0; j < W; j++) {
+            const double dj = S.dist[j];
+            if (k0 < W && j != k0 && S.wrow[j * W + k0] >= 0) {
+              const double v = __dadd_rn(dj, S.wmin[j * W + k0]);
+              if (v < nd0 - 1e-12) { nd0 = v; np0 = j; ch = 1; }
+            }
+            if (k1 < W && j != k1 && S.wrow[j * W + k1] >= 0) {
+              const double v = __dadd_rn(dj, S.wmin[j * W + k1]);
+              if (v < nd1 - 1e-12) { nd1 = v; np1 = j; ch = 1; }
+            }
+          }
+          __syncwarp();
+          if (k0 < W) { S.dist[k0] = nd0; S.pred[k0] = np0; }
+          if (k1 < W) { S.dist[k1] = nd1; S.pred[k1] = np1; }
+          ch = __any_sync(FULL_MASK, ch);
+          __syncwarp();
+          if (!ch) break;
+        }
+        if (lane == 0) {
+          int tgt = -1;
+          for (int k = 0; k < W; k++)
+            if (S.counts[k] < capw && (tgt < 0 || S.dist[k] < S.dist[tgt])) tgt = k;
+          int nmv = 0;
+          for (int j = 0; j < W; j++) S.dirty[j] = 0;
+          if (tgt < 0) {
+            s_err = 1;
+          } else {
+            // walk the path back from its end: edge j -> k moves the request
+            // behind wrow[j][k] from j to k
+            int k = tgt, steps = 0;
+            while (S.pred[k] >= 0 && steps <= W) {
+              const int j = S.pred[k];
+              const int r = S.wrow[j * W + k];
+              S.mv_row[nmv] = r;
+              S.mv_to[nmv++] = k;
+              for (int k2 = 0; k2 < W; k2++) S.dirty[j] |= S.wrow[j * W + k2] == r;
+              k = j;
+              steps++;
+            }
+            if (steps > W) {
+              s_err = 1;
+              nmv = 0;
+            } else {
+              for (int t = 0; t < nmv; t++) b.asg[base + S.mv_row[t]] = S.mv_to[t];
+              b.asg[base + r0] = k;
+              S.mv_row[nmv] = (int)r0;
+              S.mv_to[nmv++] = k;
+              S.counts[tgt]++;
+            }
+          }
+          s_nmv = nmv;
+        }
+        __syncwarp();
+        if (s_err) break;
+        // requests that moved in lower their new worker's weights; a dirty
+        // worker is rescanned whole instead
+        const int nmv = s_nmv;
+        for (int t = 0; t < nmv; t++) {
+          const int r = S.mv_row[t], to = S.mv_to[t];
+          if (S.dirty[to]) continue;
+          const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
+          const double ct = cr[to];
+          for (int k2 = lane; k2 < W; k2 += 32) {
+            if (k2 == to) continue;
+            const double v = __dsub_rn(cr[k2], ct);
+            const int wr = S.wrow[to * W + k2];
+            if (wr < 0 || v < S.wmin[to * W + k2] || (v == S.wmin[to * W + k2] && r < wr)) {
+              S.wmin[to * W + k2] = v;
+              S.wrow[to * W + k2] = r;
+            }
+          }
+        }
+        int anyd = 0;
+        for (int j = lane; j < W; j += 32) anyd |= S.dirty[j];
+        if (__any_sync(FULL_MASK, anyd)) wide_rescan(S, b, pr.scratch_base, base, m, W, lane, false);
+        __syncwarp();
+      }
+    }
+    double opt = 0.0;
+    for (int64_t r = lane; r < m; r += 32) {
+      const int q = b.order[base + r];
+      const int a = b.asg[base + r];
+      opt += a >= 0 ? b.cost[(pr.scratch_base + q) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
+    }
+    opt = warp_sum(opt);
+    if (lane == 0) {
+      b.wnum[pr.win_base + w] = num;
+      b.wstat[pr.win_base + w] = nst;
+      b.wopt[pr.win_base + w] = s_err ? __longlong_as_double(0x7FF8000000000000ll) : opt;
+      b.wcnt[pr.win_base + w] = m;
+    }
+    __syncwarp();
+  }
+}
+
 // Whole-run PoA of every replica: one warp per replica, windows summed in
 // order by lane 0 (the same order as a sequential sum).
 __global__ void __launch_bounds__(NT_POA) k_poa_total(int nprob, PoaBuffers b,
@@ -402,7 +630,17 @@ cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int split = (4 * sms + nprob - 1) / nprob;
   split = split < 1 ? 1 : (split > 16 ? 16 : split);
-  k_poa_solve<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
+  if (mc.W <= POA_WMAX) {
+    k_poa_solve<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
+  } else {
+    // one warp per CTA: 8x the CTAs for the same windows in flight
+    const size_t smem = poa_wide_smem(mc.W);
+    if ((e = cudaFuncSetAttribute(k_poa_solve_wide, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)smem)) != cudaSuccess)
+      return e;
+    const int wsplit = split * (NT_POA / 32) > 128 ? 128 : split * (NT_POA / 32);
+    k_poa_solve_wide<<<dim3(nprob, wsplit), 32, smem, st>>>(d_prob, b, mc);
+  }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   k_poa_total<<<(nprob + NT_POA / 32 - 1) / (NT_POA / 32), NT_POA, 0, st>>>(nprob, b, d_prob);
   return cudaGetLastError();

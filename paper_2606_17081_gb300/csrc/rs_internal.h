@@ -11,7 +11,8 @@ namespace rs {
 
 constexpr int NT_SIM = 256;      // threads of a simulation / router CTA
 constexpr int NT_POA = 256;      // threads of a PoA CTA (8 warps, one window each)
-constexpr int POA_WMAX = 16;     // workers supported by the PoA solver
+constexpr int POA_WMAX = 16;     // workers of the per-warp PoA solver (wider: k_poa_solve_wide)
+constexpr int POA_WMAX_WIDE = 64;  // workers supported by the PoA estimate
 constexpr int WMAX = 64;         // workers supported by the simulation
 
 // Per-worker cache bookkeeping (shared memory while a kernel runs, global

@@ -29,8 +29,10 @@ def _check(p, sample, poa=True):
         o = oracle_run(cfg, traces[r.trace], r)
         assert_replica_equal(g[k], o, p.W, check_cost=False)
         if poa:
-            _, _, _, tot = O.poa(cfg, o)
+            _, opt, _, tot = O.poa(cfg, o)
             assert abs(g[k]["result"]["poa_total"] - tot) <= 1e-4 * tot
+            st = float(np.sum(O.static_numer(cfg, o))) / float(np.sum(opt))
+            assert abs(g[k]["result"]["poa_static"] - st) <= 1e-4 * st
     return g
 
 
@@ -56,12 +58,13 @@ def test_large_shape_w64_reduced():
     # 2048 blocks; 1024 prefix groups) and its concurrency C = 4096: the
     # chunked probe, 64 lanes of costs, the per-request slots and event heap in
     # global memory (4096 in flight do not fit beside 2048-block prompts in
-    # shared memory), PoA off (the solver takes W <= 16).  Smaller caches and
-    # fewer requests so that the oracle finishes in seconds.
+    # shared memory) and the wide PoA solver (64 workers, one warp per window,
+    # windows over the per-worker capacity).  Smaller caches and fewer
+    # requests so that the oracle finishes in seconds.
     p = wk.plan("large", n_req=6000, replicas=[0, 8])
     p.K = 1 << 14
     assert all(r.C == 4096 for r in p.replicas)
-    g = _check(p, range(len(p.replicas)), poa=False)
+    g = _check(p, range(len(p.replicas)))
     assert all(x["result"]["status"] == 0 for x in g)
     assert max(x["result"]["hashed_blocks"] for x in g) > 0
 

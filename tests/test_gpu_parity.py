@@ -221,6 +221,40 @@ def test_poa_matches_oracle_per_window():
         assert abs(gt - tot) <= 1e-9 * tot
 
 
+@pytest.mark.parametrize("W", [17, 40, 64])
+def test_poa_wide_solver_per_window(W):
+    # more workers than the per-warp solver holds: four cheap workers take
+    # most requests of every window far over the capacity, so that most
+    # requests are put back along augmenting paths through the other workers
+    rng = np.random.default_rng(300 + W)
+    n = 3000
+    ctx = rs.Context(W=W, K=16)
+    cfg = oracle_cfg(ctx)
+    nbt = rng.integers(1, 200, n).astype(np.int32)
+    nf = rng.integers(24, 63, (n, W))
+    nf[:, :4] = rng.integers(0, 6, (n, 4))
+    pf = np.minimum(rng.integers(0, 200, (n, W)), nbt[:, None])
+    o = {"worker": rng.integers(0, W, n).astype(np.int32),
+         "completion": rng.uniform(0.0, 3.5 * cfg.poa_window, n),
+         "ttft": rng.uniform(0.01, 0.5, n),
+         "nbt": nbt,
+         "n_frozen": nf.astype(np.uint16),
+         "prefix": pf.astype(np.uint16)}
+    o["worker"][::97] = -1          # a few unrouted rows
+    num, opt, cnt, tot = O.poa(cfg, o)
+    assert num.size == 4 and cnt.min() > 4 * 64
+    rec, t = rs.device_records(n, W)
+    for f in ("worker", "completion", "ttft", "nbt"):
+        t[f].copy_(torch.from_numpy(np.ascontiguousarray(o[f])))
+    for f in ("n_frozen", "prefix"):
+        t[f].copy_(torch.from_numpy(o[f].reshape(-1).view(np.int16)))
+    gn, go, gc, gt, nw = rs.poa_estimate(ctx.h, rec, n, num.size + 2)
+    assert nw == num.size and np.array_equal(gc, cnt)
+    assert np.allclose(gn, num, rtol=1e-12, atol=0)
+    assert np.allclose(go, opt, rtol=1e-9, atol=0)
+    assert abs(gt - tot) <= 1e-9 * tot
+
+
 def test_poa_binding_capacity_on_gpu():
     F1 = 0.005 + 0.020 + 0.010 / 63 ** 2
     F2 = 0.010 + 0.020 + 0.010 / 62 ** 2
