@@ -469,6 +469,66 @@ double orc_p99(const double* v, int64_t n) {
   return r;
 }
 
+/* Saturation test of the PoA-growth proposition (§5.1, item 3) over load
+ * sweeps, as Experiment 2 measures it: per replica, the nearest-rank pct-th
+ * percentile of its routed TTFTs (sorted ascending, element ceil(pct n / 100)
+ * - 1, NaN without routed requests); per sweep of replicas in increasing load,
+ * the difference quotient between neighbours and the three-point second
+ * divided difference at interior points; the knee is the first interior point
+ * whose second difference exceeds theta.  Sweep s holds replicas
+ * sweep_start[s] .. sweep_start[s+1] - 1.  Outputs for replicas outside every
+ * sweep, at sweep ends, and in sweeps whose loads do not increase strictly
+ * stay NaN; such a sweep reports knee index -2 and load NaN, a sweep without a
+ * knee -1 and -1. */
+int32_t orc_sweep_knee(int32_t n_rep, const int64_t* row_start, const int32_t* worker,
+                       const double* ttft, const double* load, int32_t n_sweeps,
+                       const int32_t* sweep_start, int32_t pct, double theta, double* stat,
+                       double* d1, double* d2, double* knee_load, int32_t* knee_index) {
+  if (pct < 1 || pct > 100 || n_rep < 0 || n_sweeps < 0) return ORC_ERR_INVALID;
+  for (int32_t r = 0; r < n_rep; r++) {
+    const int64_t a = row_start[r], b = row_start[r + 1];
+    int64_t n = 0;
+    for (int64_t i = a; i < b; i++) n += worker[i] >= 0;
+    d1[r] = NAN;
+    d2[r] = NAN;
+    if (n == 0) {
+      stat[r] = NAN;
+      continue;
+    }
+    double* v = (double*)malloc(sizeof(double) * (size_t)n);
+    if (!v) return ORC_ERR_OOM;
+    int64_t m = 0;
+    for (int64_t i = a; i < b; i++)
+      if (worker[i] >= 0) v[m++] = ttft[i];
+    qsort(v, (size_t)n, sizeof(double), cmp_double);
+    stat[r] = v[((int64_t)pct * n + 99) / 100 - 1];
+    free(v);
+  }
+  for (int32_t s = 0; s < n_sweeps; s++) {
+    const int32_t a = sweep_start[s], b = sweep_start[s + 1];
+    int inc = 1;
+    for (int32_t r = a + 1; r < b; r++)
+      if (!(load[r] > load[r - 1])) inc = 0;
+    if (!inc) {
+      knee_load[s] = NAN;
+      knee_index[s] = -2;
+      continue;
+    }
+    for (int32_t r = a; r + 1 < b; r++)
+      d1[r] = (stat[r + 1] - stat[r]) / (load[r + 1] - load[r]);
+    knee_load[s] = -1.0;
+    knee_index[s] = -1;
+    for (int32_t r = a + 1; r + 1 < b; r++) {
+      d2[r] = 2.0 * (d1[r] - d1[r - 1]) / (load[r + 1] - load[r - 1]);
+      if (knee_index[s] < 0 && d2[r] > theta) {
+        knee_index[s] = r;
+        knee_load[s] = load[r];
+      }
+    }
+  }
+  return ORC_OK;
+}
+
 /* Controller state update for one sample: EWMA of Eq. (10), then the
  * three-regime classifier of Eq. (11) with k-sample hysteresis (§6.2).
  * has_window = 0 means the window held no TTFT: the previous P99 is reused. */

@@ -134,6 +134,14 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
 
 /* Nearest-rank 99th percentile (the controller's TTFT P99 of §6.2). */
 double orc_p99(const double* v, int64_t n);
+/* Saturation knee of load sweeps (§5.1, PoA-growth proposition, item 3;
+ * Experiment 2): per-replica nearest-rank percentile of routed TTFTs, first
+ * and second divided differences over each sweep, first interior point with a
+ * second difference above theta. */
+int32_t orc_sweep_knee(int32_t n_rep, const int64_t* row_start, const int32_t* worker,
+                       const double* ttft, const double* load, int32_t n_sweeps,
+                       const int32_t* sweep_start, int32_t pct, double theta, double* stat,
+                       double* d1, double* d2, double* knee_load, int32_t* knee_index);
 /* The controller alone: one sample per entry of L (NaN = empty window);
  * writes the EWMA of Eq. (10) (-1 before the first sample) and the regime of
  * Eq. (11) after each sample. */

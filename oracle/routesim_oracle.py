@@ -363,6 +363,35 @@ def p99(values) -> float:
     return float(f(_p(v), C.c_int64(v.size)))
 
 
+def sweep_knee(worker, ttft, row_start, load, sweep_start, pct: int = 99,
+               theta: float = 0.0) -> dict:
+    """Saturation knee of load sweeps (§5.1, PoA-growth proposition, item 3;
+    Experiment 2): per replica the nearest-rank pct-th percentile of its routed
+    TTFTs; per sweep the divided differences d1, d2 and the first interior
+    point with d2 > theta (knee_index -1 if none, -2 if loads do not increase)."""
+    wk = _c(worker, np.int32)
+    tt = _c(ttft, np.float64)
+    rows = _c(row_start, np.int64)
+    ld = _c(load, np.float64)
+    sw = _c(sweep_start, np.int32)
+    n_rep = rows.size - 1
+    n_sw = sw.size - 1
+    out = {"stat": np.zeros(max(n_rep, 1)), "d1": np.zeros(max(n_rep, 1)),
+           "d2": np.zeros(max(n_rep, 1)), "knee_load": np.zeros(max(n_sw, 1)),
+           "knee_index": np.zeros(max(n_sw, 1), np.int32)}
+    st = lib().orc_sweep_knee(C.c_int32(n_rep), _p(rows), _p(wk), _p(tt), _p(ld),
+                              C.c_int32(n_sw), _p(sw), C.c_int32(pct), C.c_double(theta),
+                              _p(out["stat"]), _p(out["d1"]), _p(out["d2"]),
+                              _p(out["knee_load"]), _p(out["knee_index"]))
+    if st != OK:
+        raise ValueError(f"orc_sweep_knee rejected the input ({st})")
+    for k in ("stat", "d1", "d2"):
+        out[k] = out[k][:n_rep]
+    for k in ("knee_load", "knee_index"):
+        out[k] = out[k][:n_sw]
+    return out
+
+
 def controller_run(cfg: OracleConfig, L):
     """Feed per-sample P99 values (NaN = empty window); returns (ewma, regime)."""
     x = _c(L, np.float64)

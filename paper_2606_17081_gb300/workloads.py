@@ -221,6 +221,18 @@ def plan(name: str, n_req: Optional[int] = None, replicas: Optional[list] = None
                 reps.append(Replica(sd, 32, POLICY_DYNAMO, ctl, 1.0, 0.0, sd, 9000,
                                     c_t1=120.0, c_t2=300.0, c_mid=128, c_end=32))
         p = Plan(name, W=2, K=65536, spec=spec, trace_seeds=list(range(3)), replicas=reps)
+    elif name == "sat":
+        # Experiment 2's saturation sweep: nine concurrency levels on the 70B
+        # 1P/2D topology, static routing and the adaptive controller, three
+        # seeds; each (seed, controller) pair is one sweep of increasing C.
+        spec = P2D_SPEC
+        Cs = [1, 4, 8, 16, 32, 64, 128, 256, 512]
+        reps = []
+        for sd in range(3):
+            for ctl in (0, 1):
+                for C in Cs:
+                    reps.append(Replica(sd, C, POLICY_DYNAMO, ctl, 1.0, 0.0, sd, 6000))
+        p = Plan(name, W=3, K=65536, spec=spec, trace_seeds=list(range(3)), replicas=reps)
     elif name == "large":
         spec = LARGE_SPEC
         reps = []
@@ -244,3 +256,21 @@ def plan(name: str, n_req: Optional[int] = None, replicas: Optional[list] = None
             r.trace = remap[r.trace]
         p.replicas = keep
     return p
+
+
+def sweeps(replicas) -> list:
+    """Boundaries of the load sweeps of a replica list: maximal runs of
+    consecutive replicas that differ only in C, with C increasing.  Returns
+    sweep_start (len = sweeps + 1) for the knee detector."""
+    def same(a, b):
+        return (a.trace, a.policy, a.controller, a.omega, a.tau, a.seed, a.n_req, a.c_t1,
+                a.c_t2, a.c_mid, a.c_end) == (b.trace, b.policy, b.controller, b.omega, b.tau,
+                                              b.seed, b.n_req, b.c_t1, b.c_t2, b.c_mid, b.c_end)
+    start = [0]
+    for k in range(1, len(replicas)):
+        a, b = replicas[k - 1], replicas[k]
+        if not (same(a, b) and b.C > a.C):
+            start.append(k)
+    if replicas:
+        start.append(len(replicas))
+    return start
