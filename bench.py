@@ -176,6 +176,28 @@ def _alg_bytes(results, W: int) -> float:
     return b
 
 
+def _aux_knee(rs, ctx, p, descs, params, reps: int = 5) -> dict:
+    """Outside the timed steps: the saturation-knee detector over the grid's
+    concurrency sweeps, on the records of one more simulation of the grid
+    (synchronous call: host argument copies, two kernels, result reads)."""
+    from paper_2606_17081_gb300 import workloads as wk
+    n = sum(r.n_req for r in p.replicas)
+    rec, keep = rs.device_records(n, p.W)
+    rs.simulate_replicas(ctx.h, descs, rs.RS_MEM_DEVICE, params, rec)
+    rows = np.concatenate([[0], np.cumsum([r.n_req for r in p.replicas])]).astype(np.int64)
+    load = np.array([r.C for r in p.replicas], np.float64)
+    sw = wk.sweeps(p.replicas)
+    out = rs.sweep_knee(ctx.h, rec, rows, load, sw)
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        out = rs.sweep_knee(ctx.h, rec, rows, load, sw)
+    ms = (time.perf_counter() - t0) * 1e3 / reps
+    del keep
+    return {"sweep_knee": {"ms_per_call": ms, "rows": int(n), "replicas": len(params),
+                           "sweeps": len(sw) - 1, "pct": 99, "theta": 0.0,
+                           "first_knee_C": [float(x) for x in out["knee_load"]]}}
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -244,6 +266,7 @@ def run_gpu(args):
     barrier()
     e2e_s = time.perf_counter() - t0
     ms, e2e_s = _max_over_ranks([ms, e2e_s], "cuda")
+    aux = _aux_knee(rs, ctx, p, descs_d, params) if rank == 0 else None
     if rank != 0:
         if ws > 1:
             dist.destroy_process_group()
@@ -297,6 +320,7 @@ def run_gpu(args):
         "clocks": clocks,
         "gpu_launches": int(launches),
         "cpu_baseline": cpu,
+        "aux": aux,
     }
     print(json.dumps(line))
     if ws > 1:

@@ -270,6 +270,35 @@ typedef struct {
 } rs_timing;
 rs_status route_last_timing(const rs_ctx* ctx, rs_timing* out);
 
+/* Saturation knee of load sweeps (§5.1, the PoA-growth proposition, item 3:
+ * a second derivative of latency with respect to load above a threshold
+ * marks the onset of saturation; Experiment 2 reads the difference quotients
+ * of TTFT P99 across nine concurrency levels).
+ *   records: device records as simulate_replicas wrote them; worker and ttft
+ *     are read.  Replica r owns rows row_start[r] .. row_start[r+1] - 1
+ *     (row_start: host, n_replicas + 1 nondecreasing entries, first >= 0).
+ *   pct (1..100): stat[r] = the nearest-rank pct-th percentile of replica r's
+ *     routed TTFTs (rows with worker >= 0), i.e. element ceil(pct n / 100) - 1
+ *     of them in ascending order; NaN when it routed none.
+ *   load: host, n_replicas entries, the load axis (normally C).
+ *   sweep_start: host, n_sweeps + 1 nondecreasing replica indices <=
+ *     n_replicas; sweep s = replicas sweep_start[s] .. sweep_start[s+1] - 1,
+ *     meant in increasing load.
+ * Outputs, host arrays, each may be NULL:
+ *   stat, d1, d2 (n_replicas entries): d1[r] = (stat[r+1] - stat[r]) /
+ *     (load[r+1] - load[r]) when r + 1 is in r's sweep; d2[r] = 2 (d1[r] -
+ *     d1[r-1]) / (load[r+1] - load[r-1]) at interior points; NaN elsewhere and
+ *     for replicas outside every sweep.
+ *   knee_load, knee_index (n_sweeps entries): the first interior replica of
+ *     the sweep with d2 > theta and its load; -1 / -1 if none; -2 / NaN (and
+ *     no d1, d2) when the sweep's loads do not increase strictly.
+ * Every value is computed on the device; returns after the outputs are
+ * written.  RS_ERR_INVALID for NULL or inconsistent arguments. */
+rs_status sweep_knee(rs_ctx* ctx, const rs_records* records, const int64_t* row_start,
+                     int32_t n_replicas, const double* load, const int32_t* sweep_start,
+                     int32_t n_sweeps, int32_t pct, double theta, double* stat, double* d1,
+                     double* d2, double* knee_load, int32_t* knee_index);
+
 /* Entry point that allocates nothing.  The paper has no counterpart: this
  * is a library service for callers that cannot allocate device memory when
  * they need an estimate -- a serving process whose GPU memory is owned up

@@ -17,8 +17,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libroutesim.so")
-SOURCES = ["hash_kernel.cu", "sim_kernel.cu", "poa_kernel.cu", "router_kernel.cu", "api.cu",
-           "noalloc.cu"]
+SOURCES = ["hash_kernel.cu", "sim_kernel.cu", "poa_kernel.cu", "router_kernel.cu", "knee_kernel.cu",
+           "api.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC",
          "-I" + os.path.join(ROOT, "include"), "-I" + CSRC]

@@ -40,6 +40,7 @@ struct rs_ctx {
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
       p_nwin, p_prob, p_wstat, p_tstat;
+  DevBuf k_rows, k_load, k_sweep, k_stat, k_d1, k_d2, k_kload, k_kidx;
   DevBuf h_tokens, h_offsets, h_release, h_outlen;
   int64_t* pinned = nullptr;   // small host staging for device -> host reads
   size_t pinned_n = 0;
@@ -267,7 +268,8 @@ void route_destroy(rs_ctx* ctx) {
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
                    &ctx->p_wnum, &ctx->p_wopt, &ctx->p_wcnt, &ctx->p_total, &ctx->p_nwin,
                    &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->h_tokens, &ctx->h_offsets,
-                   &ctx->h_release, &ctx->h_outlen};
+                   &ctx->h_release, &ctx->h_outlen, &ctx->k_rows, &ctx->k_load, &ctx->k_sweep,
+                   &ctx->k_stat, &ctx->k_d1, &ctx->k_d2, &ctx->k_kload, &ctx->k_kidx};
   for (DevBuf* b : all) release(*b);
   if (ctx->pinned) cudaFreeHost(ctx->pinned);
   for (auto& ev : ctx->ev)
@@ -813,6 +815,62 @@ rs_status poa_estimate(rs_ctx* ctx, const rs_records* records, int64_t n, double
     if (count_host) CK(cudaMemcpyAsync(count_host, ctx->p_wcnt.p, k * 8, cudaMemcpyDeviceToHost, ctx->st), "read");
     CK(cudaStreamSynchronize(ctx->st), "sync");
   }
+  return RS_OK;
+}
+
+rs_status sweep_knee(rs_ctx* ctx, const rs_records* records, const int64_t* row_start,
+                     int32_t n_replicas, const double* load, const int32_t* sweep_start,
+                     int32_t n_sweeps, int32_t pct, double theta, double* stat_host,
+                     double* d1_host, double* d2_host, double* knee_load_host,
+                     int32_t* knee_index_host) {
+  if (!ctx) return fail(nullptr, RS_ERR_INVALID, "ctx is NULL");
+  ctx->err.clear();
+  if (!records || !row_start || !sweep_start) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
+  if (n_replicas < 0 || n_sweeps < 0) return fail(ctx, RS_ERR_INVALID, "negative count");
+  if (pct < 1 || pct > 100) return fail(ctx, RS_ERR_INVALID, "pct must be in 1..100");
+  if (std::isnan(theta)) return fail(ctx, RS_ERR_INVALID, "theta is NaN");
+  if (row_start[0] < 0) return fail(ctx, RS_ERR_INVALID, "row_start[0] < 0");
+  for (int32_t r = 0; r < n_replicas; r++)
+    if (row_start[r + 1] < row_start[r])
+      return fail(ctx, RS_ERR_INVALID, "row_start decreases at replica %d", r);
+  const int64_t rows = row_start[n_replicas];
+  if (rows > 0 && (!records->worker || !records->ttft))
+    return fail(ctx, RS_ERR_INVALID, "records need worker and ttft");
+  if (n_replicas > 0 && !load) return fail(ctx, RS_ERR_INVALID, "load is NULL");
+  if (sweep_start[0] < 0) return fail(ctx, RS_ERR_INVALID, "sweep_start[0] < 0");
+  for (int32_t s = 0; s < n_sweeps; s++)
+    if (sweep_start[s + 1] < sweep_start[s])
+      return fail(ctx, RS_ERR_INVALID, "sweep_start decreases at sweep %d", s);
+  if (sweep_start[n_sweeps] > n_replicas)
+    return fail(ctx, RS_ERR_INVALID, "sweeps reach past the replicas");
+  const size_t nr = (size_t)n_replicas, ns = (size_t)n_sweeps;
+  rs_status r;
+  if ((r = ensure(ctx, ctx->k_rows, (nr + 1) * 8, "knee rows")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_load, nr * 8, "knee load")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_sweep, (ns + 1) * 4, "knee sweeps")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_stat, nr * 8, "knee stat")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_d1, nr * 8, "knee d1")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_d2, nr * 8, "knee d2")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_kload, ns * 8, "knee load out")) != RS_OK) return r;
+  if ((r = ensure(ctx, ctx->k_kidx, ns * 4, "knee index out")) != RS_OK) return r;
+  CK(cudaMemcpyAsync(ctx->k_rows.p, row_start, (nr + 1) * 8, cudaMemcpyHostToDevice, ctx->st), "copy");
+  if (nr) CK(cudaMemcpyAsync(ctx->k_load.p, load, nr * 8, cudaMemcpyHostToDevice, ctx->st), "copy");
+  CK(cudaMemcpyAsync(ctx->k_sweep.p, sweep_start, (ns + 1) * 4, cudaMemcpyHostToDevice, ctx->st), "copy");
+  CK(launch_sweep_knee(records->worker, records->ttft, P<int64_t>(ctx->k_rows), n_replicas,
+                       P<double>(ctx->k_load), P<int32_t>(ctx->k_sweep), n_sweeps, pct, theta,
+                       P<double>(ctx->k_stat), P<double>(ctx->k_d1), P<double>(ctx->k_d2),
+                       P<double>(ctx->k_kload), P<int32_t>(ctx->k_kidx), ctx->st),
+     "knee launch");
+  if (nr) {
+    if (stat_host) CK(cudaMemcpyAsync(stat_host, ctx->k_stat.p, nr * 8, cudaMemcpyDeviceToHost, ctx->st), "read");
+    if (d1_host) CK(cudaMemcpyAsync(d1_host, ctx->k_d1.p, nr * 8, cudaMemcpyDeviceToHost, ctx->st), "read");
+    if (d2_host) CK(cudaMemcpyAsync(d2_host, ctx->k_d2.p, nr * 8, cudaMemcpyDeviceToHost, ctx->st), "read");
+  }
+  if (ns) {
+    if (knee_load_host) CK(cudaMemcpyAsync(knee_load_host, ctx->k_kload.p, ns * 8, cudaMemcpyDeviceToHost, ctx->st), "read");
+    if (knee_index_host) CK(cudaMemcpyAsync(knee_index_host, ctx->k_kidx.p, ns * 4, cudaMemcpyDeviceToHost, ctx->st), "read");
+  }
+  CK(cudaStreamSynchronize(ctx->st), "sync");
   return RS_OK;
 }
 

@@ -132,6 +132,12 @@ struct PoaBuffers {
   rs_replica_result* res;   // optional [problems] (poa_total, n_windows filled)
 };
 
+// Saturation knee of load sweeps: per-replica percentile, divided differences, knee.
+cudaError_t launch_sweep_knee(const int32_t* worker, const double* ttft, const int64_t* row_start,
+                              int n_rep, const double* load, const int32_t* sweep_start,
+                              int n_sweeps, int pct, double theta, double* stat, double* d1,
+                              double* d2, double* knee_load, int32_t* knee_index,
+                              cudaStream_t st);
 cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
                        const ModelConsts& mc, cudaStream_t st);
 

@@ -82,7 +82,7 @@ class rs_timing(C.Structure):
 EXPORTS = ["rs_config_default", "route_init", "route_destroy", "route_last_error",
            "route_hash_blocks", "route_batch", "route_release", "route_active",
            "simulate_replicas", "poa_estimate", "route_cache_dump", "route_last_timing",
-           "poa_estimate_noalloc"]
+           "poa_estimate_noalloc", "sweep_knee"]
 
 _lib = None
 
@@ -120,6 +120,8 @@ def lib():
             "route_last_timing": (i32, [vp, C.POINTER(rs_timing)]),
             "poa_estimate_noalloc": (i32, [C.POINTER(rs_config), C.POINTER(rs_records), i64, vp,
                                            vp, vp, i64, vp, vp, vp]),
+            "sweep_knee": (i32, [vp, C.POINTER(rs_records), vp, i32, vp, vp, i32, i32,
+                                 C.c_double, vp, vp, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -231,6 +233,27 @@ def route_last_timing(ctx) -> rs_timing:
     t = rs_timing()
     lib().route_last_timing(ctx, C.byref(t))
     return t
+
+
+def sweep_knee(ctx, records: rs_records, row_start, load, sweep_start, pct: int = 99,
+               theta: float = 0.0) -> dict:
+    """Saturation knee of load sweeps over device records: per-replica
+    percentile of routed TTFTs, divided differences, first interior level with
+    a second difference above theta."""
+    rows = np.ascontiguousarray(row_start, np.int64)
+    ld = np.ascontiguousarray(load, np.float64)
+    sw = np.ascontiguousarray(sweep_start, np.int32)
+    nr, ns = rows.size - 1, sw.size - 1
+    out = {"stat": np.zeros(max(nr, 1)), "d1": np.zeros(max(nr, 1)), "d2": np.zeros(max(nr, 1)),
+           "knee_load": np.zeros(max(ns, 1)), "knee_index": np.zeros(max(ns, 1), np.int32)}
+    _check(lib().sweep_knee(ctx, C.byref(records), _ptr(rows), nr, _ptr(ld), _ptr(sw), ns, pct,
+                            theta, _ptr(out["stat"]), _ptr(out["d1"]), _ptr(out["d2"]),
+                            _ptr(out["knee_load"]), _ptr(out["knee_index"])), ctx)
+    for k in ("stat", "d1", "d2"):
+        out[k] = out[k][:nr]
+    for k in ("knee_load", "knee_index"):
+        out[k] = out[k][:ns]
+    return out
 
 
 def poa_estimate_noalloc(cfg: rs_config, records: rs_records, n: int, numer_dev, opt_dev,
