@@ -24,6 +24,12 @@
  *  - Eviction: exact LRU; the chosen worker touches every full block of the
  *    prompt in order (hits move to most-recent, misses are inserted, evicting
  *    the least-recent entry when full).
+ *  - Frequency eviction (the KV Block Manager of §2.2, the alternative): every
+ *    block carries a frequency, 1 when inserted, doubled on a hit (at most
+ *    freq_max) and lowered by 1 per decay step (never below 1); decay step
+ *    floor(a_i / decay_s) at request i's arrival.  Frequency 1 is cold, 2 and
+ *    more (eligible for promotion) hot.  The victim is the least recently used
+ *    cold block, or the least recently used block when every block is hot.
  *  - Ties of the argmin go to the lowest worker index.  Temperature sampling
  *    uses Philox4x32-10 and a 24-bit uniform.
  *  - Service: a worker serves at most cap-1 = 63 requests at once (the pole of
@@ -211,6 +217,7 @@ typedef struct {
   int64_t K, size, head /* least recent */, tail /* most recent */, nfree;
   uint64_t* key;
   int64_t *prev, *next, *chain, *freel, *bucket;
+  int64_t* freq;        /* frequency of each node (frequency eviction) */
   uint64_t mask;
 } lru_t;
 
@@ -226,7 +233,9 @@ static int lru_init(lru_t* c, int64_t K) {
   c->chain = (int64_t*)malloc(sizeof(int64_t) * K);
   c->freel = (int64_t*)malloc(sizeof(int64_t) * K);
   c->bucket = (int64_t*)malloc(sizeof(int64_t) * nb);
-  if (!c->key || !c->prev || !c->next || !c->chain || !c->freel || !c->bucket) return -1;
+  c->freq = (int64_t*)malloc(sizeof(int64_t) * K);
+  if (!c->key || !c->prev || !c->next || !c->chain || !c->freel || !c->bucket || !c->freq)
+    return -1;
   for (uint64_t b = 0; b < nb; b++) c->bucket[b] = -1;
   for (int64_t n = 0; n < K; n++) c->freel[n] = K - 1 - n;
   c->nfree = K;
@@ -236,6 +245,7 @@ static int lru_init(lru_t* c, int64_t K) {
 
 static void lru_free(lru_t* c) {
   free(c->key); free(c->prev); free(c->next); free(c->chain); free(c->freel); free(c->bucket);
+  free(c->freq);
 }
 
 static int64_t lru_find(const lru_t* c, uint64_t key) {
@@ -261,11 +271,28 @@ static void lru_touch(lru_t* c, int64_t n) {
   list_push_recent(c, n);
 }
 
-/* insert an absent key as most recent; returns 1 if an entry was evicted */
-static int lru_insert(lru_t* c, uint64_t key) {
+/* frequency eviction: `steps` decay steps lower every frequency by 1 each,
+ * never below 1 */
+static void freq_decay(lru_t* c, int64_t steps) {
+  for (int64_t n = c->head; n >= 0; n = c->next[n])
+    c->freq[n] = c->freq[n] - steps > 1 ? c->freq[n] - steps : 1;
+}
+
+/* frequency eviction's victim: the least recently used block of frequency 1
+ * (cold); when every block is hot, the least recently used block */
+static int64_t freq_victim(const lru_t* c) {
+  for (int64_t n = c->head; n >= 0; n = c->next[n])
+    if (c->freq[n] < 2) return n;
+  return c->head;
+}
+
+/* insert an absent key as most recent (frequency 1); when the cache is full
+ * the LRU entry (mode LRU) or the frequency rule's victim (mode FREQ) goes
+ * first.  Returns 1 if an entry was evicted. */
+static int lru_insert(lru_t* c, uint64_t key, int32_t mode) {
   int evicted = 0;
   if (c->size == c->K) {
-    int64_t v = c->head;
+    int64_t v = mode == ORC_EVICT_FREQ ? freq_victim(c) : c->head;
     list_unlink(c, v);
     int64_t* link = &c->bucket[c->key[v] & c->mask];
     while (*link != v) link = &c->chain[*link];
@@ -276,6 +303,7 @@ static int lru_insert(lru_t* c, uint64_t key) {
   }
   int64_t n = c->freel[--c->nfree];
   c->key[n] = key;
+  c->freq[n] = 1;
   c->chain[n] = c->bucket[key & c->mask];
   c->bucket[key & c->mask] = n;
   list_push_recent(c, n);
@@ -310,15 +338,17 @@ static int64_t cached_prefix(const lru_t* c, const uint64_t* h, int64_t nb) {
   return m;
 }
 
-/* the chosen worker touches the prompt's blocks in order */
+/* the chosen worker touches the prompt's blocks in order; under frequency
+ * eviction a hit doubles the block's frequency, up to freq_max */
 static void cache_update(lru_t* c, const uint64_t* h, int64_t nb, int64_t* inserted,
-                         int64_t* evicted) {
+                         int64_t* evicted, int32_t mode, int64_t freq_max) {
   for (int64_t k = 0; k < nb; k++) {
     int64_t n = lru_find(c, h[k]);
     if (n >= 0) {
       lru_touch(c, n);
+      if (mode == ORC_EVICT_FREQ) c->freq[n] = 2 * c->freq[n] < freq_max ? 2 * c->freq[n] : freq_max;
     } else {
-      *evicted += lru_insert(c, h[k]);
+      *evicted += lru_insert(c, h[k], mode);
       *inserted += 1;
     }
   }
@@ -637,13 +667,18 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
                      int64_t max_ticks) {
   memset(sum, 0, sizeof *sum);
   sum->first_switch_t = -1.0;
+  sum->first_evict_t = -1.0;
+  sum->rho_first_evict = -1.0;
   const int32_t W = cfg->W;
   const int64_t n = rep->n_req;
   if (W < 1 || cfg->block < 2 || (cfg->block & 1) || cfg->K < 1 || cfg->cap < 2 || rep->C < 1 ||
       n < 0 || !(rep->tau >= 0.0f) || !(rep->omega >= 0.0f) ||
       rep->policy < ORC_POLICY_DYNAMO || rep->policy > ORC_POLICY_P2C ||
       (rep->c_mid > 0 && (rep->c_end < 1 || !(rep->c_t1 >= 0.0) || !(rep->c_t2 >= rep->c_t1))) ||
-      rep->c_mid < 0) {
+      rep->c_mid < 0 || rep->eviction < ORC_EVICT_LRU || rep->eviction > ORC_EVICT_FREQ ||
+      (rep->eviction == ORC_EVICT_FREQ &&
+       (rep->freq_max < 1 || rep->freq_max > (1 << 20) || !(rep->decay_s > 0.0) ||
+        !(rep->decay_s < INFINITY)))) {
     sum->status = ORC_ERR_INVALID;
     return ORC_ERR_INVALID;
   }
@@ -698,6 +733,7 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   const int32_t B = cfg->block;
   const int64_t slots = cfg->cap - 1;
   double prev_arrival = 0.0;
+  int64_t dclock = 0;   /* decay steps applied so far (frequency eviction) */
 
   for (int64_t i = 0; i < n; i++) {
     /* closed-loop client (§7.4): request i waits until fewer than C(t)
@@ -799,7 +835,24 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
       sum->sampled++;
       sum->near_boundary += near_boundary(c, W, tau, u24);
     }
-    cache_update(&s.cache[jstar], h, nb, &sum->inserted_blocks, &sum->evicted_blocks);
+    if (rep->eviction == ORC_EVICT_FREQ) {
+      /* the decay steps since the last request, applied to every block */
+      double q = floor(a / rep->decay_s);
+      int64_t D = q < 2147483648.0 ? (int64_t)q : 2147483648ll;
+      if (D > dclock) {
+        for (int32_t j = 0; j < W; j++) freq_decay(&s.cache[j], D - dclock);
+        dclock = D;
+      }
+    }
+    const int64_t ev0 = sum->evicted_blocks;
+    cache_update(&s.cache[jstar], h, nb, &sum->inserted_blocks, &sum->evicted_blocks,
+                 rep->eviction, rep->freq_max);
+    if (ev0 == 0 && sum->evicted_blocks > 0) {
+      int64_t live = 0;
+      for (int32_t j = 0; j < W; j++) live += s.cache[j].size;
+      sum->first_evict_t = a;
+      sum->rho_first_evict = (double)live / ((double)W * (double)cfg->K);
+    }
     sum->hit_blocks += m[jstar];
     s.A[jstar] += s.blk[i];
     s.in_flight++;
@@ -824,6 +877,11 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   }
   sum->final_regime = s.ctl.regime;
   sum->final_ewma = s.ctl.have_ewma ? s.ctl.ewma : -1.0;
+  {
+    int64_t live = 0;
+    for (int32_t j = 0; j < W; j++) live += s.cache[j].size;
+    sum->rho_end = (double)live / ((double)W * (double)cfg->K);
+  }
   sum->regime_switches = s.ctl.switches;
   if (cache_sizes || cache_keys) {
     for (int32_t j = 0; j < W; j++) {
@@ -1291,7 +1349,7 @@ int32_t orc_router_route(orc_router* r, int32_t inst, const int32_t* tokens,
     uint32_t u24 = r->tau > 0.0f ? draw_u24(r->seed, r->ordinal[inst], (uint32_t)inst, TAG_ROUTE)
                                  : 0u;
     int32_t js = orc_select(c, W, r->tau, u24);
-    cache_update(&cache[js], h, nb, &ins, &ev);
+    cache_update(&cache[js], h, nb, &ins, &ev, ORC_EVICT_LRU, 1);
     A[js] += (L + out_len[i] + B - 1) / B;
     worker[i] = js;
     r->ordinal[inst]++;

@@ -46,6 +46,9 @@ enum {
 enum { ORC_POLICY_DYNAMO = 0, ORC_POLICY_LOADBAL = 1,
        /* static counterfactual policies (§9, routing baselines) */
        ORC_POLICY_ROUNDROBIN = 2, ORC_POLICY_RANDOM = 3, ORC_POLICY_P2C = 4 };
+/* eviction of the per-worker block caches: exact LRU, or the KV Block
+ * Manager's frequency rule (§2.2) */
+enum { ORC_EVICT_LRU = 0, ORC_EVICT_FREQ = 1 };
 
 typedef struct {
   int32_t W;              /* decode workers (routing-game resources) */
@@ -77,6 +80,10 @@ typedef struct {
    * c_end from c_t2 on; c_mid = 0 keeps C */
   double c_t1, c_t2;
   int32_t c_mid, c_end;
+  /* cache eviction (ORC_EVICT_*); for FREQ the frequency cap (>= 1) and the
+   * length of one decay step in s of simulated time (> 0) */
+  int32_t eviction, freq_max;
+  double decay_s;
 } orc_replica;
 
 typedef struct {
@@ -90,6 +97,11 @@ typedef struct {
   int64_t ticks_in_regime[3];
   double final_ewma;
   double first_switch_t;   /* first regime switch, -1 if none */
+  /* KV-cache pressure (the regime-transition proposition of §5.3): arrival
+   * time of the first request whose update evicted, and rho = resident
+   * blocks over W K after that update (-1, -1 if nothing was evicted);
+   * rho after the last request */
+  double first_evict_t, rho_first_evict, rho_end;
 } orc_summary;
 
 /* Per-request outputs; every pointer may be NULL.  Arrays of n (or n*W). */

@@ -21,6 +21,8 @@ OK, ERR_INVALID, ERR_OOM, ERR_CAPACITY, ERR_COLLISION = 0, -1, -2, -3, -7
 POLICY_DYNAMO, POLICY_LOADBAL = 0, 1
 # static counterfactual policies of the routing-baselines discussion (§9)
 POLICY_ROUNDROBIN, POLICY_RANDOM, POLICY_P2C = 2, 3, 4
+# cache eviction: exact LRU, or the KV Block Manager's frequency rule (§2.2)
+EVICT_LRU, EVICT_FREQ = 0, 1
 
 
 def build_oracle(force: bool = False) -> str:
@@ -48,7 +50,8 @@ class _Replica(C.Structure):
     _fields_ = [("C", C.c_int32), ("policy", C.c_int32), ("controller", C.c_int32),
                 ("omega", C.c_float), ("tau", C.c_float), ("seed", C.c_uint64),
                 ("n_req", C.c_int64), ("c_t1", C.c_double), ("c_t2", C.c_double),
-                ("c_mid", C.c_int32), ("c_end", C.c_int32)]
+                ("c_mid", C.c_int32), ("c_end", C.c_int32), ("eviction", C.c_int32),
+                ("freq_max", C.c_int32), ("decay_s", C.c_double)]
 
 
 class _Summary(C.Structure):
@@ -59,7 +62,9 @@ class _Summary(C.Structure):
                 ("evicted_blocks", C.c_int64), ("ticks", C.c_int64),
                 ("regime_switches", C.c_int64), ("final_regime", C.c_int32),
                 ("max_regime", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
-                ("final_ewma", C.c_double), ("first_switch_t", C.c_double)]
+                ("final_ewma", C.c_double), ("first_switch_t", C.c_double),
+                ("first_evict_t", C.c_double), ("rho_first_evict", C.c_double),
+                ("rho_end", C.c_double)]
 
 
 class _Records(C.Structure):
@@ -182,10 +187,12 @@ def hash_blocks(tokens, offsets, block: int = 16, seed: int = 0) -> np.ndarray:
 def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
              controller: int = 0, omega: float = 1.0, tau: float = 0.0, seed: int = 0,
              n_req=None, want_cache: bool = False, max_ticks: int = 0,
-             schedule=None) -> dict:
+             schedule=None, eviction: int = EVICT_LRU, freq_max: int = 64,
+             decay_s: float = 1.0) -> dict:
     """Run one replica.  `trace` has tokens/offsets/release/out_len arrays.
     schedule: None or (c_t1, c_t2, c_mid, c_end), the load-spike concurrency
-    of Experiment 3 (C before c_t1, c_mid until c_t2, c_end after)."""
+    of Experiment 3 (C before c_t1, c_mid until c_t2, c_end after).
+    eviction: EVICT_LRU, or EVICT_FREQ with its frequency cap and decay step."""
     n = trace.n_req if n_req is None else int(n_req)
     W = cfg.W
     t = _c(trace.tokens, np.int32)
@@ -204,7 +211,7 @@ def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
                                                 "prefix", "cost")])
     st = schedule if schedule is not None else (0.0, 0.0, 0, 0)
     rep = _Replica(C_, policy, controller, omega, tau, seed, n, float(st[0]), float(st[1]),
-                   int(st[2]), int(st[3]))
+                   int(st[2]), int(st[3]), int(eviction), int(freq_max), float(decay_s))
     s = _Summary()
     keys = np.zeros(W * cfg.K, np.uint64) if want_cache else None
     sizes = np.zeros(W, np.int64) if want_cache else None
