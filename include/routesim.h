@@ -70,6 +70,10 @@ enum { RS_POLICY_DYNAMO = 0,   /* Eq. (1) cost with the replica's omega, tau */
                                       (x0, x1 of one Philox draw), the lower Eq. (1)
                                       cost wins, ties to the lower index */ };
 
+/* Eviction of the simulated per-worker caches: exact LRU, or the KV Block
+ * Manager's frequency rule (§2.2; see rs_replica_params.eviction). */
+enum { RS_EVICT_LRU = 0, RS_EVICT_FREQ = 1 };
+
 enum { RS_MEM_DEVICE = 0, RS_MEM_HOST = 1 };
 
 /* Model and controller constants.  rs_config_default() fills the paper's:
@@ -181,6 +185,16 @@ typedef struct {
    * simulated time).  c_mid = 0: C throughout (the times are ignored). */
   double c_t1, c_t2;
   int32_t c_mid, c_end;
+  /* Cache eviction (RS_EVICT_*).  RS_EVICT_FREQ is the KV Block Manager's
+   * frequency rule (§2.2): a block's frequency is 1 when inserted, doubles
+   * on a hit up to freq_max (1 .. 2^20) and drops by 1 per decay step of
+   * decay_s seconds of simulated time (> 0, finite; step floor(a_i / decay_s)
+   * at request i's arrival), never below 1.  Frequency 1 is cold, 2 and more
+   * hot; the victim is the least recently used cold block, or the least
+   * recently used block when all are hot.  freq_max = 1 is exact LRU.
+   * Both fields are ignored under RS_EVICT_LRU. */
+  int32_t eviction, freq_max;
+  double decay_s;
 } rs_replica_params;
 
 typedef struct {
@@ -210,6 +224,10 @@ typedef struct {
   double poa_static;        /* the realized assignment under the frozen cost model of
                                §6.4: sum over windows of sum_i c_{i, worker(i)} over
                                the sum of OPTs (the static counterfactual of §9) */
+  /* KV-cache pressure (the regime-transition proposition of §5.3, rho =
+   * resident blocks / (W K)): arrival time of the first request whose update
+   * evicted and rho just after that update (-1, -1 if none); rho at the end */
+  double first_evict_t, rho_first_evict, rho_end;
 } rs_replica_result;
 
 /* Per-request records, device memory, each pointer may be NULL.  Replica r's

@@ -36,6 +36,7 @@ struct rs_ctx {
   DevBuf r_keys, r_stamp, r_log, r_tmp, r_meta, r_active, r_ord, r_status, r_hash, r_stats;
   // simulation scratch (grow-only)
   DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, dstat, wco, slots;
+  DevBuf fexp, tmpe;   // frequency eviction state and its rebuild scratch
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -269,7 +270,8 @@ void route_destroy(rs_ctx* ctx) {
                    &ctx->p_wnum, &ctx->p_wopt, &ctx->p_wcnt, &ctx->p_total, &ctx->p_nwin,
                    &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->h_tokens, &ctx->h_offsets,
                    &ctx->h_release, &ctx->h_outlen, &ctx->k_rows, &ctx->k_load, &ctx->k_sweep,
-                   &ctx->k_stat, &ctx->k_d1, &ctx->k_d2, &ctx->k_kload, &ctx->k_kidx};
+                   &ctx->k_stat, &ctx->k_d1, &ctx->k_d2, &ctx->k_kload, &ctx->k_kidx,
+                   &ctx->fexp, &ctx->tmpe};
   for (DevBuf* b : all) release(*b);
   if (ctx->pinned) cudaFreeHost(ctx->pinned);
   for (auto& ev : ctx->ev)
@@ -532,6 +534,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   }
   int64_t rows = 0, pend_cap = 0, win_slots = 0;
   int cmax = 1;
+  bool any_freq = false;   // a replica evicts by frequency: its tables need fexp
   std::vector<char> used(n_traces, 0);
   for (int r = 0; r < n_replicas; r++) {
     const rs_replica_params& p = params[r];
@@ -543,6 +546,15 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       return fail(ctx, RS_ERR_INVALID, "replica %d: bad load-spike schedule", r);
     if (p.policy < RS_POLICY_DYNAMO || p.policy > RS_POLICY_P2C)
       return fail(ctx, RS_ERR_INVALID, "replica %d: bad policy", r);
+    if (p.eviction != RS_EVICT_LRU && p.eviction != RS_EVICT_FREQ)
+      return fail(ctx, RS_ERR_INVALID, "replica %d: bad eviction", r);
+    if (p.eviction == RS_EVICT_FREQ) {
+      if (p.freq_max < 1 || p.freq_max > (1 << 20))
+        return fail(ctx, RS_ERR_INVALID, "replica %d: freq_max out of 1..2^20", r);
+      if (!(p.decay_s > 0.0) || !std::isfinite(p.decay_s))
+        return fail(ctx, RS_ERR_INVALID, "replica %d: decay_s must be finite and > 0", r);
+      any_freq = true;
+    }
     if (!(p.omega >= 0.0f) || !(p.tau >= 0.0f) || !std::isfinite(p.omega) || !std::isfinite(p.tau))
       return fail(ctx, RS_ERR_INVALID, "replica %d: omega/tau must be finite and >= 0", r);
     if (p.n_req < 0 || p.n_req > traces[p.trace].n_req)
@@ -675,6 +687,9 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   if (slots_global &&
       (r = ensure(ctx, ctx->slots, nsim * sim_slot_bytes(cmax), "request slots")) != RS_OK)
     return r;
+  if (any_freq && ((r = ensure(ctx, ctx->fexp, nsl * 4, "frequency state")) ||
+                   (r = ensure(ctx, ctx->tmpe, nsim * g.K * 4, "frequency rebuild scratch"))))
+    return r;
   // w_c * (m / nbt) table for prompts up to nbmax blocks (none beyond 2048)
   const bool use_tab = nbmax <= 2048;
   if (use_tab &&
@@ -702,7 +717,10 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     d.c_end = p.c_mid > 0 ? p.c_end : 0;
     d.policy = p.policy;
     d.controller = p.controller ? 1 : 0;
+    d.eviction = p.eviction;
+    d.freq_max = p.eviction == RS_EVICT_FREQ ? p.freq_max : 1;
     d.reserved = 0;
+    d.decay_s = p.eviction == RS_EVICT_FREQ ? p.decay_s : 1.0;
     d.omega = p.omega;
     d.tau = p.tau;
     d.seed = p.seed;
@@ -721,6 +739,8 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   sb.stamp = P<uint32_t>(ctx->stamp);
   sb.log = P<uint32_t>(ctx->log);
   sb.tmp = P<uint64_t>(ctx->tmp);
+  sb.fexp = any_freq ? P<uint32_t>(ctx->fexp) : nullptr;
+  sb.tmpe = any_freq ? P<uint32_t>(ctx->tmpe) : nullptr;
   sb.pend = P<double>(ctx->pend);
   sb.pend_cap = std::max<int64_t>(pend_cap, 1);
   sb.meta_out = P<CacheMeta>(ctx->meta_out);

@@ -72,6 +72,7 @@ __global__ void __launch_bounds__(NT_SIM) k_route_batch(
     t.keys = s.keys + (size_t)j * g.slots;
     t.stamp = s.stamp + (size_t)j * g.slots;
     t.log = s.log + (size_t)j * g.R;
+    t.fexp = nullptr;
     t.bmask = g.bmask;
     t.rmask = g.rmask;
     return t;
@@ -226,7 +227,7 @@ __global__ void k_clear_tables(uint64_t* keys, uint32_t* stamp, size_t nslots, C
     stamp[s] = STAMP_NONE;
   }
   for (size_t s = (size_t)blockIdx.x * blockDim.x + threadIdx.x; s < nmeta; s += stride)
-    meta[s] = CacheMeta{0u, 0u, 0u, 0u};
+    meta[s] = CacheMeta{};
 }
 
 cudaError_t launch_clear_tables(uint64_t* keys, uint32_t* stamp, size_t nslots, CacheMeta* meta,

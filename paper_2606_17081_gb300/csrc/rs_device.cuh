@@ -256,6 +256,7 @@ struct TableView {
   uint64_t* keys;     // [BUCKET * nbuckets]
   uint32_t* stamp;    // [BUCKET * nbuckets]
   uint32_t* log;      // [rmask + 1]
+  uint32_t* fexp;     // [BUCKET * nbuckets] frequency eviction state, or NULL
   uint32_t bmask;     // nbuckets - 1
   uint32_t rmask;     // log ring size - 1
 };
@@ -390,11 +391,19 @@ struct UpdateShared {   // small shared scalars of the update
   uint32_t pmin, gathered;
 };
 
+struct FreqShared {   // small shared scalars of the frequency update
+  // where the victim search started, least e and first position of the hot
+  // entries it passed, hot entries listed for the exact path
+  uint32_t fstart, femin, fhot, gb;
+};
+
 // Rebuilds the table and log of one worker from its live entries in LRU
 // order (stamps renumbered 0..size-1).  tmp: global scratch of >= size keys.
 template <int NT>
 __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* meta, uint32_t K, uint64_t* tmp,
-                              int* warp_tot, UpdateShared* us) {
+                              int* warp_tot, UpdateShared* us, uint32_t* tmpe = nullptr,
+                              FreqMeta* fm = nullptr) {
+  const bool fx = t.fexp != nullptr && tmpe != nullptr;   // frequencies move with their keys
   const uint32_t head = meta->head, T = meta->T;
   constexpr int PER = 8;   // log entries per thread per step: independent loads in flight
   uint32_t base = 0;
@@ -415,7 +424,10 @@ __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* met
 #pragma unroll
     for (int e = 0; e < PER; e++)
       if (live[e]) {
-        if (base + off < K) tmp[base + off] = __ldcg(t.keys + x[e]);
+        if (base + off < K) {
+          tmp[base + off] = __ldcg(t.keys + x[e]);
+          if (fx) tmpe[base + off] = __ldcg(t.fexp + x[e]);
+        }
         off++;
       }
     base += tot;
@@ -439,6 +451,7 @@ __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* met
     else {
       t.stamp[sl] = r;
       t.log[r & t.rmask] = sl;
+      if (fx) t.fexp[sl] = __ldcg(tmpe + r);
     }
   }
   grp_bar<NT>();
@@ -447,6 +460,7 @@ __device__ __forceinline__ void cache_rebuild(const TableView& t, CacheMeta* met
     meta->head = 0;
     meta->T = base;
     meta->tombs = 0;
+    if (fm) *fm = FreqMeta{0u, 0u};
   }
   grp_bar<NT>();
 }
@@ -480,6 +494,13 @@ __device__ __forceinline__ void update_reset(UpdateShared* us) {
   us->dup = 0;
   us->pmin = STAMP_NONE;
   us->gathered = 0;
+}
+
+// The frequency update's own scalars, reset once before the first update
+// and at the end of each.
+__device__ __forceinline__ void freq_reset(FreqShared* fs) {
+  fs->femin = 0xFFFFFFFFu;
+  fs->fhot = 0xFFFFFFFFu;
 }
 
 // Looks up every block of a request in one worker's cache (CTA-wide);
@@ -851,6 +872,478 @@ __device__ __forceinline__ void cache_apply(const TableView& t, CacheMeta* meta,
     meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
     if (E > 0) meta->head = sc.vt[sc.victim[E - 1]] + 1;
     meta->T = T + (uint32_t)nb;
+  }
+}
+
+// ---------------------------------------------------------------- frequency eviction
+//
+// The KV Block Manager's rule (§2.2) in its two-class form: frequency 1 on
+// insertion, doubled on a hit (at most fmax), lowered by 1 per decay step and
+// never below 1; a block at frequency 1 is cold, at 2 or more hot (eligible
+// for promotion).  The victim is the least recently used cold block, else the
+// least recently used block.  A slot keeps the frequency lazily as e, the
+// decay step from which it is back at 1: at step D the frequency is
+// max(1, e - D + 1) and the block is cold iff e <= D.  Insertion sets e = D.
+// The log stays in recency order, so the victims are the first live cold
+// entries after the head; FreqMeta::fscan/fmin let a search skip a prefix of
+// hot entries it has already passed.
+
+// e after a hit at decay step D
+__device__ __forceinline__ uint32_t freq_hit(uint32_t e, uint32_t D, uint32_t fmax) {
+  const uint32_t f = e > D ? e - D + 1u : 1u;
+  const uint32_t f2 = 2u * f < fmax ? 2u * f : fmax;
+  return D + f2 - 1u;
+}
+
+// Where a victim search starts: fscan while the hot entries passed there
+// are still hot, else the head.
+__device__ __forceinline__ uint32_t freq_start(const CacheMeta* meta, const FreqMeta* fm,
+                                               uint32_t D) {
+  return D < fm->fmin ? fm->fscan : meta->head;
+}
+
+// The first `want` live cold log entries from *pos on (as gather_live; slot
+// with VSLOT_EMPTY_OK, position).  The live hot entries passed on the way
+// lower fs->femin (their least e) and fs->fhot (their first position); hot
+// entries of the last chunk past the last victim count too, which only makes
+// the next search start earlier.
+template <int NT>
+__device__ __forceinline__ void gather_cold(const TableView& t, const CacheMeta* meta, uint32_t* pos,
+                                            uint32_t want, uint32_t D, UpdateScratch& sc,
+                                            UpdateShared* us, FreqShared* fs, int* warp_tot) {
+  const uint32_t T = meta->T;
+  uint32_t have = us->gathered;
+  uint32_t p0 = *pos;
+  uint32_t he = 0xFFFFFFFFu, hp = 0xFFFFFFFFu;
+  while (have < want && p0 < T) {
+    const uint32_t p = p0 + threadIdx.x;
+    bool cold = false, empty_ok = false;
+    uint32_t x = 0;
+    if (p < T) {
+      x = t.log[p & t.rmask];
+      const bool look = threadIdx.x < 2 * (want - have) + 32;
+      uint64_t v[BUCKET];
+      if (look) ld_bucket(t.keys, x / BUCKET, v);
+      const bool live = __ldcg(t.stamp + x) == p;
+      const uint32_t e = __ldcg(t.fexp + x);
+      cold = live && e <= D;
+      if (live && e > D) {
+        he = min(he, e);
+        hp = min(hp, p);
+      }
+      if (look) {
+#pragma unroll
+        for (int q = 0; q < BUCKET; q++) empty_ok |= v[q] == KEY_EMPTY;
+      }
+    }
+    int tot;
+    const int r = cta_rank<NT>(cold, warp_tot, &tot);
+    if (cold && have + r < want) {
+      sc.vslot[have + r] = x | (empty_ok ? VSLOT_EMPTY_OK : 0u);
+      sc.vt[have + r] = p;
+    }
+    have = min(want, have + (uint32_t)tot);
+    p0 += NT;
+  }
+  he = __reduce_min_sync(FULL_MASK, he);
+  hp = __reduce_min_sync(FULL_MASK, hp);
+  if ((threadIdx.x & 31) == 0) {
+    if (he != 0xFFFFFFFFu) atomicMin(&fs->femin, he);
+    if (hp != 0xFFFFFFFFu) atomicMin(&fs->fhot, hp);
+  }
+  grp_bar<NT>();
+  if (threadIdx.x == 0) {
+    us->gathered = have;
+    *pos = p0;
+  }
+  grp_bar<NT>();
+}
+
+// The first `want` live hot entries from the head, packed (position << 32 |
+// slot) into global scratch `out`, in order; fs->gb = how many.
+template <int NT>
+__device__ __forceinline__ void gather_hot(const TableView& t, const CacheMeta* meta, uint32_t want,
+                                           uint32_t D, uint64_t* out, FreqShared* fs,
+                                           int* warp_tot) {
+  const uint32_t T = meta->T;
+  uint32_t have = 0;
+  for (uint32_t p0 = meta->head; have < want && p0 < T; p0 += NT) {
+    const uint32_t p = p0 + threadIdx.x;
+    bool hot = false;
+    uint32_t x = 0;
+    if (p < T) {
+      x = t.log[p & t.rmask];
+      hot = __ldcg(t.stamp + x) == p && __ldcg(t.fexp + x) > D;
+    }
+    int tot;
+    const int r = cta_rank<NT>(hot, warp_tot, &tot);
+    if (hot && have + r < want) out[have + r] = ((uint64_t)p << 32) | x;
+    have = min(want, have + (uint32_t)tot);
+  }
+  grp_bar<NT>();
+  if (threadIdx.x == 0) fs->gb = have;
+  grp_bar<NT>();
+}
+
+// As cache_prepare_captured, for frequency eviction: present blocks keep
+// their stamp in pst and their e in fslot (an absent block's fslot is its
+// insert position); us->pmin = the least stamp of a present cold block; the
+// first chunk of cold entries from the search start.  us must be reset.
+template <int NT>
+__device__ __forceinline__ void cache_prepare_captured_freq(const TableView& t, const CacheMeta* meta,
+                                                            const FreqMeta* fm,
+                                                            uint32_t K, const uint32_t* pslot,
+                                                            const uint32_t* pfree, int nb, int nabs,
+                                                            uint32_t D, UpdateScratch& sc,
+                                                            UpdateShared* us, FreqShared* fs,
+                                                            int* warp_tot, uint32_t* scan_pos) {
+  const uint32_t size = meta->size, T = meta->T;
+  const uint32_t start = freq_start(meta, fm, D);
+  const uint32_t free_slots = K - size;
+  const uint32_t E0 = (uint32_t)nabs > free_slots ? (uint32_t)nabs - free_slots : 0u;
+  const uint32_t p = start + threadIdx.x;
+  const bool gp = E0 > 0 && p < T;
+  uint32_t x = 0;
+  if (gp) x = t.log[p & t.rmask];
+  uint32_t pmin = STAMP_NONE;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const uint32_t sl = pslot[k];
+    sc.slot[k] = sl;
+    sc.evk[k] = 0;
+    uint32_t st = STAMP_NONE, f = pfree[k];
+    if (sl != SLOT_NONE) {
+      st = __ldcg(t.stamp + sl);
+      f = __ldcg(t.fexp + sl);
+      if (f <= D) pmin = min(pmin, st);
+    }
+    sc.pst[k] = st;
+    sc.fslot[k] = f;
+  }
+  bool cold = false, empty_ok = false;
+  uint32_t he = 0xFFFFFFFFu, hp = 0xFFFFFFFFu;
+  if (gp) {
+    const bool look = threadIdx.x < 2 * E0 + 32;
+    uint64_t v[BUCKET];
+    if (look) ld_bucket(t.keys, x / BUCKET, v);
+    const bool live = __ldcg(t.stamp + x) == p;
+    const uint32_t e = __ldcg(t.fexp + x);
+    cold = live && e <= D;
+    if (live && e > D) {
+      he = e;
+      hp = p;
+    }
+    if (look) {
+#pragma unroll
+      for (int q = 0; q < BUCKET; q++) empty_ok |= v[q] == KEY_EMPTY;
+    }
+  }
+  pmin = __reduce_min_sync(FULL_MASK, pmin);
+  he = __reduce_min_sync(FULL_MASK, he);
+  hp = __reduce_min_sync(FULL_MASK, hp);
+  if ((threadIdx.x & 31) == 0) {
+    if (pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+    if (he != 0xFFFFFFFFu) atomicMin(&fs->femin, he);
+    if (hp != 0xFFFFFFFFu) atomicMin(&fs->fhot, hp);
+  }
+  int tot;
+  const int r = cta_rank<NT>(cold, warp_tot, &tot);
+  if (cold && (uint32_t)r < E0) {
+    sc.vslot[r] = x | (empty_ok ? VSLOT_EMPTY_OK : 0u);
+    sc.vt[r] = p;
+  }
+  if (threadIdx.x == 0) {
+    us->n_absent = nabs;
+    us->gathered = min(E0, (uint32_t)tot);
+    fs->fstart = start;
+    *scan_pos = start + NT;
+  }
+  grp_bar<NT>();
+}
+
+// After cache_lookup_all: present blocks' e into fslot, us->pmin = the least
+// stamp of a present cold block, the search start.
+template <int NT>
+__device__ __forceinline__ void freq_present(const TableView& t, const CacheMeta* meta,
+                                             const FreqMeta* fm, int nb, uint32_t D,
+                                             UpdateScratch& sc, UpdateShared* us,
+                                             FreqShared* fs, uint32_t* scan_pos) {
+  if (threadIdx.x == 0) {
+    us->pmin = STAMP_NONE;
+    us->gathered = 0;
+    fs->fstart = freq_start(meta, fm, D);
+    *scan_pos = fs->fstart;
+  }
+  grp_bar<NT>();
+  uint32_t pmin = STAMP_NONE;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const uint32_t sl = sc.slot[k];
+    if (sl == SLOT_NONE) continue;
+    const uint32_t e = __ldcg(t.fexp + sl);
+    sc.fslot[k] = e;
+    if (e <= D) pmin = min(pmin, sc.pst[k]);
+  }
+  pmin = __reduce_min_sync(FULL_MASK, pmin);
+  if ((threadIdx.x & 31) == 0 && pmin != STAMP_NONE) atomicMin(&us->pmin, pmin);
+  grp_bar<NT>();
+}
+
+// Victim codes of the frequency update: >= 0 an index into vslot/vt; -1 a
+// block this request inserted and evicts again (nothing to clear); <= -2 the
+// slot -code - 2, cleared to a tombstone.
+constexpr int32_t VICTIM_OWN_INSERT = -1;
+
+// Binary search of stamp st among n packed (position << 32 | slot) entries
+// in increasing position order; the index or -1.
+__device__ __forceinline__ int32_t packed_find(const uint64_t* a, uint32_t n, uint32_t st) {
+  uint32_t lo = 0, hi = n;
+  while (lo < hi) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if ((uint32_t)(__ldcg(a + mid) >> 32) < st) lo = mid + 1; else hi = mid;
+  }
+  return lo < n && (uint32_t)(__ldcg(a + lo) >> 32) == st ? (int32_t)lo : -1;
+}
+
+// Applies one request's block list to the chosen worker's cache under
+// frequency eviction, with the semantics of touching blocks 0..nb-1 in order
+// (a hit doubles the frequency and makes the block most recent, a miss
+// inserts at frequency 1 after evicting the rule's victim when the cache is
+// full).  Fast path: the first E0 live cold entries are the victims when no
+// present cold block is older than the last of them.  Otherwise one thread
+// replays the sequence over the first 2 nb cold entries (shared scratch), the
+// first 2 nb hot ones (global scratch `gtmp`, only when the cold ones run
+// out) and the request's own blocks.  CTA-wide; updates meta.
+template <int NT>
+__device__ __forceinline__ void cache_apply_freq(const TableView& t, CacheMeta* meta, FreqMeta* fm,
+                                                 uint32_t K,
+                                                 const uint64_t* hbuf, int nb, uint32_t D,
+                                                 uint32_t fmax, UpdateScratch& sc,
+                                                 UpdateShared* us, FreqShared* fs, int* warp_tot,
+                                                 uint32_t* scan_pos, uint64_t* gtmp) {
+  const uint32_t size = meta->size;
+  const int nabs = us->n_absent;
+  const uint32_t free_slots = K - size;
+  const uint32_t E0 = (uint32_t)nabs > free_slots ? (uint32_t)nabs - free_slots : 0u;
+  if (E0 > 0 && us->gathered < E0) gather_cold<NT>(t, meta, scan_pos, E0, D, sc, us, fs, warp_tot);
+  const bool fast = E0 == 0 || (us->gathered >= E0 && us->pmin > sc.vt[E0 - 1]);
+  if (fast) {
+    for (int k = threadIdx.x; k < nb; k += NT) sc.kind[k] = sc.slot[k] == SLOT_NONE;
+    for (uint32_t v = threadIdx.x; v < E0; v += NT) sc.victim[v] = (int32_t)v;
+    if (threadIdx.x == 0) us->n_victims = (int)E0;
+    grp_bar<NT>();
+  } else {
+    // list A: the first 2 nb live cold entries from the search start
+    const uint32_t want = min(size, 2u * (uint32_t)nb);
+    grp_bar<NT>();
+    if (threadIdx.x == 0) {
+      us->gathered = 0;
+      *scan_pos = fs->fstart;
+    }
+    grp_bar<NT>();
+    gather_cold<NT>(t, meta, scan_pos, want, D, sc, us, fs, warp_tot);
+    const uint32_t G = us->gathered;
+    // list B, when the cold entries ran out: the first 2 nb live hot entries
+    if (G < want) {
+      gather_hot<NT>(t, meta, want, D, gtmp, fs, warp_tot);
+    } else if (threadIdx.x == 0) {
+      fs->gb = 0;
+    }
+    for (uint32_t q = threadIdx.x; q < G; q += NT) {
+      sc.owner[q] = -1;
+      sc.touched[q] = 0;
+    }
+    grp_bar<NT>();
+    const uint32_t last = G ? sc.vt[G - 1] : 0u;
+    for (int k = threadIdx.x; k < nb; k += NT) {
+      const uint32_t st = sc.pst[k];
+      if (st != STAMP_NONE && G && st <= last && sc.fslot[k] <= D) {
+        uint32_t lo = 0, hi = G;
+        while (lo < hi) {
+          const uint32_t mid = (lo + hi) >> 1;
+          if (sc.vt[mid] < st) lo = mid + 1; else hi = mid;
+        }
+        if (lo < G && sc.vt[lo] == st) sc.owner[lo] = k;
+      }
+    }
+    grp_bar<NT>();
+    if (threadIdx.x == 0) {
+      const uint32_t GB = fs->gb;
+      const bool hits_cold = fmax < 2u;   // a hit at cap 1 leaves the block cold
+      uint32_t pa = 0, pb = 0, sz = size;
+      int qc = 0, qh = 0, E = 0;
+      for (int k = 0; k < nb; k++) {
+        const bool present = sc.slot[k] != SLOT_NONE && !sc.evk[k];
+        if (present) {
+          sc.kind[k] = 0;
+          const uint32_t st = sc.pst[k];
+          if (sc.fslot[k] <= D) {   // a cold entry: in list A if old enough
+            if (G && st <= last) {
+              uint32_t lo = 0, hi = G;
+              while (lo < hi) {
+                const uint32_t mid = (lo + hi) >> 1;
+                if (sc.vt[mid] < st) lo = mid + 1; else hi = mid;
+              }
+              if (lo < G && sc.vt[lo] == st) sc.touched[lo] = 1;
+            }
+          } else if (GB) {          // a hot entry: in list B if old enough
+            const int32_t ib = packed_find(gtmp, GB, st);
+            if (ib >= 0) gtmp[ib] |= 0x80000000ull;   // touched
+          }
+          continue;
+        }
+        sc.kind[k] = 1;
+        if (sz < K) {
+          sz++;
+          continue;
+        }
+        // the victim: old cold, own cold, old hot, own hot -- each oldest first
+        while (pa < G && sc.touched[pa]) pa++;
+        if (pa < G) {
+          sc.victim[E++] = (int32_t)pa;
+          const int32_t ow = sc.owner[pa];
+          if (ow >= 0) {   // a block of this request, evicted before its turn
+            sc.evk[ow] = 1;
+            sc.fslot[ow] = SLOT_NONE;
+          }
+          pa++;
+          continue;
+        }
+        while (qc < k && !(sc.kind[qc] == 1 || (hits_cold && sc.kind[qc] == 0))) qc++;
+        if (qc < k) {
+          if (sc.kind[qc] == 1) {
+            sc.kind[qc] = 2;   // inserted and evicted again
+            sc.victim[E++] = VICTIM_OWN_INSERT;
+          } else {
+            sc.kind[qc] = 3;   // hit, then evicted
+            sc.victim[E++] = -(int32_t)sc.slot[qc] - 2;
+          }
+          qc++;
+          continue;
+        }
+        while (pb < GB && (__ldcg(gtmp + pb) & 0x80000000ull)) pb++;
+        if (pb < GB) {
+          const uint64_t ent = __ldcg(gtmp + pb);
+          const uint32_t x = (uint32_t)ent;
+          sc.victim[E++] = -(int32_t)x - 2;
+          // a present hot block evicted before its turn
+          for (int k2 = k + 1; k2 < nb; k2++)
+            if (sc.slot[k2] == x && !sc.evk[k2]) {
+              sc.evk[k2] = 1;
+              sc.fslot[k2] = SLOT_NONE;
+            }
+          pb++;
+          continue;
+        }
+        while (qh < k && sc.kind[qh] != 0) qh++;
+        if (qh < k) {
+          sc.kind[qh] = 3;
+          sc.victim[E++] = -(int32_t)sc.slot[qh] - 2;
+          qh++;
+          continue;
+        }
+        us->err = RS_ERR_TIMEOUT;   // nothing to evict: inconsistent state
+        break;
+      }
+      us->n_victims = E;
+      us->slow = 1;
+    }
+    grp_bar<NT>();
+  }
+  const int E = us->n_victims;
+  int ntomb = 0;
+  for (int v = threadIdx.x; v < E; v += NT) {
+    const int32_t iv = sc.victim[v];
+    if (iv == VICTIM_OWN_INSERT) continue;
+    uint32_t x;
+    bool tomb = true;
+    if (iv >= 0) {
+      const uint32_t xv = sc.vslot[iv];
+      x = xv & ~VSLOT_EMPTY_OK;
+      tomb = (xv & VSLOT_EMPTY_OK) == 0u;
+    } else {
+      x = (uint32_t)(-(iv + 2));
+    }
+    t.keys[x] = tomb ? KEY_TOMB : KEY_EMPTY;
+    t.stamp[x] = STAMP_NONE;
+    ntomb += tomb;
+  }
+  ntomb = __reduce_add_sync(FULL_MASK, (unsigned)ntomb);
+  if ((threadIdx.x & 31) == 0 && ntomb) atomicAdd(&us->n_tomb, ntomb);
+  const uint32_t T = meta->T;
+  int nins = 0, recl = 0, err = 0;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const int kd = sc.kind[k];
+    if (kd == 2) nins++;
+    if (kd != 1) continue;
+    const uint32_t fr = sc.fslot[k];
+    uint32_t sl = SLOT_NONE;
+    int32_t cl = -1;
+    if (fr != SLOT_NONE) {
+      const uint32_t x = fr & ~FREE_TOMB;
+      cl = slot_claim(sc, x);
+      if (cl >= 0) {
+        t.keys[x] = hbuf[k];
+        sl = x;
+        recl += (fr & FREE_TOMB) != 0;
+      }
+    }
+    sc.slot[k] = sl;
+    sc.pst[k] = (uint32_t)cl;
+    nins++;
+  }
+  grp_bar<NT>();
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const int kd = sc.kind[k];
+    const uint32_t pos = T + (uint32_t)k;
+    if (kd >= 2) {   // evicted within this request: its log position stays dead
+      t.log[pos & t.rmask] = 0u;
+      continue;
+    }
+    uint32_t sl = sc.slot[k];
+    uint32_t e = D;
+    if (kd == 1) {
+      const int32_t cl = (int32_t)sc.pst[k];
+      if (cl >= 0) sc.dupset[cl] = 0ull;
+      if (sl == SLOT_NONE) {
+        int wt = 0;
+        sl = table_insert(t, hbuf[k], &wt, &err);
+        recl += wt;
+        sc.slot[k] = sl;
+      }
+    } else {
+      e = freq_hit(sc.fslot[k], D, fmax);
+    }
+    if (sl != SLOT_NONE) {
+      t.stamp[sl] = pos;
+      t.fexp[sl] = e;
+      t.log[pos & t.rmask] = sl;
+    }
+  }
+  nins = __reduce_add_sync(FULL_MASK, (unsigned)nins);
+  recl = __reduce_add_sync(FULL_MASK, (unsigned)recl);
+  if ((threadIdx.x & 31) == 0) {
+    if (nins) atomicAdd(&us->n_ins, nins);
+    if (recl) atomicAdd(&us->reclaimed, recl);
+  }
+  if (err) us->err = RS_ERR_TIMEOUT;
+  grp_bar<NT>();
+  if (threadIdx.x == 0) {
+    meta->tombs = meta->tombs + (uint32_t)us->n_tomb - (uint32_t)us->reclaimed;
+    meta->size = meta->size + (uint32_t)us->n_ins - (uint32_t)E;
+    if (us->slow) {
+      fm->fscan = meta->head;   // the next search starts at the head
+      fm->fmin = 0;
+    } else if (E > 0) {
+      const uint32_t next = sc.vt[E - 1] + 1;
+      if (fs->fstart == meta->head) {
+        meta->head = min(fs->fhot, next);
+        fm->fmin = fs->femin;
+      } else {
+        fm->fmin = min(fm->fmin, fs->femin);
+      }
+      fm->fscan = next;
+    }
+    meta->T = T + (uint32_t)nb;
+    freq_reset(fs);
   }
 }
 

@@ -24,6 +24,14 @@ struct CacheMeta {
   uint32_t tombs;   // tombstoned slots
 };
 
+// Frequency eviction's search state of one worker: while the decay step is
+// below fmin, the log range [head, fscan) holds no live cold entry (fmin = 0:
+// search from the head).
+struct FreqMeta {
+  uint32_t fscan;
+  uint32_t fmin;
+};
+
 // Geometry of one worker's table: 8 * nbuckets slots (>= 4 K) and a log ring
 // of R entries (>= 4 K).
 struct TableGeom {
@@ -44,11 +52,13 @@ struct SimDesc {
   const uint64_t* hashes;   // block hashes of the replica's trace
   int64_t n_req;
   int64_t rec_base;         // first record row
-  int32_t C, policy, controller, reserved;
+  int32_t C, policy, controller, eviction;   // eviction: RS_EVICT_*
   float omega, tau;
   uint64_t seed;
   double c_t1, c_t2;        // load-spike schedule: C, then c_mid on [c_t1, c_t2),
   int32_t c_mid, c_end;     // then c_end (c_mid = 0: C throughout)
+  int32_t freq_max, reserved;   // frequency eviction: cap, and decay step length (s)
+  double decay_s;
 };
 
 struct ModelConsts {
@@ -61,7 +71,9 @@ struct SimBuffers {
   uint64_t* keys;           // [nsim][W][slots]
   uint32_t* stamp;          // [nsim][W][slots]
   uint32_t* log;            // [nsim][W][R]
-  uint64_t* tmp;            // [nsim][K] rebuild scratch
+  uint32_t* fexp;           // [nsim][W][slots] frequency eviction state, or NULL
+  uint64_t* tmp;            // [nsim][K] rebuild scratch (and the frequency slow path's list)
+  uint32_t* tmpe;           // [nsim][K] rebuild scratch of fexp, or NULL
   double* pend;             // [nsim][4][pend_cap]: 2 buffers x (first token, TTFT)
   int64_t pend_cap;
   CacheMeta* meta_out;      // [nsim][W]

@@ -37,7 +37,7 @@ struct SimLayout {
   size_t ftab, wwco, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
   size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
-  size_t wmeta, winserv, wqh, wqt, wm, wcost, wopen, wabs;
+  size_t wmeta, wfreq, winserv, wqh, wqt, wm, wcost, wopen, wabs;
   size_t kind, evk, touched;
   size_t total;
   size_t slot_bytes;   // per-replica global bytes of the slot arrays (0: in shared memory)
@@ -97,6 +97,7 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(vslot, 4 * nv, 4)
   TAKE(vt, 4 * nv, 4)
   TAKE(wmeta, sizeof(CacheMeta) * (size_t)W, 16)
+  TAKE(wfreq, sizeof(FreqMeta) * (size_t)W, 8)
   TAKE(winserv, 4 * (size_t)W, 4)
   TAKE(wqh, 4 * (size_t)W, 4)
   TAKE(wqt, 4 * (size_t)W, 4)
@@ -147,6 +148,7 @@ struct SimScalars {
   ReqState q[2];
   RawReq nraw;                 // the request after the next one to arrive, as read
   double prev_arrival, min_ft, tick_t, lastL, ewma, sum_ttft, sum_e2e, makespan, first_switch_t;
+  int64_t first_evict_i, first_live;   // first evicting update: request, resident blocks after it
   int64_t next_tick, np;
   int64_t near_ties, exact_ties, sampled, near_bd, hit_blocks, inserted, evicted, slow, rebuilds;
   int64_t ticks, switches, tir[3], n_routed, probe_blocks, hashed_blocks;
@@ -154,11 +156,13 @@ struct SimScalars {
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
   int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, nabs;
+  uint32_t dclock;             // decay step of the request being updated (frequency eviction)
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
   int hist[256];
   double red[NT_SIM / 32];
+  FreqShared fs;               // the frequency update's scalars
 };
 
 // Everything a device helper needs, resolved once per CTA.
@@ -173,6 +177,7 @@ struct SimCtx {
   uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
+  FreqMeta* wfreq;
   int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs, *dclaim;
   uint32_t *pslot, *pfree;
   int64_t* wA;
@@ -190,6 +195,7 @@ struct SimCtx {
     t.keys = b->keys + wi * L->g.slots;
     t.stamp = b->stamp + wi * L->g.slots;
     t.log = b->log + wi * L->g.R;
+    t.fexp = b->fexp ? b->fexp + wi * L->g.slots : nullptr;
     t.bmask = L->g.bmask;
     t.rmask = L->g.rmask;
     return t;
@@ -613,9 +619,12 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   grp_bar<NT>();
 }
 
-// Cache update of the chosen worker (update group, warps 0-6).
+// Cache update of the chosen worker (update group, warps 0-6) for request i.
+// FREQ: the launch holds replicas that evict by frequency (the LRU-only
+// kernel carries none of that code).
+template <bool FREQ>
 __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb,
-                                              bool full) {
+                                              bool full, int64_t i) {
   SimScalars& S = *c.S;
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
@@ -625,22 +634,46 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     if (threadIdx.x == 0) S.status = RS_ERR_COLLISION;
     return;
   }
+  uint64_t* gtmp = c.b->tmp + (size_t)c.sid * g.K;
   if (S.rebuild) {
-    cache_rebuild<NT_UPD>(tv, meta, g.K, c.b->tmp + (size_t)c.sid * g.K, S.warp_tot, &S.us);
+    cache_rebuild<NT_UPD>(tv, meta, g.K, gtmp, S.warp_tot, &S.us,
+                          FREQ && c.b->tmpe ? c.b->tmpe + (size_t)c.sid * g.K : nullptr,
+                          FREQ ? &c.wfreq[j] : nullptr);
     if (threadIdx.x == 0) S.rebuilds++;
   }
   const bool captured = full && !S.rebuild;
-  if (captured)
-    cache_prepare_captured<NT_UPD>(tv, meta, g.K, c.pslot + (size_t)j * nb,
-                                   c.pfree + (size_t)j * nb, nb, S.nabs, c.sc, &S.us,
-                                   S.warp_tot, &S.scan_pos);
-  else
-    cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
-  cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos, captured);
+  if (FREQ && c.d->eviction == RS_EVICT_FREQ) {
+    // the KV Block Manager's frequency rule
+    const uint32_t D = S.dclock;
+    FreqMeta* fm = &c.wfreq[j];
+    if (captured) {
+      cache_prepare_captured_freq<NT_UPD>(tv, meta, fm, g.K, c.pslot + (size_t)j * nb,
+                                          c.pfree + (size_t)j * nb, nb, S.nabs, D, c.sc, &S.us,
+                                          &S.fs, S.warp_tot, &S.scan_pos);
+    } else {
+      cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
+      freq_present<NT_UPD>(tv, meta, fm, nb, D, c.sc, &S.us, &S.fs, &S.scan_pos);
+    }
+    cache_apply_freq<NT_UPD>(tv, meta, fm, g.K, hbuf, nb, D, (uint32_t)c.d->freq_max, c.sc, &S.us,
+                             &S.fs, S.warp_tot, &S.scan_pos, gtmp);
+  } else {
+    if (captured)
+      cache_prepare_captured<NT_UPD>(tv, meta, g.K, c.pslot + (size_t)j * nb,
+                                     c.pfree + (size_t)j * nb, nb, S.nabs, c.sc, &S.us,
+                                     S.warp_tot, &S.scan_pos);
+    else
+      cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
+    cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos, captured);
+  }
   if (threadIdx.x == 0) {
     if (S.us.err) S.status = S.us.err;
     S.inserted += S.us.n_ins;
     S.evicted += S.us.n_victims;
+    if (S.us.n_victims > 0 && S.first_evict_i < 0) {
+      // the first update that evicted; resident blocks = inserted - evicted
+      S.first_evict_i = i;
+      S.first_live = S.inserted - S.evicted;
+    }
     S.slow += S.us.slow;
     update_reset(&S.us);   // for the next request
     S.us.err = 0;
@@ -736,7 +769,7 @@ __device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q,
 // every replica has an SM to itself.
 // SG: the per-request slot arrays are in global memory (a compile-time
 // choice, so that in the common case the compiler knows they are shared).
-template <int MINB, bool SG>
+template <int MINB, bool SG, bool FREQ>
 __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
   extern __shared__ __align__(16) unsigned char smem[];
@@ -775,6 +808,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.h_f = reinterpret_cast<int32_t*>(slotbase + lay.h_f);
   c.freestk = reinterpret_cast<int32_t*>(slotbase + lay.freestk);
   c.wmeta = reinterpret_cast<CacheMeta*>(smem + lay.wmeta);
+  c.wfreq = reinterpret_cast<FreqMeta*>(smem + lay.wfreq);
   c.winserv = reinterpret_cast<int32_t*>(smem + lay.winserv);
   c.wqh = reinterpret_cast<int32_t*>(smem + lay.wqh);
   c.wqt = reinterpret_cast<int32_t*>(smem + lay.wqt);
@@ -820,7 +854,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     const int cslots = max(d.C, max(d.c_mid, d.c_end));
     for (int p = threadIdx.x; p < cslots; p += NT_SIM) c.freestk[p] = cslots - 1 - p;
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
-      c.wmeta[j] = CacheMeta{0u, 0u, 0u, 0u};
+      c.wmeta[j] = CacheMeta{};
+      c.wfreq[j] = FreqMeta{0u, 0u};
       c.winserv[j] = 0;
       c.wA[j] = 0;
       c.wqh[j] = -1;
@@ -833,6 +868,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       S.tick_t = mc.dt;
       S.nfree = max(d.C, max(d.c_mid, d.c_end));
       S.first_switch_t = -1.0;
+      S.first_evict_i = -1;
+      freq_reset(&S.fs);
     }
     __syncthreads();
   }
@@ -907,6 +944,10 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
                                                   TAG_SIM);
         S.jstar = js;
         S.hit_blocks += c.wm[js];
+        if (FREQ && d.eviction == RS_EVICT_FREQ) {   // decay step of this request's arrival
+          const double q = floor(__ddiv_rn(S.q[p].a, d.decay_s));
+          S.dclock = q < 2147483648.0 ? (uint32_t)q : 2147483648u;
+        }
         // the chosen worker's absent blocks, latched before the control warp
         // resets the probe state for the next request
         S.nabs = c.wabs[js];
@@ -967,7 +1008,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     const int js = S.jstar;
     if (warp < NT_SIM / 32 - 1) {
       // ---- the chosen worker's LRU cache (warps 0-6)
-      update_chosen(c, hb, js, nb, full);
+      update_chosen<FREQ>(c, hb, js, nb, full, i);
     } else {
       // ---- control warp: request i's load and latency; request i+1's
       // scalars, probe state and block hashes
@@ -1073,6 +1114,15 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     r.slow_path = S.slow;
     r.rebuilds = S.rebuilds;
     r.first_switch_t = S.first_switch_t;
+    // KV-cache pressure: resident blocks over W K (resident = inserted - evicted)
+    const double cap = __dmul_rn((double)W, (double)L.g.K);
+    r.first_evict_t = -1.0;
+    r.rho_first_evict = -1.0;
+    if (S.first_evict_i >= 0) {
+      r.first_evict_t = b.rec.arrival[d.rec_base + S.first_evict_i];
+      r.rho_first_evict = __ddiv_rn((double)S.first_live, cap);
+    }
+    r.rho_end = __ddiv_rn((double)(S.inserted - S.evicted), cap);
     b.res[sid] = r;
   }
   for (int j = threadIdx.x; j < W; j += NT_SIM) b.meta_out[(size_t)sid * W + j] = c.wmeta[j];
@@ -1161,9 +1211,14 @@ cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaun
   if (e != cudaSuccess) return e;
   // one replica per SM: the kernel may use every register
   const bool one = L.nsim <= sms;
-  void (*kern)(const SimDesc*, SimBuffers, SimLaunch) =
-      one ? (L.slots_global ? k_sim<1, true> : k_sim<1, false>)
-          : (L.slots_global ? k_sim<2, true> : k_sim<2, false>);
+  // frequency eviction state present: the kernel with the frequency rule
+  void (*kern)(const SimDesc*, SimBuffers, SimLaunch);
+  if (b.fexp)
+    kern = one ? (L.slots_global ? k_sim<1, true, true> : k_sim<1, false, true>)
+               : (L.slots_global ? k_sim<2, true, true> : k_sim<2, false, true>);
+  else
+    kern = one ? (L.slots_global ? k_sim<1, true, false> : k_sim<1, false, false>)
+               : (L.slots_global ? k_sim<2, true, false> : k_sim<2, false, false>);
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   kern<<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);

@@ -22,6 +22,7 @@ RS_ERR_CUDA, RS_ERR_TIMEOUT, RS_ERR_STATE, RS_ERR_COLLISION = -4, -5, -6, -7
 RS_POLICY_DYNAMO, RS_POLICY_LOADBAL = 0, 1
 RS_POLICY_ROUNDROBIN, RS_POLICY_RANDOM, RS_POLICY_P2C = 2, 3, 4
 RS_MEM_DEVICE, RS_MEM_HOST = 0, 1
+RS_EVICT_LRU, RS_EVICT_FREQ = 0, 1
 RS_SIM_NO_POA = 1
 
 
@@ -45,7 +46,8 @@ class rs_replica_params(C.Structure):
     _fields_ = [("trace", C.c_int32), ("C", C.c_int32), ("policy", C.c_int32),
                 ("controller", C.c_int32), ("omega", C.c_float), ("tau", C.c_float),
                 ("seed", C.c_uint64), ("n_req", C.c_int64), ("c_t1", C.c_double),
-                ("c_t2", C.c_double), ("c_mid", C.c_int32), ("c_end", C.c_int32)]
+                ("c_t2", C.c_double), ("c_mid", C.c_int32), ("c_end", C.c_int32),
+                ("eviction", C.c_int32), ("freq_max", C.c_int32), ("decay_s", C.c_double)]
 
 
 class rs_replica_result(C.Structure):
@@ -60,7 +62,9 @@ class rs_replica_result(C.Structure):
                 ("final_ewma", C.c_double), ("probes", C.c_int64),
                 ("probe_blocks", C.c_int64), ("hashed_blocks", C.c_int64),
                 ("slow_path", C.c_int64), ("rebuilds", C.c_int64),
-                ("first_switch_t", C.c_double), ("poa_static", C.c_double)]
+                ("first_switch_t", C.c_double), ("poa_static", C.c_double),
+                ("first_evict_t", C.c_double), ("rho_first_evict", C.c_double),
+                ("rho_end", C.c_double)]
 
     def as_dict(self) -> dict:
         return {f: (list(getattr(self, f)) if f == "ticks_in_regime" else getattr(self, f))
@@ -303,7 +307,9 @@ def host_trace(trace, pinned: bool = True) -> TraceBuffers:
 def replica_params(r) -> rs_replica_params:
     return rs_replica_params(r.trace, r.C, r.policy, r.controller, r.omega, r.tau, r.seed, r.n_req,
                              float(getattr(r, "c_t1", 0.0)), float(getattr(r, "c_t2", 0.0)),
-                             int(getattr(r, "c_mid", 0)), int(getattr(r, "c_end", 0)))
+                             int(getattr(r, "c_mid", 0)), int(getattr(r, "c_end", 0)),
+                             int(getattr(r, "eviction", RS_EVICT_LRU)),
+                             int(getattr(r, "freq_max", 64)), float(getattr(r, "decay_s", 1.0)))
 
 
 def device_records(rows: int, W: int, device="cuda", with_cost: bool = False):

@@ -136,6 +136,11 @@ class Replica:
     c_t2: float = 0.0
     c_mid: int = 0
     c_end: int = 0
+    # cache eviction: 0 exact LRU, 1 the KV Block Manager's frequency rule
+    # with its frequency cap and decay step (s)
+    eviction: int = 0
+    freq_max: int = 64
+    decay_s: float = 1.0
 
 
 @dataclass

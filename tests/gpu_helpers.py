@@ -50,7 +50,8 @@ def oracle_run(cfg, trace, r, want_cache=False, max_ticks=0):
     sched = (r.c_t1, r.c_t2, r.c_mid, r.c_end) if getattr(r, "c_mid", 0) > 0 else None
     return O.simulate(cfg, trace, r.C, policy=r.policy, controller=r.controller, omega=r.omega,
                       tau=r.tau, seed=r.seed, n_req=r.n_req, want_cache=want_cache,
-                      max_ticks=max_ticks, schedule=sched)
+                      max_ticks=max_ticks, schedule=sched, eviction=getattr(r, "eviction", 0),
+                      freq_max=getattr(r, "freq_max", 64), decay_s=getattr(r, "decay_s", 1.0))
 
 
 def assert_replica_equal(g, o, W, times_rtol=1e-12, check_cost=True):
@@ -66,6 +67,8 @@ def assert_replica_equal(g, o, W, times_rtol=1e-12, check_cost=True):
         assert np.allclose(g[f], o[f], rtol=times_rtol, atol=0), f
     gr, orr = g["result"], o["summary"]
     assert gr["first_switch_t"] == orr["first_switch_t"], (gr["first_switch_t"], orr["first_switch_t"])
+    for f in ("first_evict_t", "rho_first_evict", "rho_end"):
+        assert gr[f] == orr[f], (f, gr[f], orr[f])
     for f in ("n_routed", "near_ties", "exact_ties", "sampled", "near_boundary", "hit_blocks",
               "inserted_blocks", "evicted_blocks", "ticks", "regime_switches", "final_regime",
               "max_regime"):
