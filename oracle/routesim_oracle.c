@@ -289,10 +289,11 @@ static int64_t freq_victim(const lru_t* c) {
 /* insert an absent key as most recent (frequency 1); when the cache is full
  * the LRU entry (mode LRU) or the frequency rule's victim (mode FREQ) goes
  * first.  Returns 1 if an entry was evicted. */
-static int lru_insert(lru_t* c, uint64_t key, int32_t mode) {
+static int lru_insert(lru_t* c, uint64_t key, int32_t mode, uint64_t* victim_key) {
   int evicted = 0;
   if (c->size == c->K) {
     int64_t v = mode == ORC_EVICT_FREQ ? freq_victim(c) : c->head;
+    if (victim_key) *victim_key = c->key[v];
     list_unlink(c, v);
     int64_t* link = &c->bucket[c->key[v] & c->mask];
     while (*link != v) link = &c->chain[*link];
@@ -309,6 +310,16 @@ static int lru_insert(lru_t* c, uint64_t key, int32_t mode) {
   list_push_recent(c, n);
   c->size++;
   return evicted;
+}
+
+/* removes node n (a present key) */
+static void lru_remove(lru_t* c, int64_t n) {
+  list_unlink(c, n);
+  int64_t* link = &c->bucket[c->key[n] & c->mask];
+  while (*link != n) link = &c->chain[*link];
+  *link = c->chain[n];
+  c->freel[c->nfree++] = n;
+  c->size--;
 }
 
 /* keys from least to most recent */
@@ -348,10 +359,60 @@ static void cache_update(lru_t* c, const uint64_t* h, int64_t nb, int64_t* inser
       lru_touch(c, n);
       if (mode == ORC_EVICT_FREQ) c->freq[n] = 2 * c->freq[n] < freq_max ? 2 * c->freq[n] : freq_max;
     } else {
-      *evicted += lru_insert(c, h[k], mode);
+      *evicted += lru_insert(c, h[k], mode, NULL);
       *inserted += 1;
     }
   }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Game 2 tiers (§4.2): exclusive G1, G2, G3 caches per worker               */
+/* ------------------------------------------------------------------------ */
+
+/* key enters tier t (0 = G1) as most recent; a full tier passes its least
+ * recent block down to the next tier, the last tier drops it.  Counts the
+ * blocks that left G1 and the blocks dropped. */
+static void tier_push(lru_t* const* tier, int32_t ntier, int32_t t, uint64_t key,
+                      int64_t* left_g1, int64_t* dropped) {
+  uint64_t k = key;
+  for (; t < ntier; t++) {
+    uint64_t v;
+    if (!lru_insert(tier[t], k, ORC_EVICT_LRU, &v)) return;
+    if (t == 0) (*left_g1)++;
+    k = v;
+  }
+  (*dropped)++;
+}
+
+/* the chosen worker accesses the prompt's blocks in order: a block in G1 is
+ * touched; a block in a lower tier moves to G1; an absent block is inserted
+ * into G1 */
+static void tier_update(lru_t* const* tier, int32_t ntier, const uint64_t* h, int64_t nb,
+                        int64_t* inserted, int64_t* left_g1, int64_t* dropped) {
+  for (int64_t k = 0; k < nb; k++) {
+    int64_t n = lru_find(tier[0], h[k]);
+    if (n >= 0) {
+      lru_touch(tier[0], n);
+      continue;
+    }
+    int found = 0;
+    for (int32_t t = 1; t < ntier && !found; t++) {
+      n = lru_find(tier[t], h[k]);
+      if (n >= 0) {
+        lru_remove(tier[t], n);
+        found = 1;
+      }
+    }
+    if (!found) *inserted += 1;
+    tier_push(tier, ntier, 0, h[k], left_g1, dropped);
+  }
+}
+
+/* tier (1, 2, 3) of key on a worker, 0 if absent; tid maps list index to tier */
+static int32_t tier_of(lru_t* const* tier, const int32_t* tid, int32_t ntier, uint64_t key) {
+  for (int32_t t = 0; t < ntier; t++)
+    if (lru_find(tier[t], key) >= 0) return tid[t];
+  return 0;
 }
 
 /* ------------------------------------------------------------------------ */
@@ -438,6 +499,8 @@ typedef struct {
   uint16_t *n_frozen, *prefix; float* cost;
   /* per worker */
   lru_t* cache; int64_t *inservice, *A, *qhead, *qtail;
+  lru_t *g2, *g3;      /* Game 2 tiers below G1 (tiered), else NULL */
+  double* kv_cost;     /* per request, or NULL */
   /* events */
   cev* heap; int64_t nheap; int64_t in_flight;
   /* controller */
@@ -660,6 +723,79 @@ static double next_step_time(const orc_replica* r, double t) {
   return INFINITY;
 }
 
+/* worker j's tiers from G1 down */
+static void worker_tiers(sim_t* s, int32_t j, int32_t ntier, const int32_t* tid, lru_t** out) {
+  for (int32_t t = 0; t < ntier; t++)
+    out[t] = tid[t] == 1 ? &s->cache[j] : tid[t] == 2 ? &s->g2[j] : &s->g3[j];
+}
+
+/* blocks resident on all workers, every tier */
+static int64_t resident(const sim_t* s) {
+  int64_t live = 0;
+  for (int32_t j = 0; j < s->W; j++) {
+    live += s->cache[j].size;
+    if (s->g2) live += s->g2[j].size + s->g3[j].size;
+  }
+  return live;
+}
+
+/* Eq. kv-cost (§4.2) of request i's blocks on worker sigma, as the caches
+ * stand when it is routed: per block alpha_t for sigma's own tier t; else
+ * the cheapest d(sigma, j) + alpha_t over copies on other workers (ties:
+ * same node before other node, then G1 before G2 before G3); else gamma.
+ * The request's cost sums the categories in a fixed order. */
+static void kv_charge(sim_t* s, int32_t sigma, const uint64_t* h, int64_t nb, int32_t ntier,
+                      const int32_t* tid, int64_t i) {
+  const orc_config* cfg = s->cfg;
+  const int32_t W = s->W;
+  int64_t cnt[10] = {0};   /* own G1..G3, near G1..G3, far G1..G3, recompute */
+  lru_t* own[3];
+  worker_tiers(s, sigma, ntier, tid, own);
+  for (int64_t k = 0; k < nb; k++) {
+    const int32_t t = tier_of(own, tid, ntier, h[k]);
+    if (t > 0) {
+      cnt[t - 1]++;
+      continue;
+    }
+    int has[2][3] = {{0, 0, 0}, {0, 0, 0}};
+    for (int32_t j = 0; j < W; j++) {
+      if (j == sigma) continue;
+      lru_t* tl[3];
+      worker_tiers(s, j, ntier, tid, tl);
+      const int32_t tj = tier_of(tl, tid, ntier, h[k]);
+      if (tj > 0) has[j / cfg->tier_node == sigma / cfg->tier_node ? 0 : 1][tj - 1] = 1;
+    }
+    int cat = 9;
+    double best = INFINITY;
+    for (int r = 0; r < 2; r++)
+      for (int q = 0; q < 3; q++) {
+        if (!has[r][q]) continue;
+        const double v = (r == 0 ? cfg->tier_d_near : cfg->tier_d_far) + cfg->tier_alpha[q];
+        if (v < best) {
+          best = v;
+          cat = 3 + 3 * r + q;
+        }
+      }
+    cnt[cat]++;
+  }
+  const double* al = cfg->tier_alpha;
+  const double dn = cfg->tier_d_near, df = cfg->tier_d_far;
+  double c = al[0] * (double)cnt[0];
+  c = c + al[1] * (double)cnt[1];
+  c = c + al[2] * (double)cnt[2];
+  for (int q = 0; q < 3; q++) c = c + (dn + al[q]) * (double)cnt[3 + q];
+  for (int q = 0; q < 3; q++) c = c + (df + al[q]) * (double)cnt[6 + q];
+  c = c + cfg->tier_gamma * (double)cnt[9];
+  orc_summary* sum = s->sum;
+  sum->kv_g1 += cnt[0];
+  sum->kv_g2 += cnt[1];
+  sum->kv_g3 += cnt[2];
+  sum->kv_remote += cnt[3] + cnt[4] + cnt[5] + cnt[6] + cnt[7] + cnt[8];
+  sum->kv_recompute += cnt[9];
+  sum->kv_cost = sum->kv_cost + c;
+  if (s->kv_cost) s->kv_cost[i] = c;
+}
+
 int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t* offsets,
                      const double* release, const int32_t* out_len, const orc_replica* rep,
                      orc_records* rec, orc_summary* sum, uint64_t* cache_keys,
@@ -678,7 +814,14 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
       rep->c_mid < 0 || rep->eviction < ORC_EVICT_LRU || rep->eviction > ORC_EVICT_FREQ ||
       (rep->eviction == ORC_EVICT_FREQ &&
        (rep->freq_max < 1 || rep->freq_max > (1 << 20) || !(rep->decay_s > 0.0) ||
-        !(rep->decay_s < INFINITY)))) {
+        !(rep->decay_s < INFINITY))) ||
+      (cfg->tiered &&
+       (rep->eviction != ORC_EVICT_LRU || cfg->tier_k2 < 0 || cfg->tier_k3 < 0 ||
+        cfg->tier_node < 1 || !(cfg->tier_alpha[0] < cfg->tier_alpha[1]) ||
+        !(cfg->tier_alpha[1] < cfg->tier_alpha[2]) || !(cfg->tier_alpha[2] < cfg->tier_gamma) ||
+        !(cfg->tier_gamma < INFINITY) || !(cfg->tier_alpha[0] >= 0.0) ||
+        !(cfg->tier_d_near >= 0.0) || !(cfg->tier_d_far >= 0.0) ||
+        !(cfg->tier_d_near < INFINITY) || !(cfg->tier_d_far < INFINITY)))) {
     sum->status = ORC_ERR_INVALID;
     return ORC_ERR_INVALID;
   }
@@ -705,6 +848,11 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   s.window = (double*)malloc(sizeof(double) * nn);
   s.heap = (cev*)malloc(sizeof(cev) * nn);
   s.cache = (lru_t*)calloc(W, sizeof(lru_t));
+  if (cfg->tiered) {
+    s.g2 = (lru_t*)calloc(W, sizeof(lru_t));
+    s.g3 = (lru_t*)calloc(W, sizeof(lru_t));
+  }
+  s.kv_cost = rec ? rec->kv_cost : NULL;
   s.inservice = (int64_t*)calloc(W, sizeof(int64_t));
   s.A = (int64_t*)calloc(W, sizeof(int64_t));
   s.qhead = (int64_t*)malloc(sizeof(int64_t) * W);
@@ -725,9 +873,21 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
     status = ORC_ERR_OOM;
     goto done;
   }
+  if (cfg->tiered && (!s.g2 || !s.g3)) { status = ORC_ERR_OOM; goto done; }
   for (int32_t j = 0; j < W; j++) {
     if (lru_init(&s.cache[j], cfg->K)) { status = ORC_ERR_OOM; goto done; }
+    if (cfg->tiered && ((cfg->tier_k2 > 0 && lru_init(&s.g2[j], cfg->tier_k2)) ||
+                        (cfg->tier_k3 > 0 && lru_init(&s.g3[j], cfg->tier_k3)))) {
+      status = ORC_ERR_OOM;
+      goto done;
+    }
     s.qhead[j] = s.qtail[j] = -1;
+  }
+  /* the tiers of every worker as a list from G1 down, with their tier numbers */
+  int32_t ntier = 1, tid[3] = {1, 2, 3};
+  if (cfg->tiered) {
+    if (cfg->tier_k2 > 0) tid[ntier++] = 2;
+    if (cfg->tier_k3 > 0) tid[ntier++] = 3;
   }
   s.next_tick = 1;
   const int32_t B = cfg->block;
@@ -844,14 +1004,21 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
         dclock = D;
       }
     }
-    const int64_t ev0 = sum->evicted_blocks;
-    cache_update(&s.cache[jstar], h, nb, &sum->inserted_blocks, &sum->evicted_blocks,
-                 rep->eviction, rep->freq_max);
-    if (ev0 == 0 && sum->evicted_blocks > 0) {
-      int64_t live = 0;
-      for (int32_t j = 0; j < W; j++) live += s.cache[j].size;
+    if (cfg->tiered) kv_charge(&s, jstar, h, nb, ntier, tid, i);
+    int64_t out_g1 = 0;   /* blocks that left the chosen worker's G1 */
+    if (cfg->tiered) {
+      lru_t* tl[3];
+      worker_tiers(&s, jstar, ntier, tid, tl);
+      tier_update(tl, ntier, h, nb, &sum->inserted_blocks, &out_g1, &sum->evicted_blocks);
+    } else {
+      const int64_t ev0 = sum->evicted_blocks;
+      cache_update(&s.cache[jstar], h, nb, &sum->inserted_blocks, &sum->evicted_blocks,
+                   rep->eviction, rep->freq_max);
+      out_g1 = sum->evicted_blocks - ev0;
+    }
+    if (out_g1 > 0 && sum->first_evict_t < 0.0) {
       sum->first_evict_t = a;
-      sum->rho_first_evict = (double)live / ((double)W * (double)cfg->K);
+      sum->rho_first_evict = (double)resident(&s) / ((double)W * (double)cfg->K);
     }
     sum->hit_blocks += m[jstar];
     s.A[jstar] += s.blk[i];
@@ -877,16 +1044,20 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
   }
   sum->final_regime = s.ctl.regime;
   sum->final_ewma = s.ctl.have_ewma ? s.ctl.ewma : -1.0;
-  {
-    int64_t live = 0;
-    for (int32_t j = 0; j < W; j++) live += s.cache[j].size;
-    sum->rho_end = (double)live / ((double)W * (double)cfg->K);
-  }
+  sum->rho_end = (double)resident(&s) / ((double)W * (double)cfg->K);
   sum->regime_switches = s.ctl.switches;
   if (cache_sizes || cache_keys) {
+    /* least to most recent; tiered: G3, then G2, then G1 (one recency stack
+     * of K + tier_k2 + tier_k3 blocks per worker) */
+    const int64_t per = cfg->tiered ? cfg->K + cfg->tier_k2 + cfg->tier_k3 : cfg->K;
     for (int32_t j = 0; j < W; j++) {
-      int64_t sz = cache_keys ? lru_dump(&s.cache[j], cache_keys + (int64_t)j * cfg->K)
-                              : s.cache[j].size;
+      int64_t sz = 0;
+      uint64_t* out = cache_keys ? cache_keys + (int64_t)j * per : NULL;
+      if (cfg->tiered) {
+        if (cfg->tier_k3 > 0) sz += out ? lru_dump(&s.g3[j], out + sz) : s.g3[j].size;
+        if (cfg->tier_k2 > 0) sz += out ? lru_dump(&s.g2[j], out + sz) : s.g2[j].size;
+      }
+      sz += out ? lru_dump(&s.cache[j], out + sz) : s.cache[j].size;
       if (cache_sizes) cache_sizes[j] = sz;
     }
   }
@@ -894,6 +1065,12 @@ done:
   sum->status = status;
   if (s.cache)
     for (int32_t j = 0; j < W; j++) lru_free(&s.cache[j]);
+  if (s.g2)
+    for (int32_t j = 0; j < W; j++) lru_free(&s.g2[j]);
+  if (s.g3)
+    for (int32_t j = 0; j < W; j++) lru_free(&s.g3[j]);
+  free(s.g2);
+  free(s.g3);
   if (!(rec && rec->worker)) free(s.worker);
   if (!(rec && rec->arrival)) free(s.arrival);
   if (!(rec && rec->start)) free(s.start);

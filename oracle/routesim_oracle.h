@@ -67,6 +67,18 @@ typedef struct {
   float regime_tau[3];    /* Table 2; entry 0 replaced by the replica's own */
   float regime_omega[3];
   double poa_window;      /* window length of Eq. (12), s */
+  /* Game 2 (§4.2, Eq. kv-cost): tiered = 1 gives every worker the exclusive
+   * tiers G1 (K blocks), G2 (tier_k2) and G3 (tier_k3); an access brings a
+   * block to G1, and each full tier hands its least recently used block to
+   * the next (the last drops it).  Routing sees G1.  Each routed request is
+   * charged, per full block on its worker i, alpha_t for its own tier t,
+   * else d(i, j) + alpha_t for the cheapest copy on another worker j, else
+   * gamma; d = tier_d_near within a node of tier_node workers, else
+   * tier_d_far. */
+  int32_t tiered, tier_node;
+  int64_t tier_k2, tier_k3;
+  double tier_alpha[3];
+  double tier_gamma, tier_d_near, tier_d_far;
 } orc_config;
 
 typedef struct {
@@ -98,10 +110,14 @@ typedef struct {
   double final_ewma;
   double first_switch_t;   /* first regime switch, -1 if none */
   /* KV-cache pressure (the regime-transition proposition of §5.3): arrival
-   * time of the first request whose update evicted, and rho = resident
-   * blocks over W K after that update (-1, -1 if nothing was evicted);
-   * rho after the last request */
+   * time of the first request whose update pushed a block out of a G1
+   * cache, and rho = resident blocks (all tiers) over W K after that update
+   * (-1, -1 if none); rho after the last request */
   double first_evict_t, rho_first_evict, rho_end;
+  /* Game 2 accounting (tiered): blocks found in the own G1 / G2 / G3, on
+   * another worker, nowhere; and the summed cost of Eq. kv-cost */
+  int64_t kv_g1, kv_g2, kv_g3, kv_remote, kv_recompute;
+  double kv_cost;
 } orc_summary;
 
 /* Per-request outputs; every pointer may be NULL.  Arrays of n (or n*W). */
@@ -116,6 +132,7 @@ typedef struct {
   uint16_t* n_frozen;     /* [n*W] min(in-service_j(a_i) + 1, cap - 1) */
   uint16_t* prefix;       /* [n*W] m_ij: cached-prefix blocks on worker j */
   float* cost;            /* [n*W] router cost c_j used for the decision */
+  double* kv_cost;        /* Eq. kv-cost of the request's blocks on its worker (tiered) */
 } orc_records;
 
 /* Block hashes of every full block.  Request i's hashes are written to

@@ -43,7 +43,10 @@ class _Config(C.Structure):
                 ("itl", C.c_double), ("dt", C.c_double), ("alpha", C.c_double),
                 ("theta1", C.c_double), ("theta2", C.c_double), ("eps_frac", C.c_double),
                 ("hyst_k", C.c_int32), ("regime_tau", C.c_float * 3),
-                ("regime_omega", C.c_float * 3), ("poa_window", C.c_double)]
+                ("regime_omega", C.c_float * 3), ("poa_window", C.c_double),
+                ("tiered", C.c_int32), ("tier_node", C.c_int32), ("tier_k2", C.c_int64),
+                ("tier_k3", C.c_int64), ("tier_alpha", C.c_double * 3), ("tier_gamma", C.c_double),
+                ("tier_d_near", C.c_double), ("tier_d_far", C.c_double)]
 
 
 class _Replica(C.Structure):
@@ -64,14 +67,16 @@ class _Summary(C.Structure):
                 ("max_regime", C.c_int32), ("ticks_in_regime", C.c_int64 * 3),
                 ("final_ewma", C.c_double), ("first_switch_t", C.c_double),
                 ("first_evict_t", C.c_double), ("rho_first_evict", C.c_double),
-                ("rho_end", C.c_double)]
+                ("rho_end", C.c_double), ("kv_g1", C.c_int64), ("kv_g2", C.c_int64),
+                ("kv_g3", C.c_int64), ("kv_remote", C.c_int64), ("kv_recompute", C.c_int64),
+                ("kv_cost", C.c_double)]
 
 
 class _Records(C.Structure):
     _fields_ = [("worker", C.c_void_p), ("arrival", C.c_void_p), ("start", C.c_void_p),
                 ("first_token", C.c_void_p), ("completion", C.c_void_p), ("ttft", C.c_void_p),
                 ("nbt", C.c_void_p), ("n_frozen", C.c_void_p), ("prefix", C.c_void_p),
-                ("cost", C.c_void_p)]
+                ("cost", C.c_void_p), ("kv_cost", C.c_void_p)]
 
 
 @dataclass
@@ -97,13 +102,29 @@ class OracleConfig:
     regime_tau: tuple = (0.0, 0.7, 0.8)
     regime_omega: tuple = (1.0, 1.0, 0.1)
     poa_window: float = 5.0
+    # Game 2 tiers (§4.2, Eq. kv-cost); the paper gives no values
+    tiered: int = 0
+    tier_node: int = 1
+    tier_k2: int = 0
+    tier_k3: int = 0
+    tier_alpha: tuple = (1.0, 4.0, 20.0)
+    tier_gamma: float = 100.0
+    tier_d_near: float = 2.0
+    tier_d_far: float = 10.0
+
+    @property
+    def K_stack(self) -> int:
+        """Blocks a worker holds across its tiers."""
+        return self.K + (self.tier_k2 + self.tier_k3 if self.tiered else 0)
 
     def c(self) -> _Config:
         return _Config(self.W, self.block, self.K, self.hash_seed, self.lat_a, self.lat_b,
                        self.lat_d, self.cap, self.w_c, self.itl, self.dt, self.alpha,
                        self.theta1, self.theta2, self.eps_frac, self.hyst_k,
                        (C.c_float * 3)(*self.regime_tau), (C.c_float * 3)(*self.regime_omega),
-                       self.poa_window)
+                       self.poa_window, self.tiered, self.tier_node, self.tier_k2, self.tier_k3,
+                       (C.c_double * 3)(*self.tier_alpha), self.tier_gamma, self.tier_d_near,
+                       self.tier_d_far)
 
 
 _lib = None
@@ -205,15 +226,16 @@ def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
         "first_token": np.zeros(nn), "completion": np.zeros(nn), "ttft": np.zeros(nn),
         "nbt": np.zeros(nn, np.int32), "n_frozen": np.zeros(nn * W, np.uint16),
         "prefix": np.zeros(nn * W, np.uint16), "cost": np.zeros(nn * W, np.float32),
+        "kv_cost": np.zeros(nn),
     }
     rec = _Records(*[_p(r[k]).value for k in ("worker", "arrival", "start", "first_token",
                                                 "completion", "ttft", "nbt", "n_frozen",
-                                                "prefix", "cost")])
+                                                "prefix", "cost", "kv_cost")])
     st = schedule if schedule is not None else (0.0, 0.0, 0, 0)
     rep = _Replica(C_, policy, controller, omega, tau, seed, n, float(st[0]), float(st[1]),
                    int(st[2]), int(st[3]), int(eviction), int(freq_max), float(decay_s))
     s = _Summary()
-    keys = np.zeros(W * cfg.K, np.uint64) if want_cache else None
+    keys = np.zeros(W * cfg.K_stack, np.uint64) if want_cache else None
     sizes = np.zeros(W, np.int64) if want_cache else None
     te = np.zeros(max(max_ticks, 1)) if max_ticks else None
     tr = np.zeros(max(max_ticks, 1), np.int32) if max_ticks else None
@@ -228,7 +250,8 @@ def simulate(cfg: OracleConfig, trace, C_: int, policy: int = POLICY_DYNAMO,
     out["summary"] = {f: (list(getattr(s, f)) if f == "ticks_in_regime" else getattr(s, f))
                       for f, _ in _Summary._fields_}
     if want_cache:
-        out["cache"] = [keys[j * cfg.K: j * cfg.K + int(sizes[j])].copy() for j in range(W)]
+        ks = cfg.K_stack
+        out["cache"] = [keys[j * ks: j * ks + int(sizes[j])].copy() for j in range(W)]
     if max_ticks:
         k = min(int(s.ticks), max_ticks)
         out["tick_ewma"] = te[:k].copy()
