@@ -101,6 +101,25 @@ typedef struct {
   float regime_tau[3];     /* Table 2; entry 0 unused (replica's own tau) */
   float regime_omega[3];   /* Table 2; entry 0 unused (replica's own omega) */
   double poa_window;       /* window of Eq. (12), s (> 0) */
+  /* Game 2 tiers (§4.2, Eq. kv-cost), simulation only.  tiered = 1 gives
+   * every simulated worker the exclusive tiers G1 (cache_blocks), G2
+   * (tier_k2) and G3 (tier_k3 blocks, each >= 0): an access brings a block
+   * to G1, and a full tier hands its least recently used block to the next
+   * (the last drops it), i.e. one recency stack of cache_blocks + tier_k2 +
+   * tier_k3 blocks cut into three bands.  Routing (Eq. (1)'s cached prefix)
+   * sees G1.  Every routed request is charged per full block on its worker i
+   * tier_alpha[t] for its own tier t, else the cheapest d(i, j) +
+   * tier_alpha[t] over copies on other workers j (d = tier_d_near when i and
+   * j share a node of tier_node workers, else tier_d_far; ties: same node,
+   * then the lower tier), else tier_gamma (recomputation); requires
+   * 0 <= alpha_G1 < alpha_G2 < alpha_G3 < gamma < inf, finite d >= 0,
+   * tier_node >= 1, W * (longest prompt's full blocks) <= 2048, and LRU
+   * replicas.  Defaults (the paper gives no values): off, alpha 1 / 4 / 20,
+   * gamma 100, d 2 / 10, one worker per node.  route_batch ignores tiers. */
+  int32_t tiered, tier_node;
+  int64_t tier_k2, tier_k3;
+  double tier_alpha[3];
+  double tier_gamma, tier_d_near, tier_d_far;
 } rs_config;
 
 /* Fills *cfg with the paper's constants (see above), W = 3, cache 65536. */
@@ -225,9 +244,15 @@ typedef struct {
                                §6.4: sum over windows of sum_i c_{i, worker(i)} over
                                the sum of OPTs (the static counterfactual of §9) */
   /* KV-cache pressure (the regime-transition proposition of §5.3, rho =
-   * resident blocks / (W K)): arrival time of the first request whose update
-   * evicted and rho just after that update (-1, -1 if none); rho at the end */
+   * resident blocks of every tier / (W cache_blocks)): arrival time of the
+   * first request whose update pushed a block out of a G1 cache and rho just
+   * after that update (-1, -1 if none); rho at the end */
   double first_evict_t, rho_first_evict, rho_end;
+  /* Game 2 accounting (tiered, else 0): full blocks of routed requests found
+   * in their worker's own G1 / G2 / G3, on another worker, nowhere; summed
+   * Eq. kv-cost */
+  int64_t kv_g1, kv_g2, kv_g3, kv_remote, kv_recompute;
+  double kv_cost;
 } rs_replica_result;
 
 /* Per-request records, device memory, each pointer may be NULL.  Replica r's
@@ -244,6 +269,7 @@ typedef struct {
   uint16_t* n_frozen;     /* [rows*W] min(in-service_j at a_i + 1, cap - 1) */
   uint16_t* prefix;       /* [rows*W] m_ij */
   float* cost;            /* [rows*W] Eq. (1) cost at the decision */
+  double* kv_cost;        /* [rows] Eq. kv-cost of the request on its worker (tiered; optional) */
 } rs_records;
 
 enum { RS_SIM_NO_POA = 1 };   /* flags of simulate_replicas */

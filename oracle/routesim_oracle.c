@@ -937,7 +937,11 @@ int32_t orc_simulate(const orc_config* cfg, const int32_t* tokens, const int64_t
     int64_t nb = L / B;
     int64_t nbt = (L + B - 1) / B;
     s.blk[i] = (L + out_len[i] + B - 1) / B;
-    if (nb > cfg->K) { status = ORC_ERR_CAPACITY; goto done; }
+    /* a prompt must fit the worker's cache (all tiers when tiered) */
+    if (nb > cfg->K + (cfg->tiered ? cfg->tier_k2 + cfg->tier_k3 : 0)) {
+      status = ORC_ERR_CAPACITY;
+      goto done;
+    }
     hash_request(tokens + offsets[i], nb, B, cfg->hash_seed, h);
     if (has_duplicate(h, nb, hs)) { status = ORC_ERR_COLLISION; goto done; }
     float tau = rep->tau, omega = rep->omega;

@@ -29,7 +29,8 @@ struct rs_ctx {
   cudaStream_t st = nullptr;
   int device = 0;
   std::string err;
-  TableGeom g;
+  TableGeom g;    // the live routers' caches (cache_blocks)
+  TableGeom gs;   // the simulated workers' caches (all tiers)
   ModelConsts mc;
   // live router instances
   int32_t ninst = 0;
@@ -130,6 +131,20 @@ rs_status check_config(const rs_config* cfg) {
   for (int r = 0; r < 3; r++)
     if (!(cfg->regime_tau[r] >= 0.0f) || !(cfg->regime_omega[r] >= 0.0f))
       return fail(nullptr, RS_ERR_INVALID, "regime parameters must be >= 0");
+  if (cfg->tiered != 0 && cfg->tiered != 1) return fail(nullptr, RS_ERR_INVALID, "tiered must be 0 or 1");
+  if (cfg->tiered) {
+    const double* a = cfg->tier_alpha;
+    if (cfg->tier_k2 < 0 || cfg->tier_k3 < 0 ||
+        cfg->cache_blocks + cfg->tier_k2 + cfg->tier_k3 > (1ll << 24))
+      return fail(nullptr, RS_ERR_INVALID, "tier sizes must be >= 0, all tiers <= 2^24 blocks");
+    if (!(a[0] >= 0.0 && a[0] < a[1] && a[1] < a[2] && a[2] < cfg->tier_gamma) ||
+        !std::isfinite(cfg->tier_gamma))
+      return fail(nullptr, RS_ERR_INVALID, "need 0 <= alpha_G1 < alpha_G2 < alpha_G3 < gamma < inf");
+    if (!(cfg->tier_d_near >= 0.0) || !(cfg->tier_d_far >= 0.0) ||
+        !std::isfinite(cfg->tier_d_near) || !std::isfinite(cfg->tier_d_far))
+      return fail(nullptr, RS_ERR_INVALID, "tier_d_near and tier_d_far must be finite and >= 0");
+    if (cfg->tier_node < 1) return fail(nullptr, RS_ERR_INVALID, "tier_node must be >= 1");
+  }
   return RS_OK;
 }
 
@@ -140,6 +155,11 @@ ModelConsts make_consts(const rs_config& c) {
   m.eps_frac = c.eps_frac; m.poa_window = c.poa_window; m.cap = c.cap; m.hyst_k = c.hyst_k;
   m.W = c.W; m.write_cost = 0;
   for (int r = 0; r < 3; r++) { m.regime_tau[r] = c.regime_tau[r]; m.regime_omega[r] = c.regime_omega[r]; }
+  for (int t = 0; t < 3; t++) m.tier_alpha[t] = c.tier_alpha[t];
+  m.tier_gamma = c.tier_gamma;
+  m.tier_dn = c.tier_d_near;
+  m.tier_df = c.tier_d_far;
+  m.tier_node = c.tier_node > 0 ? c.tier_node : 1;
   return m;
 }
 
@@ -190,6 +210,14 @@ void rs_config_default(rs_config* c) {
   c->regime_tau[0] = 0.0f; c->regime_tau[1] = 0.7f; c->regime_tau[2] = 0.8f;
   c->regime_omega[0] = 1.0f; c->regime_omega[1] = 1.0f; c->regime_omega[2] = 0.1f;
   c->poa_window = 5.0;
+  c->tiered = 0;          // Game 2 tiers off; the paper gives no tier costs
+  c->tier_node = 1;
+  c->tier_k2 = 0;
+  c->tier_k3 = 0;
+  c->tier_alpha[0] = 1.0; c->tier_alpha[1] = 4.0; c->tier_alpha[2] = 20.0;
+  c->tier_gamma = 100.0;
+  c->tier_d_near = 2.0;
+  c->tier_d_far = 10.0;
 }
 
 const char* route_last_error(const rs_ctx* ctx) {
@@ -215,6 +243,7 @@ rs_status route_init(rs_ctx** out, const rs_config* cfg, int32_t n_instances, vo
   ctx->st = reinterpret_cast<cudaStream_t>(cuda_stream);
   cudaGetDevice(&ctx->device);
   ctx->g = table_geom(cfg->cache_blocks);
+  ctx->gs = cfg->tiered ? table_geom(cfg->cache_blocks + cfg->tier_k2 + cfg->tier_k3) : ctx->g;
   ctx->mc = make_consts(*cfg);
   memset(&ctx->timing, 0, sizeof ctx->timing);
   for (auto& ev : ctx->ev) {
@@ -464,6 +493,7 @@ static rs_status records_effective(rs_ctx* ctx, const rs_records* user, int64_t 
       (r = pick_rec(ctx, u.prefix, ctx->rec_prefix, R * 2 * W, &eff->prefix)))
     return r;
   eff->cost = want_cost ? u.cost : nullptr;
+  eff->kv_cost = u.kv_cost;   // optional
   return RS_OK;
 }
 
@@ -522,7 +552,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   if (trace_mem != RS_MEM_DEVICE && trace_mem != RS_MEM_HOST)
     return fail(ctx, RS_ERR_INVALID, "trace_mem must be RS_MEM_DEVICE or RS_MEM_HOST");
   const int W = ctx->cfg.W;
-  const TableGeom& g = ctx->g;
+  const TableGeom& g = ctx->gs;
   for (int t = 0; t < n_traces; t++) {
     const rs_trace& tr = traces[t];
     if (tr.n_req < 0) return fail(ctx, RS_ERR_INVALID, "trace %d: n_req < 0", t);
@@ -554,6 +584,8 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       if (!(p.decay_s > 0.0) || !std::isfinite(p.decay_s))
         return fail(ctx, RS_ERR_INVALID, "replica %d: decay_s must be finite and > 0", r);
       any_freq = true;
+      if (ctx->cfg.tiered)
+        return fail(ctx, RS_ERR_INVALID, "replica %d: frequency eviction with tiers", r);
     }
     if (!(p.omega >= 0.0f) || !(p.tau >= 0.0f) || !std::isfinite(p.omega) || !std::isfinite(p.tau))
       return fail(ctx, RS_ERR_INVALID, "replica %d: omega/tau must be finite and >= 0", r);
@@ -661,10 +693,15 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   const size_t smem_room = (size_t)maxsmem > sizeof(int) * 2048 ? maxsmem - sizeof(int) * 2048 : 0;
   // per-request slot arrays in shared memory when they fit, else in global memory
   bool slots_global = false;
-  size_t smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, false);
+  const bool tiered = ctx->cfg.tiered != 0;
+  if (tiered && (int64_t)W * nbmax > SIM_PROBE_CAP)
+    return fail(ctx, RS_ERR_CAPACITY,
+                "tiers need W * (longest prompt's full blocks) <= %d; have %d * %lld", SIM_PROBE_CAP,
+                W, (long long)nbmax);
+  size_t smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, false, tiered);
   if (smem > smem_room) {
     slots_global = true;
-    smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, true);
+    smem = sim_smem_bytes(W, (int)nbmax, cmax, ctx->cfg.cap, true, tiered);
   }
   if (smem > smem_room)
     return fail(ctx, RS_ERR_CAPACITY,
@@ -753,6 +790,9 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   SimLaunch L;
   L.nsim = (int)nsim;
   L.nbmax = (int)nbmax;
+  L.tiered = tiered ? 1 : 0;
+  L.k1 = ctx->cfg.cache_blocks;
+  L.k12 = ctx->cfg.cache_blocks + (tiered ? ctx->cfg.tier_k2 : 0);
   L.cmax = cmax;
   L.slots_global = slots_global ? 1 : 0;
   L.g = g;
@@ -901,7 +941,7 @@ rs_status route_cache_dump(rs_ctx* ctx, int32_t source, int32_t index, int32_t w
   if (!size || (capacity > 0 && !keys_host)) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
   const int W = ctx->cfg.W;
   if (worker < 0 || worker >= W) return fail(ctx, RS_ERR_INVALID, "worker out of range");
-  const TableGeom& g = ctx->g;
+  const TableGeom& g = source == 1 ? ctx->gs : ctx->g;
   const uint64_t* kp;
   const uint32_t* sp;
   const uint32_t* lp;

@@ -24,6 +24,18 @@ struct CacheMeta {
   uint32_t tombs;   // tombstoned slots
 };
 
+// Game 2 tiers of one simulated worker: the log positions from which the
+// live entries are the top K_G1 (b1) and the top K_G1 + K_G2 (b2) of its
+// recency stack, i.e. G1 = [b1, T), G2 = [b2, b1), G3 = [head, b2).
+struct TierMeta {
+  uint32_t b1;
+  uint32_t b2;
+};
+
+// Kernel variants of the simulation: exact LRU, the frequency rule, Game 2 tiers.
+constexpr int SIM_LRU = 0, SIM_FREQ = 1, SIM_TIER = 2;
+constexpr int SIM_PROBE_CAP = 2048;   // W * nb up to which the probe captures every slot
+
 // Frequency eviction's search state of one worker: while the decay step is
 // below fmin, the log range [head, fscan) holds no live cold entry (fmin = 0:
 // search from the head).
@@ -65,6 +77,8 @@ struct ModelConsts {
   double lat_a, lat_b, lat_d, w_c, itl, dt, alpha, theta1, theta2, eps_frac, poa_window;
   int32_t cap, hyst_k, W, write_cost;
   float regime_tau[3], regime_omega[3];
+  double tier_alpha[3], tier_gamma, tier_dn, tier_df;   // Game 2 costs (Eq. kv-cost)
+  int32_t tier_node, reserved;
 };
 
 struct SimBuffers {
@@ -78,7 +92,7 @@ struct SimBuffers {
   int64_t pend_cap;
   CacheMeta* meta_out;      // [nsim][W]
   rs_replica_result* res;   // [nsim]
-  rs_records rec;           // every field non-NULL except possibly cost
+  rs_records rec;           // every field non-NULL except possibly cost and kv_cost
   float* dstat;             // [rows][6]: two lowest costs, draw position (see k_decision_stats)
   const double* wco_tab;    // [(nbmax+1)(nbmax+2)] w_c * (m / nbt), or NULL
   int wco_dim;              // nbmax + 2 (row length of wco_tab)
@@ -90,13 +104,16 @@ struct SimLaunch {
   int nbmax;                // max full blocks of any routed prompt
   int cmax;                 // max concurrency over replicas
   int slots_global;         // 1: per-request slot arrays in SimBuffers::slotmem
+  int tiered;               // 1: Game 2 tiers (g.K = all tiers of a worker)
+  int64_t k1, k12;          // G1 capacity, G1 + G2 capacity (k1 = g.K without tiers)
   TableGeom g;
   ModelConsts mc;
 };
 
 // Dynamic shared memory of one replica CTA; with slots_global the per-request
 // slot arrays are in global memory instead (sim_slot_bytes per replica).
-size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global);
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global,
+                      bool tiered = false);
 size_t sim_slot_bytes(int cmax);
 
 // One trace for the block-hash kernels: requests req_base .. req_base+n_req-1

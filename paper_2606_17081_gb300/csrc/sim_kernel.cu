@@ -28,7 +28,7 @@ namespace rs {
 constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (warps 0-6)
 constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
 constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
-constexpr int PROBE_CAP = 2048;          // W * nb up to which the probe captures every slot
+constexpr int PROBE_CAP = SIM_PROBE_CAP;   // W * nb up to which the probe captures every slot
 constexpr int PROBE_ILP = 2;             // lookups a thread keeps in flight
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -37,7 +37,7 @@ struct SimLayout {
   size_t ftab, wwco, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
   size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
-  size_t wmeta, wfreq, winserv, wqh, wqt, wm, wcost, wopen, wabs;
+  size_t wmeta, wfreq, wtier, ptier, winserv, wqh, wqt, wm, wcost, wopen, wabs;
   size_t kind, evk, touched;
   size_t total;
   size_t slot_bytes;   // per-replica global bytes of the slot arrays (0: in shared memory)
@@ -49,7 +49,8 @@ struct SimLayout {
 // whose slots do not fit in shared memory; their offsets are then relative to
 // the replica's global slot area.
 __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax, int nft,
-                                                     bool slots_global = false) {
+                                                     bool slots_global = false,
+                                                     bool tiered = false) {
   SimLayout L;
   size_t o = 0, og = 0;
   const size_t nb = (size_t)(nbmax > 0 ? nbmax : 1);
@@ -98,6 +99,8 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(vt, 4 * nv, 4)
   TAKE(wmeta, sizeof(CacheMeta) * (size_t)W, 16)
   TAKE(wfreq, sizeof(FreqMeta) * (size_t)W, 8)
+  TAKE(wtier, tiered ? sizeof(TierMeta) * (size_t)W : 0, 8)
+  TAKE(ptier, tiered ? (size_t)PROBE_CAP : 0, 4)
   TAKE(winserv, 4 * (size_t)W, 4)
   TAKE(wqh, 4 * (size_t)W, 4)
   TAKE(wqt, 4 * (size_t)W, 4)
@@ -117,8 +120,8 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
 
 __host__ __device__ inline int ftab_size(int cap) { return cap < FTAB_MAX ? cap : FTAB_MAX; }
 
-size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global) {
-  return make_sim_layout(W, nbmax, cmax, ftab_size(cap), slots_global).total;
+size_t sim_smem_bytes(int W, int nbmax, int cmax, int cap, bool slots_global, bool tiered) {
+  return make_sim_layout(W, nbmax, cmax, ftab_size(cap), slots_global, tiered).total;
 }
 
 size_t sim_slot_bytes(int cmax) {
@@ -157,6 +160,10 @@ struct SimScalars {
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
   int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, nabs;
   uint32_t dclock;             // decay step of the request being updated (frequency eviction)
+  int64_t kv[5];               // Game 2: own G1 / G2 / G3, remote, recompute blocks
+  double kv_cost;              // summed Eq. kv-cost
+  int kvacc[10];               // one request's Game 2 categories (update group)
+  int64_t tier_out;            // blocks the last update pushed out of G1
   UpdateShared us;
   uint32_t scan_pos;
   int warp_tot[NT_SIM / 32];
@@ -178,6 +185,8 @@ struct SimCtx {
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
   CacheMeta* wmeta;
   FreqMeta* wfreq;
+  TierMeta* wtier;    // Game 2 band boundaries per worker (tiered)
+  uint8_t* ptier;     // [W][nb] tier of each (worker, block) pair, 0 = absent (tiered)
   int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs, *dclaim;
   uint32_t *pslot, *pfree;
   int64_t* wA;
@@ -566,7 +575,10 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
 // PROBE_CAP): each thread issues the first-bucket loads of PROBE_ILP pairs
 // before resolving them, and the slot found (or the first free slot of the
 // probe path) is kept for the chosen worker's update.
-template <int NT>
+// TIER: m_j counts the leading blocks in G1 (a found slot's stamp at or
+// past the worker's b1); every pair's tier goes to ptier; the absent count
+// is of blocks in no tier.
+template <int NT, bool TIER = false>
 __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
@@ -593,6 +605,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
     for (int r = 0; r < PROBE_ILP; r++) {
       const int it = base + r * NT + threadIdx.x;
       int miss = 0x7FFFFFFF;
+      bool absent = false;
       if (jj[r] >= 0) {
         const uint64_t h = hbuf[kk[r]];
         uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
@@ -603,14 +616,29 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
         }
         c.pslot[it] = sl;
         c.pfree[it] = fr;
-        if (sl == SLOT_NONE) miss = kk[r];
+        if (TIER) {
+          int tier = 0;
+          if (sl != SLOT_NONE) {
+            const uint32_t st = __ldcg(c.table(jj[r]).stamp + sl);
+            const TierMeta tm = c.wtier[jj[r]];
+            tier = st >= tm.b1 ? 1 : (st >= tm.b2 ? 2 : 3);
+          }
+          c.ptier[it] = (uint8_t)tier;
+          absent = sl == SLOT_NONE;
+          if (tier != 1) miss = kk[r];
+        } else if (sl == SLOT_NONE) {
+          miss = kk[r];
+        }
       }
       const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
       const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
-      const unsigned nab = __popc(__ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp);
-      if (jj[r] >= 0 && (__ffs(grp) - 1) == (int)(threadIdx.x & 31) && nab) {
+      const unsigned nab =
+          __popc(__ballot_sync(FULL_MASK, TIER ? absent : miss != 0x7FFFFFFF) & grp);
+      // (tiers: a block below G1 ends the prefix though it is present)
+      if (jj[r] >= 0 && (__ffs(grp) - 1) == (int)(threadIdx.x & 31) &&
+          (nab || (TIER && m != 0x7FFFFFFF))) {
         atomicMin(&c.wm[jj[r]], m);
-        atomicAdd(&c.wabs[jj[r]], (int)nab);   // absent blocks, for the update's victim count
+        if (nab) atomicAdd(&c.wabs[jj[r]], (int)nab);   // absent blocks, for the victim count
       }
     }
   }
@@ -619,12 +647,154 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   grp_bar<NT>();
 }
 
+// Game 2 charge of request i (Eq. kv-cost, §4.2) on its worker sigma, from the
+// probe's tiers (update group, before the update): per block alpha_t for
+// sigma's own tier t; else the cheapest d(sigma, j) + alpha_t over other
+// workers' copies (same node before other node, then the lower tier); else
+// gamma.  The categories are counted, and the cost summed in a fixed order.
+template <int NT>
+__device__ __forceinline__ void tier_charge(SimCtx& c, int sigma, int nb, int64_t row) {
+  SimScalars& S = *c.S;
+  const ModelConsts& mc = c.L->mc;
+  const int W = mc.W;
+  const int node = sigma / mc.tier_node;
+  int cnt[10];
+#pragma unroll
+  for (int q = 0; q < 10; q++) cnt[q] = 0;
+  for (int k = threadIdx.x; k < nb; k += NT) {
+    const int t = c.ptier[sigma * nb + k];
+    if (t > 0) {
+      cnt[t - 1]++;
+      continue;
+    }
+    unsigned has = 0;   // bit 3 r + (q - 1): a copy at tier q, r = 0 same node, 1 other
+    for (int j = 0; j < W; j++) {
+      const int tj = c.ptier[j * nb + k];
+      if (j == sigma || tj == 0) continue;
+      has |= 1u << (3 * (j / mc.tier_node == node ? 0 : 1) + tj - 1);
+    }
+    int cat = 9;
+    double best = __longlong_as_double(0x7FF0000000000000ll);
+    for (int b = 0; b < 6; b++) {
+      if (!(has >> b & 1u)) continue;
+      const double v = __dadd_rn(b < 3 ? mc.tier_dn : mc.tier_df, mc.tier_alpha[b % 3]);
+      if (v < best) {
+        best = v;
+        cat = 3 + b;
+      }
+    }
+    cnt[cat]++;
+  }
+#pragma unroll
+  for (int q = 0; q < 10; q++) {
+    const int v = (int)__reduce_add_sync(FULL_MASK, (unsigned)cnt[q]);
+    if ((threadIdx.x & 31) == 0 && v) atomicAdd(&S.kvacc[q], v);
+  }
+  grp_bar<NT>();
+  if (threadIdx.x == 0) {
+    const double* al = mc.tier_alpha;
+    double cost = __dmul_rn(al[0], (double)S.kvacc[0]);
+    cost = __dadd_rn(cost, __dmul_rn(al[1], (double)S.kvacc[1]));
+    cost = __dadd_rn(cost, __dmul_rn(al[2], (double)S.kvacc[2]));
+    for (int q = 0; q < 3; q++)
+      cost = __dadd_rn(cost, __dmul_rn(__dadd_rn(mc.tier_dn, al[q]), (double)S.kvacc[3 + q]));
+    for (int q = 0; q < 3; q++)
+      cost = __dadd_rn(cost, __dmul_rn(__dadd_rn(mc.tier_df, al[q]), (double)S.kvacc[6 + q]));
+    cost = __dadd_rn(cost, __dmul_rn(mc.tier_gamma, (double)S.kvacc[9]));
+    S.kv[0] += S.kvacc[0];
+    S.kv[1] += S.kvacc[1];
+    S.kv[2] += S.kvacc[2];
+    S.kv[3] += S.kvacc[3] + S.kvacc[4] + S.kvacc[5] + S.kvacc[6] + S.kvacc[7] + S.kvacc[8];
+    S.kv[4] += S.kvacc[9];
+    S.kv_cost = __dadd_rn(S.kv_cost, cost);
+    if (c.b->rec.kv_cost) c.b->rec.kv_cost[row] = cost;
+#pragma unroll
+    for (int q = 0; q < 10; q++) S.kvacc[q] = 0;   // for the next request
+  }
+}
+
+// Moves a band boundary of the recency stack past `excess` live log entries
+// (they drop to the band below): the new boundary follows the excess-th live
+// entry at or after *b.  CTA-wide.
+template <int NT>
+__device__ __forceinline__ void tier_shift(const TableView& t, const CacheMeta* meta, uint32_t* b,
+                                           uint32_t excess, int* warp_tot, uint32_t* out) {
+  if (excess == 0) return;
+  const uint32_t T = meta->T;
+  uint32_t have = 0;
+  for (uint32_t p0 = *b; p0 < T; p0 += NT) {   // uniform
+    const uint32_t p = p0 + threadIdx.x;
+    bool live = false;
+    if (p < T) live = __ldcg(t.stamp + t.log[p & t.rmask]) == p;
+    int tot;
+    const int r = cta_rank<NT>(live, warp_tot, &tot);
+    if (live && have + (uint32_t)r == excess - 1) *out = p + 1;
+    have += (uint32_t)tot;
+    if (have >= excess) break;
+  }
+  grp_bar<NT>();
+  if (threadIdx.x == 0) *b = have >= excess ? *out : T;
+  grp_bar<NT>();
+}
+
+// After the chosen worker's LRU update of its whole stack: the G1 and G2
+// bands move down by the live entries that no longer fit.  size0, b0: the
+// stack size and boundaries before the update; us/sc: the update's record
+// (kinds, present blocks' old stamps, victims).  Sets S.tier_out = blocks that
+// left G1 (moved below b1, or evicted from it).
+template <int NT>
+__device__ __forceinline__ void tier_advance(SimCtx& c, const TableView& tv, const CacheMeta* meta,
+                                             TierMeta* tm, uint32_t size0, TierMeta b0, int nb) {
+  SimScalars& S = *c.S;
+  const UpdateScratch& sc = c.sc;
+  int d1 = 0, d2 = 0, v1 = 0;
+  for (int k = threadIdx.x; k < nb; k += NT)
+    if (sc.kind[k] == 0) {
+      d1 += sc.pst[k] >= b0.b1;
+      d2 += sc.pst[k] >= b0.b2;
+    }
+  const int E = S.us.n_victims;
+  for (int v = threadIdx.x; v < E; v += NT) {
+    const uint32_t p = sc.vt[sc.victim[v]];
+    v1 += p >= b0.b1;
+    d2 += p >= b0.b2;
+  }
+  d1 += v1;
+  d1 = (int)__reduce_add_sync(FULL_MASK, (unsigned)d1);
+  d2 = (int)__reduce_add_sync(FULL_MASK, (unsigned)d2);
+  v1 = (int)__reduce_add_sync(FULL_MASK, (unsigned)v1);
+  if ((threadIdx.x & 31) == 0) {
+    atomicAdd(&S.kvacc[0], d1);   // kvacc is free between charges
+    atomicAdd(&S.kvacc[1], d2);
+    atomicAdd(&S.kvacc[2], v1);
+  }
+  grp_bar<NT>();
+  const uint32_t size = meta->size;
+  const int64_t k1 = c.L->k1, k12 = c.L->k12;
+  const int64_t live1 = min((int64_t)size0, k1) - S.kvacc[0] + nb;
+  const int64_t live2 = min((int64_t)size0, k12) - S.kvacc[1] + nb;
+  const int64_t x1 = live1 - min((int64_t)size, k1);
+  const int64_t x2 = live2 - min((int64_t)size, k12);
+  const int vout = S.kvacc[2];
+  grp_bar<NT>();
+  if (threadIdx.x == 0) {
+    S.kvacc[0] = S.kvacc[1] = S.kvacc[2] = 0;
+    S.tier_out = (x1 > 0 ? x1 : 0) + vout;
+    if ((int64_t)size <= k1) tm->b1 = meta->head;
+    if ((int64_t)size <= k12) tm->b2 = meta->head;
+  }
+  if ((int64_t)size > k1 && x1 > 0) tier_shift<NT>(tv, meta, &tm->b1, (uint32_t)x1, S.warp_tot, &S.scan_pos);
+  if ((int64_t)size > k12 && x2 > 0) tier_shift<NT>(tv, meta, &tm->b2, (uint32_t)x2, S.warp_tot, &S.scan_pos);
+  grp_bar<NT>();
+}
+
 // Cache update of the chosen worker (update group, warps 0-6) for request i.
-// FREQ: the launch holds replicas that evict by frequency (the LRU-only
-// kernel carries none of that code).
-template <bool FREQ>
+// MODE: SIM_FREQ when the launch holds replicas that evict by frequency,
+// SIM_TIER for Game 2 tiers (the LRU-only kernel carries neither).
+template <int MODE>
 __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb,
                                               bool full, int64_t i) {
+  constexpr bool FREQ = MODE == SIM_FREQ, TIER = MODE == SIM_TIER;
   SimScalars& S = *c.S;
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
@@ -639,8 +809,18 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     cache_rebuild<NT_UPD>(tv, meta, g.K, gtmp, S.warp_tot, &S.us,
                           FREQ && c.b->tmpe ? c.b->tmpe + (size_t)c.sid * g.K : nullptr,
                           FREQ ? &c.wfreq[j] : nullptr);
-    if (threadIdx.x == 0) S.rebuilds++;
+    if (threadIdx.x == 0) {
+      S.rebuilds++;
+      if (TIER) {   // stamps renumbered 0 .. size-1 in recency order
+        const int64_t sz = meta->size;
+        c.wtier[j].b1 = (uint32_t)(sz - min(sz, c.L->k1));
+        c.wtier[j].b2 = (uint32_t)(sz - min(sz, c.L->k12));
+      }
+    }
+    if (TIER) grp_bar<NT_UPD>();
   }
+  const uint32_t size0 = meta->size;   // before this update (tiers)
+  const TierMeta b0 = TIER ? c.wtier[j] : TierMeta{0u, 0u};
   const bool captured = full && !S.rebuild;
   if (FREQ && c.d->eviction == RS_EVICT_FREQ) {
     // the KV Block Manager's frequency rule
@@ -664,12 +844,16 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
     else
       cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
     cache_apply<NT_UPD>(tv, meta, g.K, hbuf, nb, c.sc, &S.us, S.warp_tot, &S.scan_pos, captured);
+    if (TIER) {
+      grp_bar<NT_UPD>();   // the meta update of cache_apply
+      tier_advance<NT_UPD>(c, tv, meta, &c.wtier[j], size0, b0, nb);
+    }
   }
   if (threadIdx.x == 0) {
     if (S.us.err) S.status = S.us.err;
     S.inserted += S.us.n_ins;
     S.evicted += S.us.n_victims;
-    if (S.us.n_victims > 0 && S.first_evict_i < 0) {
+    if ((TIER ? S.tier_out : (int64_t)S.us.n_victims) > 0 && S.first_evict_i < 0) {
       // the first update that evicted; resident blocks = inserted - evicted
       S.first_evict_i = i;
       S.first_live = S.inserted - S.evicted;
@@ -769,9 +953,10 @@ __device__ __forceinline__ void stage_hashes(const SimCtx& c, const ReqState& q,
 // every replica has an SM to itself.
 // SG: the per-request slot arrays are in global memory (a compile-time
 // choice, so that in the common case the compiler knows they are shared).
-template <int MINB, bool SG, bool FREQ>
+template <int MINB, bool SG, int MODE>
 __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
+  constexpr bool FREQ = MODE == SIM_FREQ, TIER = MODE == SIM_TIER;
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ SimScalars S;
   const int sid = blockIdx.x;
@@ -779,7 +964,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   const int W = L.mc.W;
   const ModelConsts& mc = L.mc;
   const int nft = ftab_size(mc.cap);
-  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax, nft, SG);
+  const SimLayout lay = make_sim_layout(W, L.nbmax, L.cmax, nft, SG, TIER);
   // the slot arrays: shared memory, or this replica's global slot area
   unsigned char* slotbase;
   if constexpr (SG)
@@ -809,6 +994,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.freestk = reinterpret_cast<int32_t*>(slotbase + lay.freestk);
   c.wmeta = reinterpret_cast<CacheMeta*>(smem + lay.wmeta);
   c.wfreq = reinterpret_cast<FreqMeta*>(smem + lay.wfreq);
+  c.wtier = reinterpret_cast<TierMeta*>(smem + lay.wtier);
+  c.ptier = reinterpret_cast<uint8_t*>(smem + lay.ptier);
   c.winserv = reinterpret_cast<int32_t*>(smem + lay.winserv);
   c.wqh = reinterpret_cast<int32_t*>(smem + lay.wqh);
   c.wqt = reinterpret_cast<int32_t*>(smem + lay.wqt);
@@ -856,6 +1043,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     for (int j = threadIdx.x; j < W; j += NT_SIM) {
       c.wmeta[j] = CacheMeta{};
       c.wfreq[j] = FreqMeta{0u, 0u};
+      if (TIER) c.wtier[j] = TierMeta{0u, 0u};
       c.winserv[j] = 0;
       c.wA[j] = 0;
       c.wqh[j] = -1;
@@ -905,8 +1093,14 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     const int64_t row = d.rec_base + i;
     if (warp < NT_SIM / 32 - 1) {
       // ---- cached prefix on every worker (warps 0-6)
-      if (full) probe_full<NT_UPD>(c, hb, nb);
-      else probe_prefixes<NT_UPD>(c, hb, nb);
+      if (full) {
+        probe_full<NT_UPD, TIER>(c, hb, nb);
+      } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
+        if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
+        grp_bar<NT_UPD>();
+      } else {
+        probe_prefixes<NT_UPD>(c, hb, nb);
+      }
     } else if (lane == 0) {
       // ---- control thread, at the same time: completions and controller
       // samples up to request i's arrival (the probe needs none of them)
@@ -1008,7 +1202,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     const int js = S.jstar;
     if (warp < NT_SIM / 32 - 1) {
       // ---- the chosen worker's LRU cache (warps 0-6)
-      update_chosen<FREQ>(c, hb, js, nb, full, i);
+      if (TIER) tier_charge<NT_UPD>(c, js, nb, row);
+      update_chosen<MODE>(c, hb, js, nb, full, i);
     } else {
       // ---- control warp: request i's load and latency; request i+1's
       // scalars, probe state and block hashes
@@ -1114,8 +1309,9 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     r.slow_path = S.slow;
     r.rebuilds = S.rebuilds;
     r.first_switch_t = S.first_switch_t;
-    // KV-cache pressure: resident blocks over W K (resident = inserted - evicted)
-    const double cap = __dmul_rn((double)W, (double)L.g.K);
+    // KV-cache pressure: resident blocks of every tier over W K_G1
+    // (resident = inserted - evicted)
+    const double cap = __dmul_rn((double)W, (double)L.k1);
     r.first_evict_t = -1.0;
     r.rho_first_evict = -1.0;
     if (S.first_evict_i >= 0) {
@@ -1123,6 +1319,12 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       r.rho_first_evict = __ddiv_rn((double)S.first_live, cap);
     }
     r.rho_end = __ddiv_rn((double)(S.inserted - S.evicted), cap);
+    r.kv_g1 = S.kv[0];
+    r.kv_g2 = S.kv[1];
+    r.kv_g3 = S.kv[2];
+    r.kv_remote = S.kv[3];
+    r.kv_recompute = S.kv[4];
+    r.kv_cost = S.kv_cost;
     b.res[sid] = r;
   }
   for (int j = threadIdx.x; j < W; j += NT_SIM) b.meta_out[(size_t)sid * W + j] = c.wmeta[j];
@@ -1204,21 +1406,26 @@ cudaError_t launch_decision_stats(const SimDesc* d_desc, const SimBuffers& b, co
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,
                        cudaStream_t st) {
   if (L.nsim <= 0) return cudaSuccess;
-  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap, L.slots_global != 0);
+  const size_t smem = sim_smem_bytes(L.mc.W, L.nbmax, L.cmax, L.mc.cap, L.slots_global != 0,
+                                    L.tiered != 0);
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   // one replica per SM: the kernel may use every register
   const bool one = L.nsim <= sms;
-  // frequency eviction state present: the kernel with the frequency rule
+  // Game 2 tiers, or frequency eviction state present: the kernel with that
+  // variant; else the LRU-only kernel
   void (*kern)(const SimDesc*, SimBuffers, SimLaunch);
-  if (b.fexp)
-    kern = one ? (L.slots_global ? k_sim<1, true, true> : k_sim<1, false, true>)
-               : (L.slots_global ? k_sim<2, true, true> : k_sim<2, false, true>);
+  if (L.tiered)
+    kern = one ? (L.slots_global ? k_sim<1, true, SIM_TIER> : k_sim<1, false, SIM_TIER>)
+               : (L.slots_global ? k_sim<2, true, SIM_TIER> : k_sim<2, false, SIM_TIER>);
+  else if (b.fexp)
+    kern = one ? (L.slots_global ? k_sim<1, true, SIM_FREQ> : k_sim<1, false, SIM_FREQ>)
+               : (L.slots_global ? k_sim<2, true, SIM_FREQ> : k_sim<2, false, SIM_FREQ>);
   else
-    kern = one ? (L.slots_global ? k_sim<1, true, false> : k_sim<1, false, false>)
-               : (L.slots_global ? k_sim<2, true, false> : k_sim<2, false, false>);
+    kern = one ? (L.slots_global ? k_sim<1, true, SIM_LRU> : k_sim<1, false, SIM_LRU>)
+               : (L.slots_global ? k_sim<2, true, SIM_LRU> : k_sim<2, false, SIM_LRU>);
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   kern<<<L.nsim, NT_SIM, smem, st>>>(d_desc, b, L);

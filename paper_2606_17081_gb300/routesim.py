@@ -34,7 +34,10 @@ class rs_config(C.Structure):
                 ("w_c", C.c_double), ("itl", C.c_double), ("dt", C.c_double),
                 ("alpha", C.c_double), ("theta1", C.c_double), ("theta2", C.c_double),
                 ("eps_frac", C.c_double), ("regime_tau", C.c_float * 3),
-                ("regime_omega", C.c_float * 3), ("poa_window", C.c_double)]
+                ("regime_omega", C.c_float * 3), ("poa_window", C.c_double),
+                ("tiered", C.c_int32), ("tier_node", C.c_int32), ("tier_k2", C.c_int64),
+                ("tier_k3", C.c_int64), ("tier_alpha", C.c_double * 3), ("tier_gamma", C.c_double),
+                ("tier_d_near", C.c_double), ("tier_d_far", C.c_double)]
 
 
 class rs_trace(C.Structure):
@@ -64,7 +67,9 @@ class rs_replica_result(C.Structure):
                 ("slow_path", C.c_int64), ("rebuilds", C.c_int64),
                 ("first_switch_t", C.c_double), ("poa_static", C.c_double),
                 ("first_evict_t", C.c_double), ("rho_first_evict", C.c_double),
-                ("rho_end", C.c_double)]
+                ("rho_end", C.c_double), ("kv_g1", C.c_int64), ("kv_g2", C.c_int64),
+                ("kv_g3", C.c_int64), ("kv_remote", C.c_int64), ("kv_recompute", C.c_int64),
+                ("kv_cost", C.c_double)]
 
     def as_dict(self) -> dict:
         return {f: (list(getattr(self, f)) if f == "ticks_in_regime" else getattr(self, f))
@@ -75,7 +80,7 @@ class rs_records(C.Structure):
     _fields_ = [("worker", C.c_void_p), ("arrival", C.c_void_p), ("start", C.c_void_p),
                 ("first_token", C.c_void_p), ("completion", C.c_void_p), ("ttft", C.c_void_p),
                 ("nbt", C.c_void_p), ("n_frozen", C.c_void_p), ("prefix", C.c_void_p),
-                ("cost", C.c_void_p)]
+                ("cost", C.c_void_p), ("kv_cost", C.c_void_p)]
 
 
 class rs_timing(C.Structure):
@@ -312,7 +317,8 @@ def replica_params(r) -> rs_replica_params:
                              int(getattr(r, "freq_max", 64)), float(getattr(r, "decay_s", 1.0)))
 
 
-def device_records(rows: int, W: int, device="cuda", with_cost: bool = False):
+def device_records(rows: int, W: int, device="cuda", with_cost: bool = False,
+                   with_kv: bool = False):
     """Caller-owned record tensors and the rs_records struct pointing at them."""
     import torch
     t = {
@@ -328,6 +334,8 @@ def device_records(rows: int, W: int, device="cuda", with_cost: bool = False):
     }
     if with_cost:
         t["cost"] = torch.zeros(rows * W, dtype=torch.float32, device=device)
+    if with_kv:
+        t["kv_cost"] = torch.zeros(rows, dtype=torch.float64, device=device)
     rec = rs_records(*[t[k].data_ptr() if k in t else None for k, _ in rs_records._fields_])
     return rec, t
 
@@ -342,6 +350,8 @@ class Context:
         for k, v in fields.items():
             if k in ("regime_tau", "regime_omega"):
                 setattr(cfg, k, (C.c_float * 3)(*v))
+            elif k == "tier_alpha":
+                setattr(cfg, k, (C.c_double * 3)(*v))
             else:
                 setattr(cfg, k, v)
         self.cfg = cfg

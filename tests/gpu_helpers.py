@@ -16,7 +16,8 @@ def gpu_run(ctx, traces, replicas, trace_mem=rs.RS_MEM_DEVICE, with_cost=True, f
     bufs = [rs.device_trace(t) if trace_mem == rs.RS_MEM_DEVICE else rs.host_trace(t)
             for t in traces]
     rows = sum(r.n_req for r in replicas)
-    rec, t = rs.device_records(max(rows, 1), W, with_cost=with_cost)
+    with_kv = bool(ctx.cfg.tiered)
+    rec, t = rs.device_records(max(rows, 1), W, with_cost=with_cost, with_kv=with_kv)
     try:
         res = rs.simulate_replicas(ctx.h, [b.desc() for b in bufs], trace_mem,
                                    [rs.replica_params(r) for r in replicas], rec, flags)
@@ -30,7 +31,7 @@ def gpu_run(ctx, traces, replicas, trace_mem=rs.RS_MEM_DEVICE, with_cost=True, f
     base = 0
     for k, r in enumerate(replicas):
         n = r.n_req
-        d = {f: host[f][base:base + n] for f in REC_FIELDS}
+        d = {f: host[f][base:base + n] for f in REC_FIELDS + (("kv_cost",) if with_kv else ())}
         for f in ("n_frozen", "prefix") + (("cost",) if with_cost else ()):
             a = host[f][base * W:(base + n) * W].reshape(n, W)
             d[f] = a.view(np.uint16) if a.dtype == np.int16 else a
@@ -42,6 +43,11 @@ def gpu_run(ctx, traces, replicas, trace_mem=rs.RS_MEM_DEVICE, with_cost=True, f
 
 def oracle_cfg(ctx_or_W, K=None, **kw):
     if K is None:
+        c = ctx_or_W.cfg
+        if c.tiered:   # the context's Game 2 tiers
+            kw.update(tiered=1, tier_node=c.tier_node, tier_k2=c.tier_k2, tier_k3=c.tier_k3,
+                      tier_alpha=tuple(c.tier_alpha), tier_gamma=c.tier_gamma,
+                      tier_d_near=c.tier_d_near, tier_d_far=c.tier_d_far)
         return O.OracleConfig(W=ctx_or_W.W, K=ctx_or_W.K, **kw)
     return O.OracleConfig(W=ctx_or_W, K=K, **kw)
 
@@ -67,8 +73,11 @@ def assert_replica_equal(g, o, W, times_rtol=1e-12, check_cost=True):
         assert np.allclose(g[f], o[f], rtol=times_rtol, atol=0), f
     gr, orr = g["result"], o["summary"]
     assert gr["first_switch_t"] == orr["first_switch_t"], (gr["first_switch_t"], orr["first_switch_t"])
-    for f in ("first_evict_t", "rho_first_evict", "rho_end"):
+    for f in ("first_evict_t", "rho_first_evict", "rho_end", "kv_g1", "kv_g2", "kv_g3",
+              "kv_remote", "kv_recompute", "kv_cost"):
         assert gr[f] == orr[f], (f, gr[f], orr[f])
+    if "kv_cost" in g:
+        assert np.array_equal(g["kv_cost"], o["kv_cost"]), "Eq. kv-cost per request differs"
     for f in ("n_routed", "near_ties", "exact_ties", "sampled", "near_boundary", "hit_blocks",
               "inserted_blocks", "evicted_blocks", "ticks", "regime_switches", "final_regime",
               "max_regime"):
