@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 31854879744 + 6050301440,
-               "sources_sha256": "918833786b08d37faf7246658648fea1a0bcd57d4ccb62eda83a2e51780efdd2",
+SIM_TRAFFIC = {"bytes": 31858827520 + 6052403712,
+               "sources_sha256": "57a2909922d2afb962cf6321167cd2d610fd2d2115576b32f2066dcf123f02fc",
                "summary": "profiles/k_sim_p2d.md"}
 
 
