@@ -81,3 +81,75 @@ def test_load_spike_static_and_adaptive():
             assert fs > r.c_t1          # the adaptive replicas switch during the spike
         else:
             assert fs == -1.0
+
+
+def _full_launch(p, flags=0):
+    """One simulate_replicas call over the whole plan (the benchmark's launch
+    configuration); records stay on the device."""
+    traces = p.traces()
+    ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
+    bufs = [rs.device_trace(t) for t in traces]
+    rows = sum(r.n_req for r in p.replicas)
+    rec, t = rs.device_records(rows, p.W)
+    res = rs.simulate_replicas(ctx.h, [b.desc() for b in bufs], rs.RS_MEM_DEVICE,
+                               [rs.replica_params(r) for r in p.replicas], rec, flags)
+    torch.cuda.synchronize()
+    base = np.concatenate([[0], np.cumsum([r.n_req for r in p.replicas])]).astype(np.int64)
+    return ctx, traces, res, t, base
+
+
+def _rows(t, b0, n, W):
+    d = {f: t[f][b0:b0 + n].cpu().numpy() for f in ("worker", "arrival", "start", "first_token",
+                                                     "completion", "ttft", "nbt")}
+    for f in ("n_frozen", "prefix"):
+        d[f] = t[f][b0 * W:(b0 + n) * W].cpu().numpy().view(np.uint16).reshape(n, W)
+    return d
+
+
+def _prefix_equal(g, o, W):
+    # a replica's first N requests do not depend on later ones: the full-size
+    # run's first N records equal those of the oracle's N-request run
+    assert np.array_equal(g["worker"], o["worker"])
+    assert np.array_equal(g["prefix"], o["prefix"])
+    assert np.array_equal(g["n_frozen"], o["n_frozen"])
+    assert np.array_equal(g["nbt"], o["nbt"])
+    for f in ("arrival", "start", "first_token", "completion", "ttft"):
+        assert np.allclose(g[f], o[f], rtol=1e-12, atol=0), f
+
+
+def test_p5d_full_size_prefix_of_sampled_replicas():
+    # 256 replicas x 50 000 requests (two replicas per SM): every replica's
+    # first 4000 requests checked on a sample
+    p = wk.plan("p5d")
+    ctx, traces, res, t, base = _full_launch(p)
+    assert all(r.status == 0 for r in res)
+    cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
+    N = 4000
+    for k in (0, 101, 255):
+        r = p.replicas[k]
+        rr = wk.Replica(**{**vars(r), "n_req": N})
+        o = oracle_run(cfg, traces[r.trace], rr)
+        _prefix_equal(_rows(t, int(base[k]), N, p.W), o, p.W)
+    assert sum(x.regime_switches for x in res) > 0
+    ctx.close()
+
+
+def test_grid_full_size_sampled_replicas():
+    # 8192 replicas x 10 000 requests in one launch; sampled replicas whole,
+    # PoA included
+    p = wk.plan("grid")
+    ctx, traces, res, t, base = _full_launch(p)
+    assert all(r.status == 0 for r in res)
+    cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
+    for k in (0, 1, 4321, 8191):
+        r = p.replicas[k]
+        o = oracle_run(cfg, traces[r.trace], r)
+        g = _rows(t, int(base[k]), r.n_req, p.W)
+        _prefix_equal(g, o, p.W)
+        res_k = res[k].as_dict()
+        for f in ("n_routed", "hit_blocks", "inserted_blocks", "evicted_blocks", "exact_ties",
+                  "near_ties"):
+            assert res_k[f] == o["summary"][f], f
+        _, _, _, tot = O.poa(cfg, o)
+        assert abs(res_k["poa_total"] - tot) <= 1e-4 * tot
+    ctx.close()
