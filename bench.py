@@ -198,6 +198,50 @@ def _aux_knee(rs, ctx, p, descs, params, reps: int = 5) -> dict:
                            "first_knee_C": [float(x) for x in out["knee_load"]]}}
 
 
+def _aux_variants(rs, p, descs, reps: int = 2) -> dict:
+    """Outside the timed steps: the simulation kernel's device time on the same
+    p2d replicas under each variant of the method (frequency eviction, Game 2
+    tiers, power of two choices), and on the load-spike plan (Experiment 3).
+    Each variant runs once to warm up, then `reps` times; decisions/s counts
+    requests x W as the main line does."""
+    from dataclasses import replace as dc_replace
+    from paper_2606_17081_gb300 import workloads as wk
+    out = {}
+
+    def timed(ctx, descs_v, params_v, decisions):
+        rs.simulate_replicas(ctx.h, descs_v, rs.RS_MEM_DEVICE, params_v)
+        ms = []
+        for _ in range(reps):
+            rs.simulate_replicas(ctx.h, descs_v, rs.RS_MEM_DEVICE, params_v)
+            ms.append(rs.route_last_timing(ctx.h).sim_ms)
+        sim = statistics.mean(ms)
+        return {"sim_ms": sim, "decisions_per_s": decisions / (sim / 1e3)}
+
+    decisions = sum(r.n_req for r in p.replicas) * p.W
+    ctx = rs.Context(W=p.W, K=p.K)
+    freq = [rs.replica_params(dc_replace(r, eviction=rs.RS_EVICT_FREQ, freq_max=64, decay_s=1.0))
+            for r in p.replicas]
+    out["frequency_eviction"] = {**timed(ctx, descs, freq, decisions), "freq_max": 64,
+                                 "decay_s": 1.0}
+    p2c = [rs.replica_params(dc_replace(r, policy=rs.RS_POLICY_P2C)) for r in p.replicas]
+    out["power_of_two_choices"] = timed(ctx, descs, p2c, decisions)
+    ctx.close()
+    ctx = rs.Context(W=p.W, K=p.K, tiered=1, tier_k2=p.K, tier_k3=2 * p.K, tier_node=1)
+    base = [rs.replica_params(r) for r in p.replicas]
+    out["game2_tiers"] = {**timed(ctx, descs, base, decisions), "tier_blocks": [p.K, p.K, 2 * p.K]}
+    ctx.close()
+    sp = wk.plan("spike")
+    trs = sp.traces()
+    dev = [rs.device_trace(t) for t in trs]
+    ctx = rs.Context(W=sp.W, K=sp.K, theta1=sp.theta1, theta2=sp.theta2)
+    out["load_spike_plan"] = {**timed(ctx, [b.desc() for b in dev],
+                                      [rs.replica_params(r) for r in sp.replicas],
+                                      sum(r.n_req for r in sp.replicas) * sp.W),
+                              "replicas": len(sp.replicas)}
+    ctx.close()
+    return out
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -266,7 +310,11 @@ def run_gpu(args):
     barrier()
     e2e_s = time.perf_counter() - t0
     ms, e2e_s = _max_over_ranks([ms, e2e_s], "cuda")
-    aux = _aux_knee(rs, ctx, p, descs_d, params) if rank == 0 else None
+    aux = None
+    if rank == 0:
+        aux = _aux_knee(rs, ctx, p, descs_d, params)
+        if not args.no_aux:
+            aux["variants"] = _aux_variants(rs, p, descs_d)
     if rank != 0:
         if ws > 1:
             dist.destroy_process_group()
@@ -401,6 +449,8 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-aux", action="store_true",
+                    help="skip the per-variant timings reported under aux.variants")
     ap.add_argument("--n-req", type=int, default=None,
                     help="truncate every replica's trace (profiling of a small case)")
     args = ap.parse_args()
