@@ -83,14 +83,14 @@ def test_load_spike_static_and_adaptive():
             assert fs == -1.0
 
 
-def _full_launch(p, flags=0):
+def _full_launch(p, flags=0, **ctx_fields):
     """One simulate_replicas call over the whole plan (the benchmark's launch
     configuration); records stay on the device."""
     traces = p.traces()
-    ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
+    ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2, **ctx_fields)
     bufs = [rs.device_trace(t) for t in traces]
     rows = sum(r.n_req for r in p.replicas)
-    rec, t = rs.device_records(rows, p.W)
+    rec, t = rs.device_records(rows, p.W, with_kv=bool(ctx.cfg.tiered))
     res = rs.simulate_replicas(ctx.h, [b.desc() for b in bufs], rs.RS_MEM_DEVICE,
                                [rs.replica_params(r) for r in p.replicas], rec, flags)
     torch.cuda.synchronize()
@@ -152,4 +152,48 @@ def test_grid_full_size_sampled_replicas():
             assert res_k[f] == o["summary"][f], f
         _, _, _, tot = O.poa(cfg, o)
         assert abs(res_k["poa_total"] - tot) <= 1e-4 * tot
+    ctx.close()
+
+
+def _whole_equal(p, ctx, traces, res, t, base, k, extra=()):
+    cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
+    r = p.replicas[k]
+    o = oracle_run(cfg, traces[r.trace], r)
+    g = _rows(t, int(base[k]), r.n_req, p.W)
+    _prefix_equal(g, o, p.W)
+    res_k = res[k].as_dict()
+    for f in ("n_routed", "hit_blocks", "inserted_blocks", "evicted_blocks", "first_evict_t",
+              "rho_first_evict", "rho_end") + tuple(extra):
+        assert res_k[f] == o["summary"][f], (f, res_k[f], o["summary"][f])
+    return g, o
+
+
+def test_frequency_eviction_p2d_full_size():
+    # the p2d launch with every replica evicting by the frequency rule
+    p = wk.plan("p2d")
+    for r in p.replicas:
+        r.eviction, r.freq_max, r.decay_s = rs.RS_EVICT_FREQ, 64, 1.0
+    ctx, traces, res, t, base = _full_launch(p, flags=rs.RS_SIM_NO_POA)
+    assert all(r.status == 0 for r in res)
+    for k in (0, 37):
+        _whole_equal(p, ctx, traces, res, t, base, k)
+    assert sum(x.evicted_blocks for x in res) > 0
+    ctx.close()
+
+
+def test_game2_tiers_p2d_full_size():
+    # the p2d launch with G2 = 64K and G3 = 128K blocks per worker beside the
+    # 64K-block G1; the charge of every request compared
+    p = wk.plan("p2d")
+    ctx, traces, res, t, base = _full_launch(p, flags=rs.RS_SIM_NO_POA, tiered=1,
+                                             tier_k2=p.K, tier_k3=2 * p.K, tier_node=1)
+    assert all(r.status == 0 for r in res)
+    for k in (5, 63):
+        r = p.replicas[k]
+        g, o = _whole_equal(p, ctx, traces, res, t, base, k,
+                            extra=("kv_g1", "kv_g2", "kv_g3", "kv_remote", "kv_recompute",
+                                   "kv_cost"))
+        b0 = int(base[k])
+        assert np.array_equal(t["kv_cost"][b0:b0 + r.n_req].cpu().numpy(), o["kv_cost"])
+    assert sum(x.kv_g2 + x.kv_g3 for x in res) > 0
     ctx.close()
