@@ -587,6 +587,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   for (int base = 0; base < total; base += NT * PROBE_ILP) {   // uniform
     int jj[PROBE_ILP], kk[PROBE_ILP];
     uint64_t v[PROBE_ILP][BUCKET];
+    uint64_t stw[PROBE_ILP][TIER ? 4 : 1];   // tiers: the home bucket's 8 stamps, beside its keys
     uint32_t bk[PROBE_ILP];
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
@@ -599,6 +600,9 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
         const TableView t = c.table(j);
         bk[r] = home_bucket(hbuf[kk[r]], t.bmask);
         ld_bucket(t.keys, bk[r], v[r]);
+        if (TIER)   // one 32-byte sector: stamps are 4-byte, buckets of 8 start 32-byte aligned
+          ld_keys4(reinterpret_cast<const uint64_t*>(t.stamp + (size_t)BUCKET * bk[r]), stw[r][0],
+                   stw[r][TIER ? 1 : 0], stw[r][TIER ? 2 : 0], stw[r][TIER ? 3 : 0]);
       }
     }
 #pragma unroll
@@ -619,7 +623,17 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
         if (TIER) {
           int tier = 0;
           if (sl != SLOT_NONE) {
-            const uint32_t st = __ldcg(c.table(jj[r]).stamp + sl);
+            uint32_t st;
+            if (sl / BUCKET == bk[r]) {   // in the home bucket: its stamp came with the keys
+              const uint32_t q = sl % BUCKET;
+              const uint64_t w2 = q < 2 ? stw[r][0]
+                                        : (q < 4 ? stw[r][TIER ? 1 : 0]
+                                                 : (q < 6 ? stw[r][TIER ? 2 : 0]
+                                                          : stw[r][TIER ? 3 : 0]));
+              st = (uint32_t)(q & 1u ? w2 >> 32 : w2);
+            } else {
+              st = __ldcg(c.table(jj[r]).stamp + sl);
+            }
             const TierMeta tm = c.wtier[jj[r]];
             tier = st >= tm.b1 ? 1 : (st >= tm.b2 ? 2 : 3);
           }
