@@ -38,6 +38,7 @@ struct rs_ctx {
   // simulation scratch (grow-only)
   DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, dstat, wco, slots;
   DevBuf fexp, tmpe;   // frequency eviction state and its rebuild scratch
+  DevBuf dupf;         // per request: a chained hash repeats within the prompt
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -292,7 +293,7 @@ void route_destroy(rs_ctx* ctx) {
   DevBuf* all[] = {&ctx->r_keys, &ctx->r_stamp, &ctx->r_log, &ctx->r_tmp, &ctx->r_meta,
                    &ctx->r_active, &ctx->r_ord, &ctx->r_status, &ctx->r_hash, &ctx->r_stats,
                    &ctx->keys, &ctx->stamp, &ctx->log, &ctx->tmp, &ctx->pend, &ctx->meta_out,
-                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->slots, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
+                   &ctx->res, &ctx->desc, &ctx->hashes, &ctx->stats, &ctx->hjobs, &ctx->dupf, &ctx->slots, &ctx->dstat, &ctx->wco, &ctx->rec_worker,
                    &ctx->rec_arrival, &ctx->rec_start, &ctx->rec_first, &ctx->rec_completion,
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
@@ -601,7 +602,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   const bool host = trace_mem == RS_MEM_HOST;
   rs_status r;
   // ---- trace geometry; host traces are staged on the device
-  std::vector<int64_t> tot(n_traces, 0), hoff(n_traces, 0);
+  std::vector<int64_t> tot(n_traces, 0), hoff(n_traces, 0), rbase(n_traces, 0);
   std::vector<const int32_t*> dtok(n_traces);
   std::vector<const int64_t*> doff(n_traces);
   std::vector<const double*> drel(n_traces);
@@ -671,18 +672,18 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   int64_t launches = 0, hashed_tokens = 0;
   CK(cudaEventRecord(ctx->ev[0], ctx->st), "event");
   CK(cudaMemsetAsync(ctx->stats.p, 0, (size_t)n_traces * 8, ctx->st), "memset");
-  {
-    std::vector<HashJob> jobs;
-    int64_t rb = 0;
-    for (int t = 0; t < n_traces; t++) {
-      if (!used[t] || traces[t].n_req == 0) continue;
-      jobs.push_back(HashJob{dtok[t], doff[t], P<uint64_t>(ctx->hashes) + hoff[t], traces[t].n_req, rb});
-      rb += traces[t].n_req;
-      hashed_tokens += tot[t];
-    }
-    if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->stats))) != RS_OK) return r;
-    launches += ((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS;
+  std::vector<HashJob> jobs;
+  int64_t req_total = 0;
+  for (int t = 0; t < n_traces; t++) {
+    if (!used[t] || traces[t].n_req == 0) continue;
+    rbase[t] = req_total;
+    jobs.push_back(HashJob{dtok[t], doff[t], P<uint64_t>(ctx->hashes) + hoff[t], traces[t].n_req,
+                           req_total});
+    req_total += traces[t].n_req;
+    hashed_tokens += tot[t];
   }
+  if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->stats))) != RS_OK) return r;
+  launches += ((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS;
   CK(cudaEventRecord(ctx->ev[1], ctx->st), "event");
   CK(cudaMemcpyAsync(ctx->pinned, ctx->stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");
   CK(cudaStreamSynchronize(ctx->st), "sync");
@@ -718,6 +719,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
       (r = ensure(ctx, ctx->meta_out, nsim * W * sizeof(CacheMeta), "cache meta")) ||
       (r = ensure(ctx, ctx->res, nsim * sizeof(rs_replica_result), "results")) ||
       (r = ensure(ctx, ctx->desc, nsim * sizeof(SimDesc), "replica descriptors")) ||
+      (r = ensure(ctx, ctx->dupf, (size_t)std::max<int64_t>(req_total, 1), "duplicate flags")) ||
       (r = ensure(ctx, ctx->dstat, (size_t)std::max<int64_t>(rows, 1) * 6 * sizeof(float),
                   "decision statistics")))
     return r;
@@ -745,6 +747,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     d.release = drel[p.trace];
     d.out_len = dol[p.trace];
     d.hashes = P<uint64_t>(ctx->hashes) + hoff[p.trace];
+    d.dupflag = P<uint8_t>(ctx->dupf) + rbase[p.trace];
     d.n_req = p.n_req;
     d.rec_base = rb;
     d.C = p.C;
@@ -800,6 +803,16 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   L.mc.write_cost = want_cost ? 1 : 0;
   if (use_tab) {
     CK(launch_wco_table(P<double>(ctx->wco), (int)nbmax, ctx->cfg.w_c, ctx->st), "table launch");
+    launches++;
+  }
+  // per-request duplicate-hash flags, over the jobs as the hashing left them
+  for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
+    const int64_t base = jobs[g0].req_base;
+    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - base;
+    CK(launch_dup_flags(P<HashJob>(ctx->hjobs) + g0, (int)(g1 - g0), total, nbmax,
+                        P<uint8_t>(ctx->dupf) + base, ctx->st),
+       "duplicate flags launch");
     launches++;
   }
   CK(launch_sim(P<SimDesc>(ctx->desc), sb, L, ctx->st), "simulation launch");

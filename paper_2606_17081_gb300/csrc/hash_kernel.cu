@@ -11,6 +11,7 @@
 //  3. the lane stores mix(H_k ^ k); lane 31's H carries to the next chunk.
 // No serial chain per request remains: the pass streams tokens once (4 bytes
 // per token in) and hashes once (8 bytes per block out), the HBM floor.
+#include <algorithm>
 #include <climits>
 
 #include "rs_device.cuh"
@@ -140,6 +141,86 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
   int64_t nblk = (total_req + HASH_NT / 32 - 1) / (HASH_NT / 32);   // one warp per request
   if (nblk > (int64_t)sms * 16) nblk = (int64_t)sms * 16;
   k_block_hash<<<(unsigned)nblk, HASH_NT, 0, st>>>(jobs_dev, njobs, total_req, seed, nbmax_out);
+  return cudaGetLastError();
+}
+
+// Duplicate block hashes within one prompt (a 64-bit collision, which the
+// simulation reports as RS_ERR_COLLISION at that request): flags[r] = 1 when
+// two blocks of request r share a chained hash, else 0.  One warp per request,
+// each warp with an open-addressing set of cap entries in shared memory (cap a
+// power of two >= 2 nbmax; the set of a request uses the first power of two
+// >= 2 nb of them).  Hashes are >= 2, so 0 marks an empty entry.  Requests
+// longer than cap / 2 blocks are not checked: they are longer than the cache
+// and stop their replica for capacity before any update.
+__global__ void __launch_bounds__(256) k_dup_flags(const HashJob* __restrict__ jobs, int njobs,
+                                                   int64_t total_req, uint32_t cap,
+                                                   uint8_t* __restrict__ flags) {
+  extern __shared__ unsigned long long dset[];
+  __shared__ HashJob s_jobs[HASH_MAX_JOBS];
+  for (int j = threadIdx.x; j < njobs; j += blockDim.x) s_jobs[j] = jobs[j];
+  __syncthreads();
+  const int lane = threadIdx.x & 31, wpc = (int)(blockDim.x >> 5);
+  unsigned long long* set = dset + (size_t)(threadIdx.x >> 5) * cap;
+  const int64_t nw = (int64_t)gridDim.x * wpc;
+  for (int64_t r = (int64_t)blockIdx.x * wpc + (threadIdx.x >> 5); r < total_req; r += nw) {
+    const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
+    const int64_t i = r - J.req_base;
+    const int64_t o0 = __ldg(J.offsets + i);
+    const int64_t nb = (__ldg(J.offsets + i + 1) - o0) >> 4;
+    int dup = 0;
+    if (nb >= 2 && 2 * nb <= (int64_t)cap) {   // warp-uniform
+      uint32_t m = 2;
+      while (m < 2 * nb) m <<= 1;
+      const uint32_t mask = m - 1;
+      for (uint32_t e = lane; e < m; e += 32) set[e] = 0ull;
+      __syncwarp();
+      const uint64_t* h = J.out + (o0 >> 4);
+      for (int64_t k = lane; k < nb; k += 32) {
+        const unsigned long long x = __ldg(h + k);
+        uint32_t d = (uint32_t)(x ^ (x >> 29)) & mask;
+        for (uint32_t it = 0; it <= mask; it++) {
+          const unsigned long long prev = atomicCAS(set + d, 0ull, x);
+          if (prev == 0ull) break;
+          if (prev == x) {
+            dup = 1;
+            break;
+          }
+          d = (d + 1) & mask;
+        }
+      }
+      dup = __any_sync(FULL_MASK, dup);   // (every lane's claims are made before the next clear)
+    }
+    if (lane == 0) flags[r] = (uint8_t)dup;
+  }
+}
+
+cudaError_t launch_dup_flags(const HashJob* jobs_dev, int njobs, int64_t total_req, int64_t nbmax,
+                             uint8_t* flags, cudaStream_t st) {
+  if (total_req <= 0) return cudaSuccess;
+  if (njobs < 1 || njobs > HASH_MAX_JOBS || nbmax < 1) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0, maxsm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess)
+    e = cudaDeviceGetAttribute(&maxsm, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  uint32_t cap = 2;
+  while ((int64_t)cap < 2 * nbmax) cap <<= 1;
+  // dynamic shared memory beside the static job table: up to the default
+  // 48 KB per CTA without opting in, else one warp's set with the opt-in
+  const size_t per_warp = (size_t)cap * 8;
+  const size_t stat = sizeof(HashJob) * HASH_MAX_JOBS;
+  const size_t room = (size_t)maxsm - stat, dflt = 48 * 1024 - stat;
+  if (per_warp > room) return cudaErrorInvalidValue;
+  int wpc = (int)std::min<size_t>(8, std::max<size_t>(1, dflt / per_warp));
+  const size_t smem = per_warp * wpc;
+  if (smem > dflt) {
+    e = cudaFuncSetAttribute(k_dup_flags, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  int64_t nblk = (total_req + wpc - 1) / wpc;
+  if (nblk > (int64_t)sms * 16) nblk = (int64_t)sms * 16;
+  k_dup_flags<<<(unsigned)nblk, 32 * wpc, smem, st>>>(jobs_dev, njobs, total_req, cap, flags);
   return cudaGetLastError();
 }
 

@@ -34,9 +34,9 @@ constexpr int PROBE_ILP = 2;             // lookups a thread keeps in flight
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct SimLayout {
-  size_t ftab, wwco, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
+  size_t ftab, f_oitl, f_a, f_o, h_k, hbuf0, hbuf1, dupset, wA;
   size_t f_req, f_worker, f_blk, f_next, h_f, freestk, owner, victim;
-  size_t slot, pst, fslot, pslot, pfree, dclaim, vslot, vt;
+  size_t slot, pst, fslot, pslot, pfree, vslot, vt;
   size_t wmeta, wfreq, wtier, ptier, winserv, wqh, wqt, wm, wcost, wopen, wabs;
   size_t kind, evk, touched;
   size_t total;
@@ -72,7 +72,6 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
     TAKE(field, bytes, al)                          \
   }
   TAKE(ftab, 8 * (size_t)(nft > 0 ? nft : 1), 16)
-  TAKE(wwco, 8 * (size_t)W, 8)
   TAKES(f_oitl, 8 * C, 8)
   TAKES(f_a, 8 * C, 8)
   TAKES(f_o, 8 * C, 8)
@@ -94,7 +93,6 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(fslot, 4 * nb, 4)
   TAKE(pslot, 4 * (size_t)PROBE_CAP, 16)
   TAKE(pfree, 4 * (size_t)PROBE_CAP, 16)
-  TAKE(dclaim, 4 * nb, 4)
   TAKE(vslot, 4 * nv, 4)
   TAKE(vt, 4 * nv, 4)
   TAKE(wmeta, sizeof(CacheMeta) * (size_t)W, 16)
@@ -137,6 +135,7 @@ struct ReqState {
   double rel;      // client release time
   double twait;    // while waiting for a free client slot: the time reached
   int nb, nbt, O, phase, full;   // phase 0 new, 2 waiting for a slot, 1 arrival known
+  int dup;                       // two blocks of the prompt share a chained hash
   float tau, omega;
 };
 
@@ -144,7 +143,7 @@ struct ReqState {
 struct RawReq {
   int64_t o0, o1;
   double rel;
-  int O;
+  int O, dup;
 };
 
 struct SimScalars {
@@ -179,7 +178,7 @@ struct SimCtx {
   const SimBuffers* b;
   const SimLaunch* L;
   int sid;
-  double *f_a, *f_o, *ftab, *f_oitl, *wwco;
+  double *f_a, *f_o, *ftab, *f_oitl;
   uint64_t* h_k;
   uint64_t *hbuf0, *hbuf1;
   int32_t *f_req, *f_worker, *f_blk, *f_next, *h_f, *freestk;
@@ -187,7 +186,7 @@ struct SimCtx {
   FreqMeta* wfreq;
   TierMeta* wtier;    // Game 2 band boundaries per worker (tiered)
   uint8_t* ptier;     // [W][nb] tier of each (worker, block) pair, 0 = absent (tiered)
-  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs, *dclaim;
+  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs;
   uint32_t *pslot, *pfree;
   int64_t* wA;
   float* wcost;
@@ -878,8 +877,17 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
   }
 }
 
-// Request i's load, records and service start (control thread).
-__device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64_t i) {
+// w_c * o_ij of Eq. (9) for a cached prefix of m of the prompt's nbt blocks:
+// from the table of every (m, nbt) when there is one, else computed.
+__device__ __forceinline__ double wco_of(const SimCtx& c, int m, int nbt) {
+  if (c.b->wco_tab) return c.b->wco_tab[(size_t)m * c.b->wco_dim + nbt];
+  const double o = nbt > 0 ? __ddiv_rn((double)m, (double)nbt) : 0.0;
+  return __dmul_rn(c.L->mc.w_c, o);
+}
+
+// Request i's load, records and service start (control thread); wco: w_c *
+// o_ij of the chosen worker.
+__device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64_t i, double wco) {
   SimScalars& S = *c.S;
   const ModelConsts& mc = c.L->mc;
   const int js = S.jstar;
@@ -888,7 +896,7 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   c.f_worker[f] = js;
   c.f_blk[f] = (int32_t)q.blk;
   c.f_a[f] = q.a;
-  c.f_o[f] = c.wwco[js];
+  c.f_o[f] = wco;
   c.f_oitl[f] = q.oitl;
   c.wA[js] += q.blk;
   S.in_flight++;
@@ -907,12 +915,28 @@ __device__ __forceinline__ void book_request(SimCtx& c, const ReqState& q, int64
   S.n_routed++;
 }
 
+// Lowest-index argmin across a warp: each lane holds the minimum of its own
+// elements (cost c, index j; no element: +inf and INT_MAX); every lane ends
+// with the (cost, index) that is least in (cost, then index) order.
+__device__ __forceinline__ void argmin_warp(float& c, int& j) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float oc = __shfl_xor_sync(FULL_MASK, c, o);
+    const int oj = __shfl_xor_sync(FULL_MASK, j, o);
+    if (oc < c || (oc == c && oj < j)) {
+      c = oc;
+      j = oj;
+    }
+  }
+}
+
 __device__ __forceinline__ RawReq read_request(const SimCtx& c, int64_t i) {
   RawReq r;
   r.o0 = c.d->offsets[i];
   r.o1 = c.d->offsets[i + 1];
   r.rel = c.d->release[i];
   r.O = c.d->out_len[i];
+  r.dup = c.d->dupflag[i];
   return r;
 }
 
@@ -921,6 +945,7 @@ __device__ __forceinline__ void load_request(const SimCtx& c, ReqState& q, const
   q.off0 = r.o0;
   q.rel = r.rel;
   q.O = r.O;
+  q.dup = r.dup;
   q.oitl = __dmul_rn((double)r.O, c.L->mc.itl);
   q.nb = (L >> 4) > 0x7FFFFFFF ? 0x7FFFFFFF : (int)(L >> 4);
   q.nbt = (int)((L + 15) >> 4);
@@ -994,7 +1019,6 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.sid = sid;
   c.ftab = reinterpret_cast<double*>(smem + lay.ftab);
   c.f_oitl = reinterpret_cast<double*>(slotbase + lay.f_oitl);
-  c.wwco = reinterpret_cast<double*>(smem + lay.wwco);
   c.f_a = reinterpret_cast<double*>(slotbase + lay.f_a);
   c.f_o = reinterpret_cast<double*>(slotbase + lay.f_o);
   c.h_k = reinterpret_cast<uint64_t*>(slotbase + lay.h_k);
@@ -1023,7 +1047,6 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.sc.fslot = reinterpret_cast<uint32_t*>(smem + lay.fslot);
   c.pslot = reinterpret_cast<uint32_t*>(smem + lay.pslot);
   c.pfree = reinterpret_cast<uint32_t*>(smem + lay.pfree);
-  c.dclaim = reinterpret_cast<int32_t*>(smem + lay.dclaim);
   c.sc.kind = smem + lay.kind;
   c.sc.evk = smem + lay.evk;
   c.sc.vslot = reinterpret_cast<uint32_t*>(smem + lay.vslot);
@@ -1135,21 +1158,30 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
     if (warp == 0) {
       const float om = S.q[p].omega, tau = S.q[p].tau;
+      const bool eq2 = d.policy == RS_POLICY_DYNAMO || d.policy == RS_POLICY_LOADBAL;
+      // lane per worker; the lowest-index argmin (the choice at tau = 0) by a
+      // butterfly over (cost, index), no serial pass over shared memory
+      float bc = __int_as_float(0x7F800000);
+      int bj = 0x7FFFFFFF;
       for (int j = lane; j < W; j += 32) {
         const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
         c.wcost[j] = cj;
         b.rec.n_frozen[row * W + j] = (uint16_t)min(c.winserv[j] + 1, mc.cap - 1);
         b.rec.prefix[row * W + j] = (uint16_t)c.wm[j];
         if (mc.write_cost) b.rec.cost[row * W + j] = cj;
+        if (cj < bc || bj == 0x7FFFFFFF) {
+          bc = cj;
+          bj = j;
+        }
       }
+      argmin_warp(bc, bj);
       __syncwarp();
       if (lane == 0) {
-        const bool eq2 = d.policy == RS_POLICY_DYNAMO || d.policy == RS_POLICY_LOADBAL;
         const uint32_t u24 = eq2 && tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
         float* ds = b.dstat + row * 6;
-        const int js = eq2 ? select_worker(c.wcost, W, tau, u24, ds + 2)
-                           : static_policy_worker(d.policy, c.wcost, W, d.seed, (uint64_t)i, 0u,
-                                                  TAG_SIM);
+        const int js = !eq2 ? static_policy_worker(d.policy, c.wcost, W, d.seed, (uint64_t)i, 0u,
+                                                   TAG_SIM)
+                            : (tau == 0.0f ? bj : select_worker(c.wcost, W, tau, u24, ds + 2));
         S.jstar = js;
         S.hit_blocks += c.wm[js];
         if (FREQ && d.eviction == RS_EVICT_FREQ) {   // decay step of this request's arrival
@@ -1159,6 +1191,9 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         // the chosen worker's absent blocks, latched before the control warp
         // resets the probe state for the next request
         S.nabs = c.wabs[js];
+        // two blocks of the prompt with one chained hash (a 64-bit collision,
+        // flagged per request before the launch) would break the batched update
+        if (S.q[p].dup) S.us.dup = 1;
         // the chosen worker's table: rebuild first when its log span, its
         // tombstones or its stamps would overflow
         const CacheMeta* mt = &c.wmeta[js];
@@ -1167,50 +1202,42 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         if (eq2 && tau > 0.0f) S.sampled++;
         else ds[3] = -1.0f;   // no Eq. (2) draw
       }
-    } else if (warp == 1 && lane == 0) {
+    } else if (warp == 1) {
       // statistics of the decision, beside the choice: work done by the probe
-      int64_t pb = 0;
-      for (int j = 0; j < W; j++) pb += min(c.wm[j] + 1, nb);
-      S.probe_blocks += pb;
-      S.hashed_blocks += nb;
-      // the two lowest Eq. (1) costs, for the near-tie statistic (counted
+      // and the two lowest Eq. (1) costs, for the near-tie statistic (counted
       // after the run); recomputed from the probe results so as not to wait
       // for warp 0
       const float om = S.q[p].omega;
-      float c1 = router_cost(om, (int64_t)nbt - c.wm[0], c.wA[0]);
-      int bmin = 0;
-      for (int j = 1; j < W; j++) {
-        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
-        if (cj < c1) { c1 = cj; bmin = j; }
+      int pb = 0;
+      float c1 = __int_as_float(0x7F800000);
+      int bmin = 0x7FFFFFFF;
+      for (int j = lane; j < W; j += 32) {
+        const int m = c.wm[j];
+        pb += min(m + 1, nb);
+        const float cj = router_cost(om, (int64_t)nbt - m, c.wA[j]);
+        if (cj < c1 || bmin == 0x7FFFFFFF) {
+          c1 = cj;
+          bmin = j;
+        }
       }
+      argmin_warp(c1, bmin);
       float c2 = __int_as_float(0x7F800000);
-      for (int j = 0; j < W; j++) {
+      for (int j = lane; j < W; j += 32) {
         const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
         if (j != bmin && cj < c2) c2 = cj;
       }
-      b.dstat[row * 6] = c1;
-      b.dstat[row * 6 + 1] = c2;
-    } else if (warp == NT_SIM / 32 - 1) {
-      // w_c * o_ij for every worker (the chosen one's enters its latency)
-      for (int j = lane; j < W; j += 32) {
-        double w;
-        if (b.wco_tab) {
-          w = b.wco_tab[(size_t)c.wm[j] * b.wco_dim + nbt];
-        } else {
-          const double o = nbt > 0 ? __ddiv_rn((double)c.wm[j], (double)nbt) : 0.0;
-          w = __dmul_rn(mc.w_c, o);
-        }
-        c.wwco[j] = w;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float x = __shfl_xor_sync(FULL_MASK, c2, o);
+        if (x < c2) c2 = x;
       }
-    } else if (warp >= 2 && warp < NT_SIM / 32 - 1) {
-      // two blocks of one prompt with the same chained hash (a 64-bit
-      // collision) would break the batched update: detect them here
-      int dup = 0;
-      for (int k = threadIdx.x - 64; k < nb; k += NT_SIM - 96) c.dclaim[k] = dup_claim(c.sc, hb[k], &dup);
-      if (dup) S.us.dup = 1;
-      asm volatile("bar.sync 2, %0;" ::"n"(NT_SIM - 96) : "memory");   // warps 2-6: all claims made
-      for (int k = threadIdx.x - 64; k < nb; k += NT_SIM - 96)
-        if (c.dclaim[k] >= 0) c.sc.dupset[c.dclaim[k]] = 0ull;
+      pb = (int)__reduce_add_sync(FULL_MASK, (unsigned)pb);
+      if (lane == 0) {
+        S.probe_blocks += pb;
+        S.hashed_blocks += nb;
+        b.dstat[row * 6] = c1;
+        b.dstat[row * 6 + 1] = c2;
+      }
     }
     __syncthreads();
     const int js = S.jstar;
@@ -1223,6 +1250,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       // scalars, probe state and block hashes
       ReqState& nq = S.q[p ^ 1];
       const bool more = i + 1 < n;
+      // the chosen worker's w_c * o (a table load): issued first, used last
+      const double wco = lane == 0 ? wco_of(c, c.wm[js], nbt) : 0.0;
       if (more) {
         // request i+1's hashes: asynchronous copies into the other staging
         // buffer, waited for before the next barrier
@@ -1242,7 +1271,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         RawReq raw2;
         const bool more2 = i + 2 < n;
         if (more2) raw2 = read_request(c, i + 2);
-        book_request(c, S.q[p], i);
+        book_request(c, S.q[p], i, wco);
         if (more2) S.nraw = raw2;
       }
       cp_async_wait_all();
