@@ -265,6 +265,11 @@ __device__ __forceinline__ uint32_t home_bucket(uint64_t h, uint32_t bmask) {
   return (uint32_t)(h ^ (h >> 32)) & bmask;
 }
 
+// Brings the line holding p into L2 (no register result, no wait).
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // Four keys (one 32-byte sector) in one 256-bit load through L2; p 32-byte
 // aligned (buckets are 64-byte aligned: the key arrays start on 256-byte
 // boundaries and every table holds a multiple of 8 slots).

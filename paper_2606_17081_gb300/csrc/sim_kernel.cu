@@ -1275,6 +1275,22 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         if (more2) S.nraw = raw2;
       }
       cp_async_wait_all();
+      __syncwarp();   // every lane's copies of request i+1's hashes have landed
+      if (more && nq.full && nq.nb <= (int)L.g.K) {
+        // request i+1's home buckets on every worker, brought into L2 ahead
+        // of its probe (the update running beside may still change the
+        // chosen worker's; L2 holds the current data either way)
+        const uint64_t* hn = c.hbuf(p ^ 1);
+        const int nbn = nq.nb;
+        for (int e = lane; e < W * nbn; e += 32) {
+          const int j = e / nbn;
+          const TableView t = c.table(j);
+          const uint32_t bk = home_bucket(hn[e - j * nbn], t.bmask);
+          prefetch_l2(t.keys + (size_t)BUCKET * bk);
+          prefetch_l2(t.keys + (size_t)BUCKET * bk + 4);
+          if (TIER) prefetch_l2(t.stamp + (size_t)BUCKET * bk);
+        }
+      }
     }
   }
   __syncthreads();
