@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 31867643904 + 6049586176,
-               "sources_sha256": "c869db5275deec6679a07155f87cb2527195393738a349a3efbea28c6d2ab4e6",
+SIM_TRAFFIC = {"bytes": 31925586176 + 6057666560,
+               "sources_sha256": "9ca7896549824415266a475477cda923422662e1838659771e929837a612e3ed",
                "summary": "profiles/k_sim_p2d.md"}
 
 
