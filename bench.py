@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 31925586176 + 6057666560,
-               "sources_sha256": "9ca7896549824415266a475477cda923422662e1838659771e929837a612e3ed",
+SIM_TRAFFIC = {"bytes": 31939619072 + 6058769920,
+               "sources_sha256": "f8f12049d59ffef7514cf0b17ef8f1cb587de4fa2b7fb240d9fb93dc0e1fce03",
                "summary": "profiles/k_sim_p2d.md"}
 
 

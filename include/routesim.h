@@ -151,6 +151,21 @@ const char* route_last_error(const rs_ctx* ctx);
 rs_status route_hash_blocks(rs_ctx* ctx, const int32_t* tokens_dev, const int64_t* offsets_dev,
                             int64_t n_req, uint64_t* hashes_dev);
 
+/* Repeated block hashes within a prompt.  A cache keyed by block hash (§2.2)
+ * cannot tell apart two blocks of one prompt whose chained hashes are equal
+ * (a 64-bit collision); simulate_replicas stops a replica at such a request
+ * with RS_ERR_COLLISION, using these flags.  For each request i:
+ *   flags_dev[i] = 1  two of its floor(L_i/16) block hashes are equal,
+ *                  0  all are distinct (or it has fewer than two blocks),
+ *                  2  it has more than max_blocks blocks (not checked).
+ * hashes_dev/offsets_dev: the layout route_hash_blocks writes (request i's
+ * k-th hash at floor(offsets[i]/16) + k; every hash >= 2, as that entry
+ * produces).  flags_dev: uint8 [n_req], caller-owned.  max_blocks in
+ * [1, 8192] (one shared-memory set of 2^ceil(log2(2 max_blocks)) hashes per
+ * warp), else RS_ERR_INVALID.  Asynchronous on the context stream. */
+rs_status route_dup_flags(rs_ctx* ctx, const uint64_t* hashes_dev, const int64_t* offsets_dev,
+                          int64_t n_req, int64_t max_blocks, uint8_t* flags_dev);
+
 /* Live routing (Algorithm 1 without the controller): routes n_req requests of
  * one router instance in array order, exactly as n_req calls of size one.
  * For each request: Eq. (1) cost with cfg.omega, the instance's active blocks

@@ -324,6 +324,25 @@ rs_status route_hash_blocks(rs_ctx* ctx, const int32_t* tokens_dev, const int64_
   return hash_jobs(ctx, jobs, nullptr);
 }
 
+rs_status route_dup_flags(rs_ctx* ctx, const uint64_t* hashes_dev, const int64_t* offsets_dev,
+                          int64_t n_req, int64_t max_blocks, uint8_t* flags_dev) {
+  if (!ctx) return fail(nullptr, RS_ERR_INVALID, "ctx is NULL");
+  ctx->err.clear();
+  if (n_req < 0) return fail(ctx, RS_ERR_INVALID, "n_req < 0");
+  if (max_blocks < 1 || max_blocks > 8192)
+    return fail(ctx, RS_ERR_INVALID, "max_blocks must be in [1, 8192]");
+  if (n_req == 0) return RS_OK;
+  if (!hashes_dev || !offsets_dev || !flags_dev) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
+  HashJob job{nullptr, offsets_dev, const_cast<uint64_t*>(hashes_dev), n_req, 0};
+  rs_status r = ensure(ctx, ctx->hjobs, sizeof(HashJob), "hash jobs");
+  if (r != RS_OK) return r;
+  CK(cudaMemcpyAsync(ctx->hjobs.p, &job, sizeof(HashJob), cudaMemcpyHostToDevice, ctx->st),
+     "copy hash job");
+  CK(launch_dup_flags(P<HashJob>(ctx->hjobs), 1, n_req, max_blocks, flags_dev, ctx->st),
+     "duplicate flags launch");
+  return RS_OK;   // (a copy from pageable memory has read its source when it returns)
+}
+
 // Hashes every job (trace) in launches of up to HASH_MAX_JOBS traces.
 static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbmax_dev) {
   if (jobs.empty()) return RS_OK;

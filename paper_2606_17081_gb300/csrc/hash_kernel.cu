@@ -146,14 +146,15 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
 
 // Duplicate block hashes within one prompt (a 64-bit collision, which the
 // simulation reports as RS_ERR_COLLISION at that request): flags[r] = 1 when
-// two blocks of request r share a chained hash, else 0.  One warp per request,
-// each warp with an open-addressing set of cap entries in shared memory (cap a
-// power of two >= 2 nbmax; the set of a request uses the first power of two
-// >= 2 nb of them).  Hashes are >= 2, so 0 marks an empty entry.  Requests
-// longer than cap / 2 blocks are not checked: they are longer than the cache
-// and stop their replica for capacity before any update.
+// two blocks of request r share a chained hash, 0 when none do, 2 when the
+// request has more than nbmax blocks (not checked; in the simulation such a
+// prompt is longer than the cache and stops its replica for capacity before
+// any update).  One warp per request, each warp with an open-addressing set
+// of cap entries in shared memory (cap a power of two >= 2 nbmax; the set of
+// a request uses the first power of two >= 2 nb of them).  Hashes are >= 2,
+// so 0 marks an empty entry.
 __global__ void __launch_bounds__(256) k_dup_flags(const HashJob* __restrict__ jobs, int njobs,
-                                                   int64_t total_req, uint32_t cap,
+                                                   int64_t total_req, int64_t nbmax, uint32_t cap,
                                                    uint8_t* __restrict__ flags) {
   extern __shared__ unsigned long long dset[];
   __shared__ HashJob s_jobs[HASH_MAX_JOBS];
@@ -167,8 +168,8 @@ __global__ void __launch_bounds__(256) k_dup_flags(const HashJob* __restrict__ j
     const int64_t i = r - J.req_base;
     const int64_t o0 = __ldg(J.offsets + i);
     const int64_t nb = (__ldg(J.offsets + i + 1) - o0) >> 4;
-    int dup = 0;
-    if (nb >= 2 && 2 * nb <= (int64_t)cap) {   // warp-uniform
+    int dup = nb > nbmax ? 2 : 0;
+    if (nb >= 2 && nb <= nbmax) {   // warp-uniform (2 nb <= cap)
       uint32_t m = 2;
       while (m < 2 * nb) m <<= 1;
       const uint32_t mask = m - 1;
@@ -220,7 +221,8 @@ cudaError_t launch_dup_flags(const HashJob* jobs_dev, int njobs, int64_t total_r
   }
   int64_t nblk = (total_req + wpc - 1) / wpc;
   if (nblk > (int64_t)sms * 16) nblk = (int64_t)sms * 16;
-  k_dup_flags<<<(unsigned)nblk, 32 * wpc, smem, st>>>(jobs_dev, njobs, total_req, cap, flags);
+  k_dup_flags<<<(unsigned)nblk, 32 * wpc, smem, st>>>(jobs_dev, njobs, total_req, nbmax, cap,
+                                                     flags);
   return cudaGetLastError();
 }
 

@@ -62,7 +62,7 @@ struct SimDesc {
   const double* release;
   const int32_t* out_len;
   const uint64_t* hashes;   // block hashes of the replica's trace
-  const uint8_t* dupflag;   // per request: two blocks share a chained hash
+  const uint8_t* dupflag;   // per request: 1 when two blocks share a chained hash
   int64_t n_req;
   int64_t rec_base;         // first record row
   int32_t C, policy, controller, eviction;   // eviction: RS_EVICT_*
@@ -130,7 +130,9 @@ constexpr int HASH_MAX_JOBS = 64;
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
                               int64_t* nbmax_out, cudaStream_t st);
 // flags[r] = 1 when two blocks of request r (numbered over the launch's jobs)
-// share a chained hash; requests of more than nbmax blocks are not checked.
+// share a chained hash, 0 when none do, 2 when it has more than nbmax blocks
+// (not checked).  Fails with cudaErrorInvalidValue when one warp's set of
+// 2^ceil(log2(2 nbmax)) hashes does not fit in shared memory.
 cudaError_t launch_dup_flags(const HashJob* jobs_dev, int njobs, int64_t total_req, int64_t nbmax,
                              uint8_t* flags, cudaStream_t st);
 cudaError_t launch_sim(const SimDesc* d_desc, const SimBuffers& b, const SimLaunch& L,

@@ -936,7 +936,7 @@ __device__ __forceinline__ RawReq read_request(const SimCtx& c, int64_t i) {
   r.o1 = c.d->offsets[i + 1];
   r.rel = c.d->release[i];
   r.O = c.d->out_len[i];
-  r.dup = c.d->dupflag[i];
+  r.dup = c.d->dupflag[i] == 1;
   return r;
 }
 
