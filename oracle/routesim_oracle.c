@@ -1539,6 +1539,30 @@ int32_t orc_router_route(orc_router* r, int32_t inst, const int32_t* tokens,
   return status;
 }
 
+/* Every request's cached prefix m_ij on every worker of an instance, against
+ * the caches as they stand: the leading full blocks found (S2, the b^prefill
+ * of Eq. (1)), with no cache or load touched, so that every request sees the
+ * same snapshot. */
+int32_t orc_router_probe(orc_router* r, int32_t inst, const int32_t* tokens,
+                         const int64_t* offsets, int64_t n_req, int32_t* prefix) {
+  if (!r || inst < 0 || inst >= r->ni || n_req < 0) return ORC_ERR_INVALID;
+  const int32_t W = r->cfg.W, B = r->cfg.block;
+  const lru_t* cache = r->cache + (int64_t)inst * W;
+  int64_t nbmax = 1;
+  for (int64_t i = 0; i < n_req; i++) {
+    int64_t nb = (offsets[i + 1] - offsets[i]) / B;
+    if (nb > nbmax) nbmax = nb;
+  }
+  uint64_t* h = (uint64_t*)malloc(sizeof(uint64_t) * nbmax);
+  for (int64_t i = 0; i < n_req; i++) {
+    const int64_t nb = (offsets[i + 1] - offsets[i]) / B;
+    hash_request(tokens + offsets[i], nb, B, r->cfg.hash_seed, h);
+    for (int32_t j = 0; j < W; j++) prefix[i * W + j] = (int32_t)cached_prefix(&cache[j], h, nb);
+  }
+  free(h);
+  return ORC_OK;
+}
+
 int32_t orc_router_release(orc_router* r, int32_t inst, const int32_t* worker,
                            const int32_t* blocks, int64_t n) {
   if (!r || inst < 0 || inst >= r->ni) return ORC_ERR_INVALID;

@@ -217,6 +217,10 @@ void orc_router_free(orc_router* r);
 int32_t orc_router_route(orc_router* r, int32_t instance, const int32_t* tokens,
                          const int64_t* offsets, int64_t n_req, const int32_t* out_len,
                          int32_t* worker, float* cost, int32_t* prefix);
+/* route_probe: m_ij of every request on every worker against the current
+ * caches, nothing updated; prefix [n_req * W]. */
+int32_t orc_router_probe(orc_router* r, int32_t instance, const int32_t* tokens,
+                         const int64_t* offsets, int64_t n_req, int32_t* prefix);
 int32_t orc_router_release(orc_router* r, int32_t instance, const int32_t* worker,
                            const int32_t* blocks, int64_t n);
 int32_t orc_router_active(orc_router* r, int32_t instance, int64_t* active /* [W] */);

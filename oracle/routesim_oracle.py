@@ -154,6 +154,7 @@ def lib():
         L.orc_router_free.argtypes = [C.c_void_p]
         L.orc_router_route.restype = C.c_int32
         L.orc_router_release.restype = C.c_int32
+        L.orc_router_probe.restype = C.c_int32
         L.orc_router_active.restype = C.c_int32
         L.orc_router_cache.restype = C.c_int32
     return _lib
@@ -366,6 +367,18 @@ class Router:
         st = lib().orc_router_route(C.c_void_p(self.h), C.c_int32(instance), _p(t), _p(o),
                                     C.c_int64(n), _p(ol), _p(wk), _p(cost), _p(pre))
         return st, wk[:n], cost[: n * W].reshape(n, W), pre[: n * W].reshape(n, W)
+
+    def probe(self, instance, tokens, offsets):
+        """m_ij of every request on every worker against the current caches
+        (nothing updated): (status, int32 [n, W])."""
+        t = _c(tokens, np.int32)
+        o = _c(offsets, np.int64)
+        n = o.size - 1
+        W = self.cfg.W
+        pre = np.zeros(max(n, 1) * W, np.int32)
+        st = lib().orc_router_probe(C.c_void_p(self.h), C.c_int32(instance), _p(t), _p(o),
+                                    C.c_int64(n), _p(pre))
+        return st, pre[: n * W].reshape(n, W)
 
     def release(self, instance, worker, blocks):
         w = _c(worker, np.int32)
