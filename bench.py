@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 31939619072 + 6058769920,
-               "sources_sha256": "f8f12049d59ffef7514cf0b17ef8f1cb587de4fa2b7fb240d9fb93dc0e1fce03",
+SIM_TRAFFIC = {"bytes": 31917070848 + 6057946624,
+               "sources_sha256": "dabbdc910f9daa14357965934473d558647f8f8cfb212b8096cd6b4bfa2d1966",
                "summary": "profiles/k_sim_p2d.md"}
 
 
@@ -242,6 +242,48 @@ def _aux_variants(rs, p, descs, reps: int = 2) -> dict:
     return out
 
 
+def _aux_probe(rs, d, n: int, reps: int = 5) -> dict:
+    """Outside the timed steps: the batch probe (route_probe: S2's cached
+    prefix for many requests against one cache snapshot) on a router instance
+    of 64 workers with 65536-block caches.  The first 2000 requests (at most
+    half) of a p2d trace are routed (route_batch), then the others are probed.  The
+    call hashes the batch, then probes; its kernel time is the call's device
+    time (CUDA events) less a block-hash call on the same batch.  probes =
+    sum over (request, worker) of min(m_ij + 1, nb_i) table lookups."""
+    import torch
+    W, K, nr = 64, 65536, min(2000, n // 2)
+    if n - nr <= 0:
+        return {}
+    ctx = rs.Context(W=W, K=K, n_instances=1)
+    wo = torch.zeros(nr, dtype=torch.int32, device="cuda")
+    rs.route_batch(ctx.h, 0, d.tokens, d.offsets, nr, d.out_len, wo)
+    m = n - nr
+    offs = d.offsets[nr:]
+    po = torch.zeros(m * W, dtype=torch.int32, device="cuda")
+    hs = torch.zeros(int(offs[-1].item()) // 16 + 1, dtype=torch.int64, device="cuda")
+    rs.route_probe(ctx.h, 0, d.tokens, offs, m, po)
+    tp, th = [], []
+    for _ in range(reps):
+        e0, e1, e2 = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e0.record()
+        rs.route_probe(ctx.h, 0, d.tokens, offs, m, po)
+        e1.record()
+        rs.route_hash_blocks(ctx.h, d.tokens, offs, m, hs)
+        e2.record()
+        torch.cuda.synchronize()
+        tp.append(e0.elapsed_time(e1))
+        th.append(e1.elapsed_time(e2))
+    ctx.close()
+    pre = po.cpu().numpy().reshape(m, W).astype(np.int64)
+    nb = (np.diff(offs.cpu().numpy()) // 16)[:, None]
+    probes = int(np.minimum(pre + 1, nb).sum())
+    kern = min(tp) - min(th)
+    return {"workers": W, "cache_blocks": K, "routed": nr, "probed": m, "pairs": m * W,
+            "probes": probes, "mean_prefix": float(pre.mean()), "call_ms": min(tp),
+            "hash_ms": min(th), "kernel_ms": kern, "probes_per_s": probes / (kern / 1e3),
+            "bucket_bytes_per_s": 64 * probes / (kern / 1e3)}
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -315,6 +357,7 @@ def run_gpu(args):
         aux = _aux_knee(rs, ctx, p, descs_d, params)
         if not args.no_aux:
             aux["variants"] = _aux_variants(rs, p, descs_d)
+            aux["probe_batch"] = _aux_probe(rs, dev[0], traces[0].n_req)
     if rank != 0:
         if ws > 1:
             dist.destroy_process_group()
@@ -450,7 +493,7 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-aux", action="store_true",
-                    help="skip the per-variant timings reported under aux.variants")
+                    help="skip the timings reported under aux.variants and aux.probe_batch")
     ap.add_argument("--n-req", type=int, default=None,
                     help="truncate every replica's trace (profiling of a small case)")
     args = ap.parse_args()

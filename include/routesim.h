@@ -181,6 +181,18 @@ rs_status route_batch(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
                       const int64_t* offsets_dev, int32_t n_req, const int32_t* out_len_dev,
                       int32_t* worker_out_dev, float* cost_out_dev, int32_t* prefix_out_dev);
 
+/* Cached prefixes of a batch against one router instance, read-only (§2.2, the
+ * b^prefill input of Eq. (1), for many requests at once): prefix_out_dev[i*W
+ * + j] = m_ij, the leading full blocks of request i found in worker j's
+ * cache.  Every request sees the same snapshot -- no cache, load or ordinal
+ * changes -- so a row equals the prefix_out row route_batch would report for
+ * that request if it were routed next.  Prompts longer than the cache are
+ * probed too (m_ij <= cache_blocks).  tokens_dev/offsets_dev as in
+ * route_hash_blocks; prefix_out_dev int32 [n_req*W], caller-owned.  Reads
+ * offsets_dev[n_req] (a synchronising copy), then asynchronous. */
+rs_status route_probe(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
+                      const int64_t* offsets_dev, int64_t n_req, int32_t* prefix_out_dev);
+
 /* Completion of n requests of an instance: active blocks of worker_dev[i]
  * drop by blocks_dev[i] (int32 each); a counter never goes below zero.
  * Entries with a worker outside [0, W) are skipped and the call returns

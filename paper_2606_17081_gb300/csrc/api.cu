@@ -430,6 +430,35 @@ rs_status route_batch(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
   return RS_OK;
 }
 
+rs_status route_probe(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
+                      const int64_t* offsets_dev, int64_t n_req, int32_t* prefix_out_dev) {
+  if (!ctx) return fail(nullptr, RS_ERR_INVALID, "ctx is NULL");
+  ctx->err.clear();
+  RouterState s;
+  rs_status r = router_state(ctx, instance, &s);
+  if (r != RS_OK) return r;
+  if (n_req < 0) return fail(ctx, RS_ERR_INVALID, "n_req < 0");
+  if (n_req == 0) return RS_OK;
+  if (!tokens_dev || !offsets_dev || !prefix_out_dev) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
+  if (!aligned16(tokens_dev)) return fail(ctx, RS_ERR_INVALID, "tokens must be 16-byte aligned");
+  if ((r = ensure_pinned(ctx, 4)) != RS_OK) return r;
+  CK(cudaMemcpyAsync(ctx->pinned, offsets_dev + n_req, 8, cudaMemcpyDeviceToHost, ctx->st),
+     "read offsets");
+  CK(cudaStreamSynchronize(ctx->st), "sync");
+  const int64_t total = ctx->pinned[0];
+  if (total < 0) return fail(ctx, RS_ERR_INVALID, "offsets[n_req] < 0");
+  if ((r = ensure(ctx, ctx->r_hash, (size_t)(total / 16 + 1) * 8, "batch hashes")) != RS_OK) return r;
+  {
+    std::vector<HashJob> jobs(1);
+    jobs[0] = HashJob{tokens_dev, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, 0};
+    if ((r = hash_jobs(ctx, jobs, nullptr)) != RS_OK) return r;
+  }
+  CK(launch_probe_batch(s, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, ctx->cfg.W, ctx->g,
+                        prefix_out_dev, ctx->st),
+     "probe launch");
+  return RS_OK;
+}
+
 static rs_status router_sync_status(rs_ctx* ctx, int32_t instance, int* bad) {
   rs_status r = ensure_pinned(ctx, 4);
   if (r != RS_OK) return r;

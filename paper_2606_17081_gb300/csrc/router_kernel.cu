@@ -236,4 +236,52 @@ cudaError_t launch_clear_tables(uint64_t* keys, uint32_t* stamp, size_t nslots, 
   return cudaGetLastError();
 }
 
+// Batch probe (route_probe): one thread per (request, worker) pair walks the
+// request's blocks in order through the worker's table until the first one
+// absent: m_ij + 1 bucket reads (64 bytes each, two 32-byte sectors) and
+// m_ij + 1 hash reads, the first-miss prefix of S2.  The tables are only
+// read, so all pairs run at once; pairs are numbered request-major, so the
+// threads of a warp share requests' offsets and hash lines.
+__global__ void __launch_bounds__(256) k_probe_batch(RouterState s,
+                                                     const int64_t* __restrict__ offsets,
+                                                     const uint64_t* __restrict__ hashes,
+                                                     int64_t n_req, int W, TableGeom g,
+                                                     int32_t* __restrict__ prefix_out) {
+  const int64_t total = n_req * W;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += stride) {
+    const int64_t i = e / W;
+    const int j = (int)(e - i * W);
+    const int64_t o0 = __ldg(offsets + i);
+    const int64_t nb = (__ldg(offsets + i + 1) - o0) >> 4;
+    const uint64_t* h = hashes + (o0 >> 4);
+    TableView t;
+    t.keys = s.keys + (size_t)j * g.slots;
+    t.stamp = s.stamp + (size_t)j * g.slots;
+    t.log = s.log + (size_t)j * g.R;
+    t.fexp = nullptr;
+    t.bmask = g.bmask;
+    t.rmask = g.rmask;
+    int64_t m = 0;
+    int err = 0;
+    while (m < nb && table_find(t, __ldg(h + m), &err) != SLOT_NONE) m++;
+    prefix_out[e] = (int32_t)(m < 0x7FFFFFFF ? m : 0x7FFFFFFF);
+  }
+}
+
+cudaError_t launch_probe_batch(const RouterState& s, const int64_t* offsets, const uint64_t* hashes,
+                               int64_t n_req, int W, const TableGeom& g, int32_t* prefix_out,
+                               cudaStream_t st) {
+  if (n_req <= 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int64_t total = n_req * W;
+  int64_t nblk = (total + 255) / 256;
+  if (nblk > (int64_t)sms * 8) nblk = (int64_t)sms * 8;   // 8 x 256 threads resident per SM
+  k_probe_batch<<<(unsigned)nblk, 256, 0, st>>>(s, offsets, hashes, n_req, W, g, prefix_out);
+  return cudaGetLastError();
+}
+
 }  // namespace rs

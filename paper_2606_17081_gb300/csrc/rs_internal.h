@@ -189,6 +189,11 @@ struct RouterState {
   int32_t* status;          // [1] sticky device error
 };
 
+// m_ij of n_req requests (hashes in the route_hash_blocks layout) on every
+// worker of one router instance, read-only; prefix_out [n_req * W].
+cudaError_t launch_probe_batch(const RouterState& s, const int64_t* offsets, const uint64_t* hashes,
+                               int64_t n_req, int W, const TableGeom& g, int32_t* prefix_out,
+                               cudaStream_t st);
 cudaError_t launch_route_batch(const RouterState& s, int32_t instance, const int64_t* offsets,
                                const uint64_t* hashes, int32_t n_req, const int32_t* out_len,
                                int32_t* worker_out, float* cost_out, int32_t* prefix_out,

@@ -89,7 +89,7 @@ class rs_timing(C.Structure):
 
 
 EXPORTS = ["rs_config_default", "route_init", "route_destroy", "route_last_error",
-           "route_hash_blocks", "route_dup_flags", "route_batch", "route_release", "route_active",
+           "route_hash_blocks", "route_dup_flags", "route_batch", "route_probe", "route_release", "route_active",
            "simulate_replicas", "poa_estimate", "route_cache_dump", "route_last_timing",
            "poa_estimate_noalloc", "sweep_knee"]
 
@@ -119,6 +119,7 @@ def lib():
             "route_hash_blocks": (i32, [vp, vp, vp, i64, vp]),
             "route_dup_flags": (i32, [vp, vp, vp, i64, i64, vp]),
             "route_batch": (i32, [vp, i32, vp, vp, i32, vp, vp, vp, vp]),
+            "route_probe": (i32, [vp, i32, vp, vp, i64, vp]),
             "route_release": (i32, [vp, i32, vp, vp, i32]),
             "route_active": (i32, [vp, i32, vp]),
             "simulate_replicas": (i32, [vp, C.POINTER(rs_trace), i32, i32,
@@ -189,6 +190,11 @@ def route_hash_blocks(ctx, tokens, offsets, n_req: int, hashes) -> None:
 def route_dup_flags(ctx, hashes, offsets, n_req: int, max_blocks: int, flags) -> None:
     _check(lib().route_dup_flags(ctx, _ptr(hashes), _ptr(offsets), n_req, max_blocks,
                                  _ptr(flags)), ctx)
+
+
+def route_probe(ctx, instance: int, tokens, offsets, n_req: int, prefix_out) -> None:
+    _check(lib().route_probe(ctx, instance, _ptr(tokens), _ptr(offsets), n_req,
+                             _ptr(prefix_out)), ctx)
 
 
 def route_batch(ctx, instance: int, tokens, offsets, n_req: int, out_len, worker_out,
