@@ -197,3 +197,29 @@ def test_game2_tiers_p2d_full_size():
         assert np.array_equal(t["kv_cost"][b0:b0 + r.n_req].cpu().numpy(), o["kv_cost"])
     assert sum(x.kv_g2 + x.kv_g3 for x in res) > 0
     ctx.close()
+
+
+def test_probe_batch_in_the_bench_configuration():
+    # the batch probe as aux.probe_batch runs it: a 64-worker router instance
+    # of 65 536-block caches, the first 2 000 requests of p2d trace 0 routed,
+    # the other 18 000 probed; every (request, worker) prefix bit-exact
+    p = wk.plan("p2d")
+    tr = p.traces()[0]
+    W, K, nr = 64, 65536, 2000
+    ctx = rs.Context(W=W, K=K, n_instances=1)
+    ref = O.Router(O.OracleConfig(W=W, K=K), 1.0, 0.0, 0)
+    d = rs.device_trace(tr)
+    wo = torch.zeros(nr, dtype=torch.int32, device="cuda")
+    rs.route_batch(ctx.h, 0, d.tokens, d.offsets, nr, d.out_len, wo)
+    head = wk.Trace(tr.tokens, tr.offsets[:nr + 1], tr.release[:nr], tr.out_len[:nr],
+                    tr.group[:nr])
+    st, rw, _, _ = ref.route(0, head.tokens, head.offsets, head.out_len)
+    assert st == 0 and np.array_equal(wo.cpu().numpy(), rw)
+    m = tr.n_req - nr
+    po = torch.full((m * W,), -1, dtype=torch.int32, device="cuda")
+    rs.route_probe(ctx.h, 0, d.tokens, d.offsets[nr:], m, po)
+    torch.cuda.synchronize()
+    got = po.cpu().numpy().reshape(m, W)
+    st, want = ref.probe(0, tr.tokens, tr.offsets[nr:])
+    assert st == 0 and np.array_equal(got, want)
+    assert got.mean() > 1.0
