@@ -9,12 +9,16 @@
 // LRU cache update and load update -- and its Eq. (9) latency.
 //
 // Per request i (256 threads, 8 warps):
-//   probe      all warps: cached prefix m_ij on every worker;
-//   choose     warp 0: Eq. (1) costs and the Eq. (2) choice; warp 1: tie stats;
-//   update     warps 0-6 (named barrier): the chosen worker's cache;
-//   control    warp 7, at the same time: request i's load, service start and
-//              latency, then request i+1's completions and controller samples
-//              up to its arrival, and its block hashes into the other buffer.
+//   probe      warps 0-6: cached prefix m_ij on every worker; warp 7, at the
+//              same time: request i's completions and controller samples up
+//              to its arrival;
+//   choose     every warp alike: Eq. (1) costs and the Eq. (2) choice (no
+//              barrier after it);
+//   update     warps 0-6 (named barrier 1): the chosen worker's cache;
+//   control    warp 7, at the same time (once the update group has read its
+//              inputs, named barrier 3): the decision's records and
+//              statistics, request i's load, service start and latency, then
+//              request i+1's scalars and block hashes into the other buffer.
 // The control work is serial and runs on float64, whose dependent-operation
 // latency on this GPU is long; the cache update is memory-bound.  Neither needs
 // the other's results, so they overlap.  Times are ordered through an integer
@@ -103,7 +107,7 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(wqh, 4 * (size_t)W, 4)
   TAKE(wqt, 4 * (size_t)W, 4)
   TAKE(wm, 4 * (size_t)W, 4)
-  TAKE(wcost, 4 * (size_t)W, 4)
+  TAKE(wcost, 4 * (size_t)W * (NT_SIM / 32), 4)   // one cost row per warp
   TAKE(wopen, 4 * (size_t)W, 4)
   TAKE(wabs, 4 * (size_t)W, 4)
   TAKE(kind, nb, 1)
@@ -157,7 +161,7 @@ struct SimScalars {
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk, rebuild, nabs;
+  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk;
   uint32_t dclock;             // decay step of the request being updated (frequency eviction)
   int64_t kv[5];               // Game 2: own G1 / G2 / G3, remote, recompute blocks
   double kv_cost;              // summed Eq. kv-cost
@@ -804,21 +808,23 @@ __device__ __forceinline__ void tier_advance(SimCtx& c, const TableView& tv, con
 // Cache update of the chosen worker (update group, warps 0-6) for request i.
 // MODE: SIM_FREQ when the launch holds replicas that evict by frequency,
 // SIM_TIER for Game 2 tiers (the LRU-only kernel carries neither).
+// nabs: the worker's absent blocks (from the probe); rebuild: rebuild the
+// table first; dup: the prompt repeats a block hash (the update stops).
 template <int MODE>
 __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, int j, int nb,
-                                              bool full, int64_t i) {
+                                              bool full, int64_t i, int nabs, bool rebuild,
+                                              bool dup) {
   constexpr bool FREQ = MODE == SIM_FREQ, TIER = MODE == SIM_TIER;
   SimScalars& S = *c.S;
   const TableGeom& g = c.L->g;
   const TableView tv = c.table(j);
   CacheMeta* meta = &c.wmeta[j];
-  // (the duplicate detector was released and the rebuild decided at the choice)
-  if (S.us.dup) {
+  if (dup) {
     if (threadIdx.x == 0) S.status = RS_ERR_COLLISION;
     return;
   }
   uint64_t* gtmp = c.b->tmp + (size_t)c.sid * g.K;
-  if (S.rebuild) {
+  if (rebuild) {
     cache_rebuild<NT_UPD>(tv, meta, g.K, gtmp, S.warp_tot, &S.us,
                           FREQ && c.b->tmpe ? c.b->tmpe + (size_t)c.sid * g.K : nullptr,
                           FREQ ? &c.wfreq[j] : nullptr);
@@ -834,14 +840,14 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
   }
   const uint32_t size0 = meta->size;   // before this update (tiers)
   const TierMeta b0 = TIER ? c.wtier[j] : TierMeta{0u, 0u};
-  const bool captured = full && !S.rebuild;
+  const bool captured = full && !rebuild;
   if (FREQ && c.d->eviction == RS_EVICT_FREQ) {
     // the KV Block Manager's frequency rule
     const uint32_t D = S.dclock;
     FreqMeta* fm = &c.wfreq[j];
     if (captured) {
       cache_prepare_captured_freq<NT_UPD>(tv, meta, fm, g.K, c.pslot + (size_t)j * nb,
-                                          c.pfree + (size_t)j * nb, nb, S.nabs, D, c.sc, &S.us,
+                                          c.pfree + (size_t)j * nb, nb, nabs, D, c.sc, &S.us,
                                           &S.fs, S.warp_tot, &S.scan_pos);
     } else {
       cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
@@ -852,7 +858,7 @@ __device__ __forceinline__ void update_chosen(SimCtx& c, const uint64_t* hbuf, i
   } else {
     if (captured)
       cache_prepare_captured<NT_UPD>(tv, meta, g.K, c.pslot + (size_t)j * nb,
-                                     c.pfree + (size_t)j * nb, nb, S.nabs, c.sc, &S.us,
+                                     c.pfree + (size_t)j * nb, nb, nabs, c.sc, &S.us,
                                      S.warp_tot, &S.scan_pos);
     else
       cache_lookup_all<NT_UPD, false>(tv, hbuf, nb, c.sc, &S.us, &S.probes);
@@ -955,7 +961,14 @@ __device__ __forceinline__ void load_request(const SimCtx& c, ReqState& q, const
 }
 
 // Algorithm 1: the router parameters of the current regime (control thread).
+// Called once request q's arrival is known and its events are done; with
+// frequency eviction it also sets the decay step of that arrival.
+template <bool FREQ>
 __device__ __forceinline__ void regime_params(const SimCtx& c, ReqState& q) {
+  if (FREQ && c.d->eviction == RS_EVICT_FREQ) {   // decay step of the arrival
+    const double t = floor(__ddiv_rn(q.a, c.d->decay_s));
+    c.S->dclock = t < 2147483648.0 ? (uint32_t)t : 2147483648u;
+  }
   float tau = c.d->tau, om = c.d->omega;
   if (c.d->policy == RS_POLICY_LOADBAL) {
     tau = 0.0f;
@@ -1142,7 +1155,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       // ---- control thread, at the same time: completions and controller
       // samples up to request i's arrival (the probe needs none of them)
       S.evres = events_advance(c, S.q[p]);
-      if (S.evres == 0) regime_params(c, S.q[p]);
+      if (S.evres == 0) regime_params<FREQ>(c, S.q[p]);
     }
     __syncthreads();
     // ---- controller samples whose window needs the CTA (P99 of Eq. (10))
@@ -1150,81 +1163,70 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       tick_cta(c);
       if (threadIdx.x == CTL) {
         S.evres = events_advance(c, S.q[p]);
-        if (S.evres == 0) regime_params(c, S.q[p]);
+        if (S.evres == 0) regime_params<FREQ>(c, S.q[p]);
       }
       __syncthreads();
     }
     if (S.status != RS_OK) break;
-    // ---- Eq. (1) costs, frozen loads of Eq. (12), Eq. (2) choice (warp 0)
-    if (warp == 0) {
-      const float om = S.q[p].omega, tau = S.q[p].tau;
-      const bool eq2 = d.policy == RS_POLICY_DYNAMO || d.policy == RS_POLICY_LOADBAL;
-      // lane per worker; the lowest-index argmin (the choice at tau = 0) by a
-      // butterfly over (cost, index), no serial pass over shared memory
-      float bc = __int_as_float(0x7F800000);
-      int bj = 0x7FFFFFFF;
-      for (int j = lane; j < W; j += 32) {
-        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
-        c.wcost[j] = cj;
-        b.rec.n_frozen[row * W + j] = (uint16_t)min(c.winserv[j] + 1, mc.cap - 1);
-        b.rec.prefix[row * W + j] = (uint16_t)c.wm[j];
-        if (mc.write_cost) b.rec.cost[row * W + j] = cj;
-        if (cj < bc || bj == 0x7FFFFFFF) {
-          bc = cj;
-          bj = j;
-        }
+    // ---- Eq. (1) costs and the Eq. (2) choice, computed alike by every warp
+    // (same inputs, same operations, so the same worker) so that the update
+    // starts without a CTA barrier; the control warp records the decision
+    const float om = S.q[p].omega, tau = S.q[p].tau;
+    const bool eq2 = d.policy == RS_POLICY_DYNAMO || d.policy == RS_POLICY_LOADBAL;
+    float* wc = c.wcost + (size_t)warp * W;   // this warp's cost row
+    float bc = __int_as_float(0x7F800000);
+    int bj = 0x7FFFFFFF;
+    for (int j = lane; j < W; j += 32) {
+      const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
+      wc[j] = cj;
+      if (cj < bc || bj == 0x7FFFFFFF) {
+        bc = cj;
+        bj = j;
       }
-      argmin_warp(bc, bj);
+    }
+    argmin_warp(bc, bj);   // the lowest-index argmin (the choice at tau = 0)
+    int js = bj;
+    if (!eq2 || tau > 0.0f) {
       __syncwarp();
+      int x = 0;
       if (lane == 0) {
-        const uint32_t u24 = eq2 && tau > 0.0f ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
-        float* ds = b.dstat + row * 6;
-        const int js = !eq2 ? static_policy_worker(d.policy, c.wcost, W, d.seed, (uint64_t)i, 0u,
-                                                   TAG_SIM)
-                            : (tau == 0.0f ? bj : select_worker(c.wcost, W, tau, u24, ds + 2));
-        S.jstar = js;
-        S.hit_blocks += c.wm[js];
-        if (FREQ && d.eviction == RS_EVICT_FREQ) {   // decay step of this request's arrival
-          const double q = floor(__ddiv_rn(S.q[p].a, d.decay_s));
-          S.dclock = q < 2147483648.0 ? (uint32_t)q : 2147483648u;
-        }
-        // the chosen worker's absent blocks, latched before the control warp
-        // resets the probe state for the next request
-        S.nabs = c.wabs[js];
-        // two blocks of the prompt with one chained hash (a 64-bit collision,
-        // flagged per request before the launch) would break the batched update
-        if (S.q[p].dup) S.us.dup = 1;
-        // the chosen worker's table: rebuild first when its log span, its
-        // tombstones or its stamps would overflow
-        const CacheMeta* mt = &c.wmeta[js];
-        const uint64_t span = (uint64_t)mt->T - mt->head + (uint64_t)nb;
-        S.rebuild = span > L.g.R || mt->tombs > L.g.slots / 8 || (uint64_t)mt->T + nb > STAMP_LIMIT;
-        if (eq2 && tau > 0.0f) S.sampled++;
-        else ds[3] = -1.0f;   // no Eq. (2) draw
+        const uint32_t u24 = eq2 ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
+        x = !eq2 ? static_policy_worker(d.policy, wc, W, d.seed, (uint64_t)i, 0u, TAG_SIM)
+                 : select_worker(wc, W, tau, u24, nullptr);
       }
-    } else if (warp == 1) {
-      // statistics of the decision, beside the choice: work done by the probe
-      // and the two lowest Eq. (1) costs, for the near-tie statistic (counted
-      // after the run); recomputed from the probe results so as not to wait
-      // for warp 0
-      const float om = S.q[p].omega;
+      js = __shfl_sync(FULL_MASK, x, 0);
+    }
+    if (warp < NT_SIM / 32 - 1) {
+      // ---- the chosen worker's LRU cache (warps 0-6).  Its inputs are read
+      // before the arrival that lets the control warp reset the probe state
+      // and change the loads.
+      const int nabs = c.wabs[js];   // absent blocks (victim count)
+      // the chosen worker's table: rebuild first when its log span, its
+      // tombstones or its stamps would overflow
+      const CacheMeta* mt = &c.wmeta[js];
+      const uint64_t span = (uint64_t)mt->T - mt->head + (uint64_t)nb;
+      const bool rebuild =
+          span > L.g.R || mt->tombs > L.g.slots / 8 || (uint64_t)mt->T + nb > STAMP_LIMIT;
+      // two blocks of the prompt with one chained hash (a 64-bit collision,
+      // flagged per request before the launch) would break the batched update
+      const bool dup = S.q[p].dup != 0;
+      asm volatile("bar.arrive 3, %0;" ::"n"(NT_SIM) : "memory");
+      if (TIER) tier_charge<NT_UPD>(c, js, nb, row);
+      update_chosen<MODE>(c, hb, js, nb, full, i, nabs, rebuild, dup);
+    } else {
+      asm volatile("bar.sync 3, %0;" ::"n"(NT_SIM) : "memory");   // the update group has read
+      // records of the decision: frozen loads of Eq. (12), prefixes, costs;
+      // the work done by the probe and the two lowest Eq. (1) costs, for the
+      // near-tie statistic (counted after the run)
       int pb = 0;
-      float c1 = __int_as_float(0x7F800000);
-      int bmin = 0x7FFFFFFF;
-      for (int j = lane; j < W; j += 32) {
-        const int m = c.wm[j];
-        pb += min(m + 1, nb);
-        const float cj = router_cost(om, (int64_t)nbt - m, c.wA[j]);
-        if (cj < c1 || bmin == 0x7FFFFFFF) {
-          c1 = cj;
-          bmin = j;
-        }
-      }
-      argmin_warp(c1, bmin);
       float c2 = __int_as_float(0x7F800000);
       for (int j = lane; j < W; j += 32) {
-        const float cj = router_cost(om, (int64_t)nbt - c.wm[j], c.wA[j]);
-        if (j != bmin && cj < c2) c2 = cj;
+        const int m = c.wm[j];
+        b.rec.n_frozen[row * W + j] = (uint16_t)min(c.winserv[j] + 1, mc.cap - 1);
+        b.rec.prefix[row * W + j] = (uint16_t)m;
+        if (mc.write_cost) b.rec.cost[row * W + j] = wc[j];
+        pb += min(m + 1, nb);
+        if (j != bj && wc[j] < c2) c2 = wc[j];
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
@@ -1233,19 +1235,21 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       }
       pb = (int)__reduce_add_sync(FULL_MASK, (unsigned)pb);
       if (lane == 0) {
+        float* ds = b.dstat + row * 6;
+        ds[0] = bc;
+        ds[1] = c2;
+        if (eq2 && tau > 0.0f) {   // the draw's position, for the near-boundary statistic
+          select_worker(wc, W, tau, draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM), ds + 2);
+          S.sampled++;
+        } else {
+          ds[3] = -1.0f;   // no Eq. (2) draw
+        }
+        S.jstar = js;
+        S.hit_blocks += c.wm[js];
         S.probe_blocks += pb;
         S.hashed_blocks += nb;
-        b.dstat[row * 6] = c1;
-        b.dstat[row * 6 + 1] = c2;
       }
-    }
-    __syncthreads();
-    const int js = S.jstar;
-    if (warp < NT_SIM / 32 - 1) {
-      // ---- the chosen worker's LRU cache (warps 0-6)
-      if (TIER) tier_charge<NT_UPD>(c, js, nb, row);
-      update_chosen<MODE>(c, hb, js, nb, full, i);
-    } else {
+      __syncwarp();
       // ---- control warp: request i's load and latency; request i+1's
       // scalars, probe state and block hashes
       ReqState& nq = S.q[p ^ 1];
