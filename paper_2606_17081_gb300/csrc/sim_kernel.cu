@@ -1191,8 +1191,10 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       int x = 0;
       if (lane == 0) {
         const uint32_t u24 = eq2 ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
+        // (the control warp also records where the draw fell)
         x = !eq2 ? static_policy_worker(d.policy, wc, W, d.seed, (uint64_t)i, 0u, TAG_SIM)
-                 : select_worker(wc, W, tau, u24, nullptr);
+                 : select_worker(wc, W, tau, u24,
+                                 warp == NT_SIM / 32 - 1 ? b.dstat + row * 6 + 2 : nullptr);
       }
       js = __shfl_sync(FULL_MASK, x, 0);
     }
@@ -1238,12 +1240,8 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         float* ds = b.dstat + row * 6;
         ds[0] = bc;
         ds[1] = c2;
-        if (eq2 && tau > 0.0f) {   // the draw's position, for the near-boundary statistic
-          select_worker(wc, W, tau, draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM), ds + 2);
-          S.sampled++;
-        } else {
-          ds[3] = -1.0f;   // no Eq. (2) draw
-        }
+        if (eq2 && tau > 0.0f) S.sampled++;   // (ds[2..5] written with the draw)
+        else ds[3] = -1.0f;                    // no Eq. (2) draw
         S.jstar = js;
         S.hit_blocks += c.wm[js];
         S.probe_blocks += pb;
