@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 31917070848 + 6057946624,
-               "sources_sha256": "dabbdc910f9daa14357965934473d558647f8f8cfb212b8096cd6b4bfa2d1966",
+SIM_TRAFFIC = {"bytes": 32004636928 + 6066514432,
+               "sources_sha256": "77d9cc6287d7180f74c26acf793cbab9b8e2c81113201ce276b503b4e12c4e6d",
                "summary": "profiles/k_sim_p2d.md"}
 
 
