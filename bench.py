@@ -145,8 +145,8 @@ def _table_bytes(K: int) -> int:
 # DRAM bytes (read + write) of one full-size k_sim launch of this workload,
 # from a one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # with the SHA-256 of the simulation kernel's sources it was taken with.
-SIM_TRAFFIC = {"bytes": 32004636928 + 6066514432,
-               "sources_sha256": "77d9cc6287d7180f74c26acf793cbab9b8e2c81113201ce276b503b4e12c4e6d",
+SIM_TRAFFIC = {"bytes": 31999974144 + 6064310016,
+               "sources_sha256": "0fc67a527a3b92e59a5a8de6dff6c21835b2d735ef8812b66f6dcbeb12c818d8",
                "summary": "profiles/k_sim_p2d.md"}
 
 

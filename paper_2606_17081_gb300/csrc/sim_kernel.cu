@@ -661,7 +661,7 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   }
   if (threadIdx.x == 0) S.probes += (unsigned long long)total;
   if (err) S.status = RS_ERR_TIMEOUT;
-  grp_bar<NT>();
+  // (the CTA barrier after the probe orders these results with their readers)
 }
 
 // Game 2 charge of request i (Eq. kv-cost, §4.2) on its worker sigma, from the
@@ -1147,7 +1147,6 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
         probe_full<NT_UPD, TIER>(c, hb, nb);
       } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
         if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
-        grp_bar<NT_UPD>();
       } else {
         probe_prefixes<NT_UPD>(c, hb, nb);
       }
