@@ -369,6 +369,24 @@ static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbm
   return RS_OK;
 }
 
+// Block hashes of one batch of a router instance into ctx->r_hash (sized from
+// offsets_dev[n_req], read with a synchronising copy); nbmax_dev (nullable)
+// receives the longest prompt's full blocks.
+static rs_status hash_batch(rs_ctx* ctx, const int32_t* tokens_dev, const int64_t* offsets_dev,
+                            int64_t n_req, int64_t* nbmax_dev) {
+  rs_status r = ensure_pinned(ctx, 4);
+  if (r != RS_OK) return r;
+  CK(cudaMemcpyAsync(ctx->pinned, offsets_dev + n_req, 8, cudaMemcpyDeviceToHost, ctx->st),
+     "read offsets");
+  CK(cudaStreamSynchronize(ctx->st), "sync");
+  const int64_t total = ctx->pinned[0];
+  if (total < 0) return fail(ctx, RS_ERR_INVALID, "offsets[n_req] < 0");
+  if ((r = ensure(ctx, ctx->r_hash, (size_t)(total / 16 + 1) * 8, "batch hashes")) != RS_OK) return r;
+  std::vector<HashJob> jobs(1);
+  jobs[0] = HashJob{tokens_dev, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, 0};
+  return hash_jobs(ctx, jobs, nbmax_dev);
+}
+
 // ---------------------------------------------------------------- live router
 
 static rs_status router_state(rs_ctx* ctx, int32_t inst, RouterState* s) {
@@ -398,19 +416,9 @@ rs_status route_batch(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
   if (!tokens_dev || !offsets_dev || !out_len_dev || !worker_out_dev)
     return fail(ctx, RS_ERR_INVALID, "NULL pointer");
   if (!aligned16(tokens_dev)) return fail(ctx, RS_ERR_INVALID, "tokens must be 16-byte aligned");
-  if ((r = ensure_pinned(ctx, 4)) != RS_OK) return r;
-  CK(cudaMemcpyAsync(ctx->pinned, offsets_dev + n_req, 8, cudaMemcpyDeviceToHost, ctx->st),
-     "read offsets");
-  CK(cudaStreamSynchronize(ctx->st), "sync");
-  const int64_t total = ctx->pinned[0];
-  if (total < 0) return fail(ctx, RS_ERR_INVALID, "offsets[n_req] < 0");
-  if ((r = ensure(ctx, ctx->r_hash, (size_t)(total / 16 + 1) * 8, "batch hashes")) != RS_OK) return r;
   CK(cudaMemsetAsync(ctx->r_stats.p, 0, 8, ctx->st), "memset");
-  {
-    std::vector<HashJob> jobs(1);
-    jobs[0] = HashJob{tokens_dev, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, 0};
-    if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->r_stats))) != RS_OK) return r;
-  }
+  if ((r = hash_batch(ctx, tokens_dev, offsets_dev, n_req, P<int64_t>(ctx->r_stats))) != RS_OK)
+    return r;
   CK(cudaMemcpyAsync(ctx->pinned, ctx->r_stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");
   CK(cudaStreamSynchronize(ctx->st), "sync");
   int64_t nbmax = ctx->pinned[0];
@@ -441,18 +449,7 @@ rs_status route_probe(rs_ctx* ctx, int32_t instance, const int32_t* tokens_dev,
   if (n_req == 0) return RS_OK;
   if (!tokens_dev || !offsets_dev || !prefix_out_dev) return fail(ctx, RS_ERR_INVALID, "NULL pointer");
   if (!aligned16(tokens_dev)) return fail(ctx, RS_ERR_INVALID, "tokens must be 16-byte aligned");
-  if ((r = ensure_pinned(ctx, 4)) != RS_OK) return r;
-  CK(cudaMemcpyAsync(ctx->pinned, offsets_dev + n_req, 8, cudaMemcpyDeviceToHost, ctx->st),
-     "read offsets");
-  CK(cudaStreamSynchronize(ctx->st), "sync");
-  const int64_t total = ctx->pinned[0];
-  if (total < 0) return fail(ctx, RS_ERR_INVALID, "offsets[n_req] < 0");
-  if ((r = ensure(ctx, ctx->r_hash, (size_t)(total / 16 + 1) * 8, "batch hashes")) != RS_OK) return r;
-  {
-    std::vector<HashJob> jobs(1);
-    jobs[0] = HashJob{tokens_dev, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, 0};
-    if ((r = hash_jobs(ctx, jobs, nullptr)) != RS_OK) return r;
-  }
+  if ((r = hash_batch(ctx, tokens_dev, offsets_dev, n_req, nullptr)) != RS_OK) return r;
   CK(launch_probe_batch(s, offsets_dev, P<uint64_t>(ctx->r_hash), n_req, ctx->cfg.W, ctx->g,
                         prefix_out_dev, ctx->st),
      "probe launch");
