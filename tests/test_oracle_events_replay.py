@@ -96,3 +96,51 @@ def test_events_match_independent_replay(policy, C, rate, W, seed):
         assert (a > tr.release).any()
     if W == 1:
         assert (s > a).any()
+
+
+def _controller_replay(first, ttft, n_ticks, dt=5.0, alpha=0.3, th=(0.3, 2.0), eps=0.1, k=3):
+    """The controller of §6.2 from the records: at t_k = k dt the window is
+    every request whose first token came in [t_{k-1}, t_k); its nearest-rank
+    P99 (an empty window repeats the last value) feeds the EWMA of Eq. (10),
+    which starts at the first sample; Eq. (11)'s regime moves one step up
+    after k samples at or above the next threshold, one step down after k
+    samples below the current threshold less eps of it."""
+    ewmas, regs = [], []
+    ewma, last, regime, up, down = None, None, 0, 0, 0
+    for kk in range(1, n_ticks + 1):
+        lo, hi = (kk - 1) * dt, kk * dt
+        w = np.sort(ttft[(first >= lo) & (first < hi)])
+        if w.size:
+            last = float(w[int(np.ceil(0.99 * w.size)) - 1])
+        if last is not None:
+            ewma = last if ewma is None else alpha * last + (1.0 - alpha) * ewma
+            go_up = regime < 2 and ewma >= th[regime]
+            go_down = regime > 0 and ewma < th[regime - 1] * (1.0 - eps)
+            up = up + 1 if go_up else 0
+            down = down + 1 if go_down else 0
+            if up >= k:
+                regime, up, down = regime + 1, 0, 0
+            elif down >= k:
+                regime, up, down = regime - 1, 0, 0
+        ewmas.append(-1.0 if ewma is None else ewma)
+        regs.append(regime)
+    return np.array(ewmas), np.array(regs)
+
+
+@pytest.mark.parametrize("C,seed", [(600, 2), (250, 3)])
+def test_controller_matches_replay_from_records(C, seed):
+    # a closed loop that saturates, so that the regime moves
+    spec = Wk.TraceSpec(n_req=6000, n_groups=16, prefix_min=64, prefix_max=256, len_median=256,
+                        len_max=1024)
+    tr = Wk.make_trace(spec, seed)
+    r = O.simulate(O.OracleConfig(W=3, K=4096), tr, C, controller=1, omega=1.0, tau=0.0,
+                   seed=1, max_ticks=4000)
+    assert r["status"] == 0
+    # ticks taken while requests were still arriving: all their windows' first
+    # tokens are known from the records
+    n_ticks = int(np.floor(r["arrival"][-1] / 5.0))
+    assert n_ticks > 5
+    ewma, reg = _controller_replay(r["first_token"], r["ttft"], n_ticks)
+    assert np.allclose(r["tick_ewma"][:n_ticks], ewma, rtol=1e-12, atol=0)
+    assert np.array_equal(r["tick_regime"][:n_ticks], reg)
+    assert reg.max() >= 1
