@@ -85,7 +85,7 @@ enum { RS_MEM_DEVICE = 0, RS_MEM_HOST = 1 };
 typedef struct {
   int32_t W;               /* workers (1..64) */
   int32_t block_size;      /* tokens per KV block; must be 16 */
-  int64_t cache_blocks;    /* LRU capacity per worker, blocks (1 .. 2^26) */
+  int64_t cache_blocks;    /* LRU capacity per worker, blocks (1 .. 2^24) */
   uint64_t hash_seed;      /* h_{-1} of the block-hash chain */
   float omega, tau;        /* route_batch router parameters (>= 0) */
   uint64_t seed;           /* route_batch Philox key */
@@ -141,9 +141,13 @@ void route_destroy(rs_ctx* ctx);
 const char* route_last_error(const rs_ctx* ctx);
 
 /* KV block hashing (§2.2 "token blocks"; the hash is this library's choice):
- * g_k folds the block's 8 little-endian 64-bit token pairs through the
- * SplitMix64 finalizer starting from 0x9E3779B97F4A7C15 ^ 16; the chain is
- * h_k = mix(h_{k-1} ^ g_k ^ k) with h_{-1} = cfg.hash_seed, and 0/1 map to 2/3.
+ * the block content g_k folds the block's 8 little-endian 64-bit token pairs
+ * w in order, x = (x ^ w) * 0xBF58476D1CE4E5B9, x ^= x >> 32, from
+ * x = 0x9E3779B97F4A7C15 ^ 16, then takes the SplitMix64 finalizer of x; the
+ * prefix is H_k = H_{k-1} * 0x94D049BB133111EB + g_k (mod 2^64) with
+ * H_{-1} = cfg.hash_seed, so equal prompt prefixes give equal hashes and a
+ * change in block j changes every H_k, k >= j; the stored hash is
+ * h_k = mix(H_k ^ k), with 0 and 1 mapped to 2 and 3.
  * tokens_dev: int32, 16-byte aligned, readable for round_up(offsets[n_req], 4)
  * entries.  offsets_dev: int64 [n_req + 1], non-decreasing, offsets[0] >= 0.
  * hashes_dev: uint64, request i's k-th hash at floor(offsets[i]/16) + k for
@@ -207,13 +211,25 @@ rs_status route_active(rs_ctx* ctx, int32_t instance, int64_t* active_host);
 /* One request trace.  tokens: int32, 16-byte aligned, readable for
  * round_up(offsets[n_req], 4) entries; offsets: int64 [n_req + 1];
  * release: float64 [n_req] client release times (s, non-decreasing);
- * out_len: int32 [n_req] output tokens (>= 0). */
+ * out_len: int32 [n_req] output tokens (>= 0).
+ * hashes: used only when tokens is NULL.  A trace whose tokens are too many to
+ * hold at once (the prompts enter the router only as the block hashes of
+ * §2.2, which Eq. (1)'s cached-prefix term is computed from) is given by its
+ * block hashes instead, as route_hash_blocks writes them for these offsets:
+ * request i's k-th hash at floor(offsets[i]/16) + k, floor(offsets[n_req]/16)
+ * entries, 8-byte aligned, in trace_mem like the other arrays.  Such a trace
+ * skips the hashing step; everything else is the same.  route_hash_blocks
+ * may produce the hashes chunk by chunk: hashing requests i0 .. i1-1 from a
+ * token buffer that starts at token b = 16 * floor(offsets[i0] / 16), with
+ * offsets rebased by b and the output pointer advanced by b / 16, writes
+ * exactly their entries of this layout. */
 typedef struct {
   const int32_t* tokens;
   const int64_t* offsets;
   const double* release;
   const int32_t* out_len;
   int64_t n_req;
+  const uint64_t* hashes;
 } rs_trace;
 
 /* One replica of the closed-loop simulation (§7.4 client holding C requests
@@ -316,11 +332,14 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
 
 /* Eq. (12) on caller records of one replica (device pointers, n rows,
  * cfg.W columns in the per-worker arrays; worker < 0 marks rows to skip).
- * Windows are [k w, (k+1) w) of completion time, w = cfg.poa_window.
+ * Windows are [k w, (k+1) w) of completion time, w = cfg.poa_window; every
+ * window up to the last routed completion is computed, however sparse the
+ * records (the window scratch is sized from the records on the device first).
  * numer_host/opt_host/count_host: NULL or arrays of *n_windows_inout entries;
  * on return *n_windows_inout = windows spanned (if larger than the capacity
  * given, only that many are written).  poa_total_host: sum numer / sum OPT.
- * Synchronises. */
+ * RS_ERR_INVALID when a routed row's completion is negative or not finite;
+ * RS_ERR_CAPACITY beyond 2^31 - 2 windows.  Synchronises. */
 rs_status poa_estimate(rs_ctx* ctx, const rs_records* records, int64_t n, double* numer_host,
                        double* opt_host, int64_t* count_host, int64_t* n_windows_inout,
                        double* poa_total_host);
@@ -376,26 +395,30 @@ rs_status sweep_knee(rs_ctx* ctx, const rs_records* records, const int64_t* row_
  * front by another allocator, or a latency-critical path where cudaMalloc /
  * cudaFree would synchronise the device.
  *
- * Same result as poa_estimate (Eq. (12) per window of completion time) for
- * caller records of one replica (device pointers, n rows, cfg->W <= 64
- * columns), computed in a fixed static device array of RS_NOALLOC_POA_BYTES
- * bytes that every GPU loading the library holds until the process exits.
- * No context is needed; nothing is allocated (no cudaMalloc, cudaFree or
- * allocating library call) and nothing is read back to the host: the work is
- * enqueued on cuda_stream (NULL = legacy default stream).
+ * Same result as poa_estimate for caller records of one replica (device
+ * pointers, n rows, cfg->W <= 64 columns), computed in a fixed static device
+ * array of RS_NOALLOC_POA_BYTES bytes that every GPU loading the library
+ * holds until the process exits.  No context is needed; nothing is allocated
+ * (no cudaMalloc, cudaFree or allocating library call) and nothing is read
+ * back to the host: the work is enqueued on cuda_stream (NULL = legacy
+ * default stream).
  *   cfg: host struct; poa_window, cap, the latency constants and W are used.
  *   numer_dev/opt_dev (double) and count_dev (int64), each NULL or
  *   max_windows entries: the first min(windows, max_windows) windows.
- *   poa_total_dev (double) and n_windows_dev (int64): one entry each;
- *   *n_windows_dev = -1 if the records span more than n + 2 windows.
- * Returns RS_ERR_CAPACITY (before any work) when n rows of W columns need
- * more than the static array: about n * (8 W + 68) + 2 KB bytes, i.e. up to
- * roughly 360 000 rows at W = 3.  The first call on a device takes the
- * array's device address (cudaGetSymbolAddress) for that device; make that
- * first call before any stream capture.  All calls on a device share the one
- * array and every call rewrites what it reads, so calls that overlap on the
- * GPU (other streams, other host threads) race and must be serialised by
- * the caller. */
+ *   poa_total_dev (double) and n_windows_dev (int64): one entry each.
+ * Sizes: accepted when n (8 W + 60) + 4096 <= RS_NOALLOC_POA_BYTES, i.e. up to
+ * 399 408 rows at W = 3 (171 175 at W = 17); larger calls return
+ * RS_ERR_CAPACITY before any work.  The windows get the bytes the rows leave,
+ * 48 per window and never fewer than n + 2 windows; records that span more
+ * windows than that give *n_windows_dev = -1 (and no estimate).
+ * The first call on a device takes the array's device address
+ * (cudaGetSymbolAddress) for that device and keeps it for the life of the
+ * process; make that first call before any stream capture.  The address is
+ * not taken again, so the library cannot be used this way after a
+ * cudaDeviceReset (which unloads the array) in the same process.  All calls
+ * on a device share the one array and every call rewrites what it reads, so
+ * calls that overlap on the GPU (other streams, other host threads) race and
+ * must be serialised by the caller. */
 #define RS_NOALLOC_POA_BYTES (32u * 1024u * 1024u)
 rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records* records, int64_t n,
                                double* numer_dev, double* opt_dev, int64_t* count_dev,

@@ -39,6 +39,8 @@ struct rs_ctx {
   DevBuf keys, stamp, log, tmp, pend, meta_out, res, desc, hashes, stats, hjobs, dstat, wco, slots;
   DevBuf fexp, tmpe;   // frequency eviction state and its rebuild scratch
   DevBuf dupf;         // per request: a chained hash repeats within the prompt
+  DevBuf djobs;        // every trace in use, for the block-count and flag kernels
+  DevBuf h_hashes;     // staged block hashes of host traces given by their hashes
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
@@ -149,6 +151,9 @@ rs_status check_config(const rs_config* cfg) {
   return RS_OK;
 }
 
+}  // namespace
+
+namespace rs {
 ModelConsts make_consts(const rs_config& c) {
   ModelConsts m;
   m.lat_a = c.lat_a; m.lat_b = c.lat_b; m.lat_d = c.lat_d; m.w_c = c.w_c; m.itl = c.itl;
@@ -161,8 +166,12 @@ ModelConsts make_consts(const rs_config& c) {
   m.tier_dn = c.tier_d_near;
   m.tier_df = c.tier_d_far;
   m.tier_node = c.tier_node > 0 ? c.tier_node : 1;
+  m.reserved = 0;
   return m;
 }
+}  // namespace rs
+
+namespace {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -301,7 +310,7 @@ void route_destroy(rs_ctx* ctx) {
                    &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->h_tokens, &ctx->h_offsets,
                    &ctx->h_release, &ctx->h_outlen, &ctx->k_rows, &ctx->k_load, &ctx->k_sweep,
                    &ctx->k_stat, &ctx->k_d1, &ctx->k_d2, &ctx->k_kload, &ctx->k_kidx,
-                   &ctx->fexp, &ctx->tmpe};
+                   &ctx->fexp, &ctx->tmpe, &ctx->djobs, &ctx->h_hashes};
   for (DevBuf* b : all) release(*b);
   if (ctx->pinned) cudaFreeHost(ctx->pinned);
   for (auto& ev : ctx->ev)
@@ -343,26 +352,32 @@ rs_status route_dup_flags(rs_ctx* ctx, const uint64_t* hashes_dev, const int64_t
   return RS_OK;   // (a copy from pageable memory has read its source when it returns)
 }
 
+// The jobs with their request numbers made relative to the first job of
+// each launch group of HASH_MAX_JOBS (the kernels number requests from 0
+// within a launch); jobs must number their requests contiguously.
+static std::vector<HashJob> group_jobs(const std::vector<HashJob>& jobs) {
+  std::vector<HashJob> out(jobs);
+  for (size_t g0 = 0; g0 < out.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(out.size(), g0 + HASH_MAX_JOBS);
+    const int64_t base = jobs[g0].req_base;
+    for (size_t k = g0; k < g1; k++) out[k].req_base -= base;
+  }
+  return out;
+}
+
 // Hashes every job (trace) in launches of up to HASH_MAX_JOBS traces.
 static rs_status hash_jobs(rs_ctx* ctx, std::vector<HashJob>& jobs, int64_t* nbmax_dev) {
   if (jobs.empty()) return RS_OK;
   rs_status r = ensure(ctx, ctx->hjobs, sizeof(HashJob) * jobs.size(), "hash jobs");
   if (r != RS_OK) return r;
-  CK(cudaMemcpyAsync(ctx->hjobs.p, jobs.data(), sizeof(HashJob) * jobs.size(),
+  const std::vector<HashJob> grp = group_jobs(jobs);
+  CK(cudaMemcpyAsync(ctx->hjobs.p, grp.data(), sizeof(HashJob) * grp.size(),
                      cudaMemcpyHostToDevice, ctx->st),
      "copy hash jobs");
   for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
     const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
-    const int64_t base = jobs[g0].req_base;
-    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - base;
-    // the kernels number requests from 0 within a launch
-    std::vector<HashJob> grp(jobs.begin() + g0, jobs.begin() + g1);
-    for (auto& j : grp) j.req_base -= base;
-    if (g0 > 0 || base != 0)
-      CK(cudaMemcpyAsync(P<HashJob>(ctx->hjobs) + g0, grp.data(), sizeof(HashJob) * grp.size(),
-                         cudaMemcpyHostToDevice, ctx->st),
-         "copy hash jobs");
-    CK(launch_block_hash(P<HashJob>(ctx->hjobs) + g0, (int)grp.size(), total, ctx->cfg.hash_seed,
+    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - jobs[g0].req_base;
+    CK(launch_block_hash(P<HashJob>(ctx->hjobs) + g0, (int)(g1 - g0), total, ctx->cfg.hash_seed,
                          nbmax_dev, ctx->st),
        "block hash launch");
   }
@@ -543,8 +558,11 @@ static rs_status records_effective(rs_ctx* ctx, const rs_records* user, int64_t 
   return RS_OK;
 }
 
-static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, const std::vector<PoaProblem>& probs,
-                         int64_t rows, int64_t win_slots, rs_replica_result* res_dev) {
+// Eq. (12) for every problem in probs (rec_base, n, scratch_base set; the
+// window slots are sized here): the last window of each problem is found on
+// the device first, so that every window its records span gets a slot.
+static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, std::vector<PoaProblem>& probs,
+                         int64_t rows, rs_replica_result* res_dev) {
   const int W = ctx->cfg.W;
   const int np = (int)probs.size();
   rs_status r;
@@ -552,16 +570,38 @@ static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, const std::vector<P
       (r = ensure(ctx, ctx->p_order, (size_t)rows * 4, "poa order")) ||
       (r = ensure(ctx, ctx->p_asg, (size_t)rows * 4, "poa assignment")) ||
       (r = ensure(ctx, ctx->p_wkey, (size_t)rows * 4, "poa keys")) ||
-      (r = ensure(ctx, ctx->p_wstart, (size_t)(win_slots + np) * 8, "poa windows")) ||
+      (r = ensure(ctx, ctx->p_tstat, (size_t)np * 8, "poa totals")) ||
+      (r = ensure(ctx, ctx->p_total, (size_t)np * 8, "poa totals")) ||
+      (r = ensure(ctx, ctx->p_nwin, (size_t)np * 8, "poa totals")) ||
+      (r = ensure(ctx, ctx->p_prob, (size_t)np * sizeof(PoaProblem), "poa problems")) ||
+      (r = ensure_pinned(ctx, (size_t)np)))
+    return r;
+  CK(cudaMemcpyAsync(ctx->p_prob.p, probs.data(), np * sizeof(PoaProblem), cudaMemcpyHostToDevice,
+                     ctx->st),
+     "copy poa problems");
+  // last window of every problem (p_nwin serves as the span's output)
+  CK(launch_poa_span(P<PoaProblem>(ctx->p_prob), np, rec, ctx->cfg.poa_window,
+                     reinterpret_cast<long long*>(ctx->p_nwin.p), ctx->st),
+     "poa span launch");
+  CK(cudaMemcpyAsync(ctx->pinned, ctx->p_nwin.p, (size_t)np * 8, cudaMemcpyDeviceToHost, ctx->st),
+     "read poa spans");
+  CK(cudaStreamSynchronize(ctx->st), "sync");
+  int64_t win_slots = 0;
+  for (int k = 0; k < np; k++) {
+    const int64_t last = ctx->pinned[k];   // -1: nothing routed
+    if (last > (int64_t)INT32_MAX - 2)
+      return fail(ctx, RS_ERR_CAPACITY,
+                  "problem %d: completions span more than 2^31 - 2 PoA windows", k);
+    probs[k].win_base = win_slots;
+    probs[k].win_cap = last + 2;   // windows 0 .. last, and one to spare
+    win_slots += probs[k].win_cap;
+  }
+  if ((r = ensure(ctx, ctx->p_wstart, (size_t)(win_slots + np) * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wfill, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wnum, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wopt, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wstat, (size_t)win_slots * 8, "poa windows")) ||
-      (r = ensure(ctx, ctx->p_tstat, (size_t)np * 8, "poa totals")) ||
-      (r = ensure(ctx, ctx->p_wcnt, (size_t)win_slots * 8, "poa windows")) ||
-      (r = ensure(ctx, ctx->p_total, (size_t)np * 8, "poa totals")) ||
-      (r = ensure(ctx, ctx->p_nwin, (size_t)np * 8, "poa totals")) ||
-      (r = ensure(ctx, ctx->p_prob, (size_t)np * sizeof(PoaProblem), "poa problems")))
+      (r = ensure(ctx, ctx->p_wcnt, (size_t)win_slots * 8, "poa windows")))
     return r;
   CK(cudaMemcpyAsync(ctx->p_prob.p, probs.data(), np * sizeof(PoaProblem), cudaMemcpyHostToDevice,
                      ctx->st),
@@ -602,13 +642,15 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   for (int t = 0; t < n_traces; t++) {
     const rs_trace& tr = traces[t];
     if (tr.n_req < 0) return fail(ctx, RS_ERR_INVALID, "trace %d: n_req < 0", t);
-    if (tr.n_req > 0 && (!tr.tokens || !tr.offsets || !tr.release || !tr.out_len))
+    if (tr.n_req > 0 && ((!tr.tokens && !tr.hashes) || !tr.offsets || !tr.release || !tr.out_len))
       return fail(ctx, RS_ERR_INVALID, "trace %d: NULL pointer", t);
-    if (tr.n_req > 0 && !aligned16(tr.tokens))
+    if (tr.n_req > 0 && tr.tokens && !aligned16(tr.tokens))
       return fail(ctx, RS_ERR_INVALID, "trace %d: tokens must be 16-byte aligned", t);
+    if (tr.n_req > 0 && !tr.tokens && ((reinterpret_cast<uintptr_t>(tr.hashes) & 7u) != 0))
+      return fail(ctx, RS_ERR_INVALID, "trace %d: hashes must be 8-byte aligned", t);
     if (tr.n_req > INT32_MAX) return fail(ctx, RS_ERR_CAPACITY, "trace %d: n_req > 2^31-1", t);
   }
-  int64_t rows = 0, pend_cap = 0, win_slots = 0;
+  int64_t rows = 0, pend_cap = 0;
   int cmax = 1;
   bool any_freq = false;   // a replica evicts by frequency: its tables need fexp
   std::vector<char> used(n_traces, 0);
@@ -641,7 +683,6 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     cmax = std::max(cmax, p.C);
     if (p.c_mid > 0) cmax = std::max(cmax, std::max(p.c_mid, p.c_end));
     if (p.controller) pend_cap = std::max(pend_cap, p.n_req);
-    win_slots += p.n_req + 2;
     used[p.trace] = 1;
   }
   const bool host = trace_mem == RS_MEM_HOST;
@@ -652,39 +693,58 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   std::vector<const int64_t*> doff(n_traces);
   std::vector<const double*> drel(n_traces);
   std::vector<const int32_t*> dol(n_traces);
+  // a trace given by its block hashes (tokens NULL) skips S1
+  auto prehashed = [&](int t) { return traces[t].tokens == nullptr; };
+  std::vector<const uint64_t*> dhash(n_traces, nullptr);
   if (host) {
-    size_t tb = 0, ob = 0, nb = 0;
+    size_t tb = 0, ob = 0, nb = 0, hb = 0;
     for (int t = 0; t < n_traces; t++) {
       if (!used[t] || traces[t].n_req == 0) continue;
       const int64_t n = traces[t].n_req;
       tot[t] = traces[t].offsets[n];
-      tb += ((size_t)(tot[t] + 3) / 4 * 4) * 4 + 16;
+      if (tot[t] < 0) return fail(ctx, RS_ERR_INVALID, "trace %d: offsets[n_req] < 0", t);
+      if (prehashed(t))
+        hb += (size_t)(tot[t] / 16 + 1) * 8;
+      else
+        tb += ((size_t)(tot[t] + 3) / 4 * 4) * 4 + 16;
       ob += (size_t)(n + 1) * 8;
       nb += (size_t)n;
     }
     if ((r = ensure(ctx, ctx->h_tokens, tb, "staged tokens")) ||
+        (r = ensure(ctx, ctx->h_hashes, hb, "staged block hashes")) ||
         (r = ensure(ctx, ctx->h_offsets, ob, "staged offsets")) ||
         (r = ensure(ctx, ctx->h_release, nb * 8, "staged release")) ||
         (r = ensure(ctx, ctx->h_outlen, nb * 4, "staged out_len")))
       return r;
-    size_t to = 0, oo = 0, no = 0;
+    size_t to = 0, ho = 0, oo = 0, no = 0;
     for (int t = 0; t < n_traces; t++) {
       if (!used[t] || traces[t].n_req == 0) continue;
       const int64_t n = traces[t].n_req;
-      const size_t tbytes = (size_t)(tot[t] + 3) / 4 * 4 * 4;
-      char* tp = static_cast<char*>(ctx->h_tokens.p) + to;
-      CK(cudaMemcpyAsync(tp, traces[t].tokens, tbytes, cudaMemcpyHostToDevice, ctx->st), "H2D tokens");
+      if (prehashed(t)) {
+        const size_t hbytes = (size_t)(tot[t] / 16) * 8;
+        uint64_t* hp = P<uint64_t>(ctx->h_hashes) + ho;
+        if (hbytes)
+          CK(cudaMemcpyAsync(hp, traces[t].hashes, hbytes, cudaMemcpyHostToDevice, ctx->st),
+             "H2D hashes");
+        dhash[t] = hp;
+        ho += (size_t)(tot[t] / 16 + 1);
+      } else {
+        const size_t tbytes = (size_t)(tot[t] + 3) / 4 * 4 * 4;
+        char* tp = static_cast<char*>(ctx->h_tokens.p) + to;
+        CK(cudaMemcpyAsync(tp, traces[t].tokens, tbytes, cudaMemcpyHostToDevice, ctx->st),
+           "H2D tokens");
+        dtok[t] = reinterpret_cast<const int32_t*>(tp);
+        to += (tbytes + 15) & ~(size_t)15;
+      }
       CK(cudaMemcpyAsync(P<int64_t>(ctx->h_offsets) + oo, traces[t].offsets, (n + 1) * 8,
                          cudaMemcpyHostToDevice, ctx->st), "H2D offsets");
       CK(cudaMemcpyAsync(P<double>(ctx->h_release) + no, traces[t].release, n * 8,
                          cudaMemcpyHostToDevice, ctx->st), "H2D release");
       CK(cudaMemcpyAsync(P<int32_t>(ctx->h_outlen) + no, traces[t].out_len, n * 4,
                          cudaMemcpyHostToDevice, ctx->st), "H2D out_len");
-      dtok[t] = reinterpret_cast<const int32_t*>(tp);
       doff[t] = P<int64_t>(ctx->h_offsets) + oo;
       drel[t] = P<double>(ctx->h_release) + no;
       dol[t] = P<int32_t>(ctx->h_outlen) + no;
-      to += (tbytes + 15) & ~(size_t)15;
       oo += n + 1;
       no += n;
     }
@@ -692,6 +752,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     if ((r = ensure_pinned(ctx, (size_t)n_traces + 1)) != RS_OK) return r;
     for (int t = 0; t < n_traces; t++) {
       dtok[t] = traces[t].tokens;
+      dhash[t] = prehashed(t) ? traces[t].hashes : nullptr;
       doff[t] = traces[t].offsets;
       drel[t] = traces[t].release;
       dol[t] = traces[t].out_len;
@@ -707,29 +768,61 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   for (int t = 0; t < n_traces; t++) {
     if (tot[t] < 0) return fail(ctx, RS_ERR_INVALID, "trace %d: offsets[n_req] < 0", t);
     hoff[t] = (int64_t)hash_total;
-    if (used[t]) hash_total += (size_t)(tot[t] / 16 + 1);
+    if (used[t] && !dhash[t]) hash_total += (size_t)(tot[t] / 16 + 1);
   }
   if ((r = ensure(ctx, ctx->hashes, hash_total * 8, "block hashes")) ||
       (r = ensure(ctx, ctx->stats, (size_t)n_traces * 8, "trace stats")) ||
       (r = ensure_pinned(ctx, (size_t)n_traces + 1)))
     return r;
-  // ---- K1: block hashes of every trace in use
+  // ---- K1: block hashes of every trace in use that comes as tokens.  The
+  // hash jobs number their requests among themselves; the per-request flags
+  // number the requests of every trace in use (rbase).
   int64_t launches = 0, hashed_tokens = 0;
-  CK(cudaEventRecord(ctx->ev[0], ctx->st), "event");
-  CK(cudaMemsetAsync(ctx->stats.p, 0, (size_t)n_traces * 8, ctx->st), "memset");
-  std::vector<HashJob> jobs;
-  int64_t req_total = 0;
+  std::vector<HashJob> jobs, all;
+  int64_t req_total = 0, hreq = 0;
   for (int t = 0; t < n_traces; t++) {
     if (!used[t] || traces[t].n_req == 0) continue;
     rbase[t] = req_total;
-    jobs.push_back(HashJob{dtok[t], doff[t], P<uint64_t>(ctx->hashes) + hoff[t], traces[t].n_req,
-                           req_total});
+    uint64_t* hp = dhash[t] ? const_cast<uint64_t*>(dhash[t]) : P<uint64_t>(ctx->hashes) + hoff[t];
+    all.push_back(HashJob{dtok[t], doff[t], hp, traces[t].n_req, req_total});
+    if (!dhash[t]) {
+      jobs.push_back(HashJob{dtok[t], doff[t], hp, traces[t].n_req, hreq});
+      hreq += traces[t].n_req;
+      hashed_tokens += tot[t];
+    }
     req_total += traces[t].n_req;
-    hashed_tokens += tot[t];
   }
-  if ((r = hash_jobs(ctx, jobs, P<int64_t>(ctx->stats))) != RS_OK) return r;
-  launches += ((int64_t)jobs.size() + HASH_MAX_JOBS - 1) / HASH_MAX_JOBS;
+  if ((r = ensure(ctx, ctx->hjobs, sizeof(HashJob) * std::max<size_t>(jobs.size(), 1), "hash jobs")) ||
+      (r = ensure(ctx, ctx->djobs, sizeof(HashJob) * std::max<size_t>(all.size(), 1), "trace jobs")))
+    return r;
+  std::vector<HashJob> hj = group_jobs(jobs);
+  if (!jobs.empty())
+    CK(cudaMemcpyAsync(ctx->hjobs.p, hj.data(), sizeof(HashJob) * hj.size(), cudaMemcpyHostToDevice,
+                       ctx->st), "copy hash jobs");
+  std::vector<HashJob> aj = group_jobs(all);
+  CK(cudaMemcpyAsync(ctx->djobs.p, aj.data(), sizeof(HashJob) * aj.size(), cudaMemcpyHostToDevice,
+                     ctx->st), "copy trace jobs");
+  CK(cudaMemsetAsync(ctx->stats.p, 0, (size_t)n_traces * 8, ctx->st), "memset");
+  // the events time the hash launches alone
+  CK(cudaEventRecord(ctx->ev[0], ctx->st), "event");
+  for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
+    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - jobs[g0].req_base;
+    CK(launch_block_hash(P<HashJob>(ctx->hjobs) + g0, (int)(g1 - g0), total, ctx->cfg.hash_seed,
+                         nullptr, ctx->st),
+       "block hash launch");
+    launches++;
+  }
   CK(cudaEventRecord(ctx->ev[1], ctx->st), "event");
+  // the longest prompt's full blocks, over every trace in use
+  for (size_t g0 = 0; g0 < all.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(all.size(), g0 + HASH_MAX_JOBS);
+    const int64_t total = all[g1 - 1].req_base + all[g1 - 1].n_req - all[g0].req_base;
+    CK(launch_nbmax(P<HashJob>(ctx->djobs) + g0, (int)(g1 - g0), total, P<int64_t>(ctx->stats),
+                    ctx->st),
+       "block count launch");
+    launches++;
+  }
   CK(cudaMemcpyAsync(ctx->pinned, ctx->stats.p, 8, cudaMemcpyDeviceToHost, ctx->st), "read stats");
   CK(cudaStreamSynchronize(ctx->st), "sync");
   int64_t nbmax = std::max<int64_t>(1, ctx->pinned[0]);
@@ -784,14 +877,14 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   if ((r = records_effective(ctx, records, rows, W, want_cost, &rec)) != RS_OK) return r;
   std::vector<SimDesc> desc(nsim);
   std::vector<PoaProblem> probs(nsim);
-  int64_t rb = 0, wb = 0;
+  int64_t rb = 0;
   for (size_t k = 0; k < nsim; k++) {
     const rs_replica_params& p = params[k];
     SimDesc& d = desc[k];
     d.offsets = doff[p.trace];
     d.release = drel[p.trace];
     d.out_len = dol[p.trace];
-    d.hashes = P<uint64_t>(ctx->hashes) + hoff[p.trace];
+    d.hashes = dhash[p.trace] ? dhash[p.trace] : P<uint64_t>(ctx->hashes) + hoff[p.trace];
     d.dupflag = P<uint8_t>(ctx->dupf) + rbase[p.trace];
     d.n_req = p.n_req;
     d.rec_base = rb;
@@ -812,10 +905,7 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     probs[k].rec_base = rb;
     probs[k].n = p.n_req;
     probs[k].scratch_base = rb;
-    probs[k].win_base = wb;
-    probs[k].win_cap = p.n_req + 2;
     rb += p.n_req;
-    wb += p.n_req + 2;
   }
   CK(cudaMemcpyAsync(ctx->desc.p, desc.data(), nsim * sizeof(SimDesc), cudaMemcpyHostToDevice, ctx->st),
      "copy descriptors");
@@ -850,12 +940,12 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
     CK(launch_wco_table(P<double>(ctx->wco), (int)nbmax, ctx->cfg.w_c, ctx->st), "table launch");
     launches++;
   }
-  // per-request duplicate-hash flags, over the jobs as the hashing left them
-  for (size_t g0 = 0; g0 < jobs.size(); g0 += HASH_MAX_JOBS) {
-    const size_t g1 = std::min(jobs.size(), g0 + HASH_MAX_JOBS);
-    const int64_t base = jobs[g0].req_base;
-    const int64_t total = jobs[g1 - 1].req_base + jobs[g1 - 1].n_req - base;
-    CK(launch_dup_flags(P<HashJob>(ctx->hjobs) + g0, (int)(g1 - g0), total, nbmax,
+  // per-request duplicate-hash flags of every trace in use
+  for (size_t g0 = 0; g0 < all.size(); g0 += HASH_MAX_JOBS) {
+    const size_t g1 = std::min(all.size(), g0 + HASH_MAX_JOBS);
+    const int64_t base = all[g0].req_base;
+    const int64_t total = all[g1 - 1].req_base + all[g1 - 1].n_req - base;
+    CK(launch_dup_flags(P<HashJob>(ctx->djobs) + g0, (int)(g1 - g0), total, nbmax,
                         P<uint8_t>(ctx->dupf) + base, ctx->st),
        "duplicate flags launch");
     launches++;
@@ -865,8 +955,8 @@ rs_status simulate_replicas(rs_ctx* ctx, const rs_trace* traces, int32_t n_trace
   launches += 2;
   CK(cudaEventRecord(ctx->ev[2], ctx->st), "event");
   if (!(flags & RS_SIM_NO_POA)) {
-    if ((r = run_poa(ctx, rec, probs, rows, win_slots, sb.res)) != RS_OK) return r;
-    launches += 3;
+    if ((r = run_poa(ctx, rec, probs, rows, sb.res)) != RS_OK) return r;
+    launches += 4;
   }
   CK(cudaEventRecord(ctx->ev[3], ctx->st), "event");
   CK(cudaMemcpyAsync(results_host, sb.res, nsim * sizeof(rs_replica_result), cudaMemcpyDeviceToHost,
@@ -907,11 +997,7 @@ rs_status poa_estimate(rs_ctx* ctx, const rs_records* records, int64_t n, double
   probs[0].rec_base = 0;
   probs[0].n = n;
   probs[0].scratch_base = 0;
-  probs[0].win_base = 0;
-  // windows spanned are bounded by the largest completion time; read it on the host side
-  // from the device is avoided: allow up to n + 2 windows, report overflow otherwise
-  probs[0].win_cap = n + 2;
-  rs_status r = run_poa(ctx, u, probs, std::max<int64_t>(n, 1), n + 2, nullptr);
+  rs_status r = run_poa(ctx, u, probs, std::max<int64_t>(n, 1), nullptr);
   if (r != RS_OK) return r;
   const int64_t cap = *n_windows_inout;
   if ((r = ensure_pinned(ctx, 2)) != RS_OK) return r;
@@ -922,8 +1008,7 @@ rs_status poa_estimate(rs_ctx* ctx, const rs_records* records, int64_t n, double
   double tot;
   memcpy(&tot, ctx->pinned + 1, 8);
   if (nw < 0)
-    return fail(ctx, nw == -2 ? RS_ERR_INVALID : RS_ERR_CAPACITY,
-                "windows exceed n + 2 (requests more than 5 windows apart on average)");
+    return fail(ctx, RS_ERR_INVALID, "a routed row has a negative or non-finite completion time");
   *n_windows_inout = nw;
   *poa_total_host = tot;
   const int64_t k = std::min(cap, nw);

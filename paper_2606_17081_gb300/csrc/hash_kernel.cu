@@ -144,6 +144,50 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
   return cudaGetLastError();
 }
 
+// The largest number of full blocks of any request of the jobs (offsets
+// only): atomicMax into *nbmax, which the caller clears.
+__global__ void __launch_bounds__(256) k_nbmax(const HashJob* __restrict__ jobs, int njobs,
+                                               int64_t total_req, int64_t* __restrict__ nbmax) {
+  __shared__ HashJob s_jobs[HASH_MAX_JOBS];
+  __shared__ int64_t s_max[8];
+  for (int j = threadIdx.x; j < njobs; j += blockDim.x) s_jobs[j] = jobs[j];
+  __syncthreads();
+  int64_t m = 0;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < total_req;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    const HashJob& J = s_jobs[find_job(s_jobs, njobs, r)];
+    const int64_t i = r - J.req_base;
+    const int64_t nb = (__ldg(J.offsets + i + 1) - __ldg(J.offsets + i)) >> 4;
+    m = nb > m ? nb : m;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const int64_t v = __shfl_xor_sync(FULL_MASK, m, o);
+    m = v > m ? v : m;
+  }
+  if ((threadIdx.x & 31) == 0) s_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int64_t x = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); w++) x = s_max[w] > x ? s_max[w] : x;
+    if (x > 0) atomicMax(reinterpret_cast<unsigned long long*>(nbmax), (unsigned long long)x);
+  }
+}
+
+cudaError_t launch_nbmax(const HashJob* jobs_dev, int njobs, int64_t total_req, int64_t* nbmax,
+                         cudaStream_t st) {
+  if (total_req <= 0) return cudaSuccess;
+  if (njobs < 1 || njobs > HASH_MAX_JOBS) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  int64_t nblk = (total_req + 255) / 256;
+  if (nblk > (int64_t)sms * 4) nblk = (int64_t)sms * 4;
+  k_nbmax<<<(unsigned)nblk, 256, 0, st>>>(jobs_dev, njobs, total_req, nbmax);
+  return cudaGetLastError();
+}
+
 // Duplicate block hashes within one prompt (a 64-bit collision, which the
 // simulation reports as RS_ERR_COLLISION at that request): flags[r] = 1 when
 // two blocks of request r share a chained hash, 0 when none do, 2 when the

@@ -25,31 +25,49 @@ void* g_scratch_ptr[kMaxDevices] = {};   // device address of g_poa_scratch per 
 
 size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Carve-up of the static array for n rows of W workers (byte offsets).
+// Carve-up of the static array for n rows of W workers (byte offsets): the
+// fixed entries and the row arrays first, then the window arrays, which get
+// every byte that remains (win slots each).
 struct NoallocLayout {
-  size_t prob, total, nwin, cost, order, asg, wkey, wstart, wfill, wnum, wopt, wcnt, wstat,
-      tstat, end;
+  size_t prob, total, nwin, tstat, cost, order, asg, wkey, wstart, wfill, wnum, wopt, wcnt, wstat,
+      end;
+  int64_t win;   // window slots (< 1: the rows leave no room)
 };
+
+// Accepted sizes: n (8 W + 60) + NOALLOC_SLACK <= RS_NOALLOC_POA_BYTES, i.e. per
+// row its cost row (8 W), order, assignment and window key (12) and six
+// window entries (48) for n of the windows; the slack covers the fixed
+// entries, two more windows and the 256-byte alignment of 14 arrays.
+constexpr size_t NOALLOC_SLACK = 4096;
+
+bool noalloc_fits(int64_t n, int W) {
+  const size_t rows = (size_t)(n > 0 ? n : 1);
+  return rows <= ((size_t)RS_NOALLOC_POA_BYTES - NOALLOC_SLACK) / (size_t)(8 * W + 60);
+}
 
 NoallocLayout layout(int64_t n, int W) {
   NoallocLayout L;
   const size_t rows = (size_t)(n > 0 ? n : 1);
-  const size_t win = rows + 2;
   size_t o = 0;
   L.prob = o; o = up256(o + sizeof(PoaProblem));
   L.total = o; o = up256(o + 8);
   L.nwin = o; o = up256(o + 8);
+  L.tstat = o; o = up256(o + 8);
   L.cost = o; o = up256(o + rows * (size_t)W * 8);
   L.order = o; o = up256(o + rows * 4);
   L.asg = o; o = up256(o + rows * 4);
   L.wkey = o; o = up256(o + rows * 4);
+  // six window arrays of win entries (wstart one more), each 256-aligned
+  const size_t room = (size_t)RS_NOALLOC_POA_BYTES > o + 6 * 256 + 8
+                          ? (size_t)RS_NOALLOC_POA_BYTES - o - 6 * 256 - 8 : 0;
+  L.win = (int64_t)(room / 48);
+  const size_t win = (size_t)(L.win > 0 ? L.win : 0);
   L.wstart = o; o = up256(o + (win + 1) * 8);
   L.wfill = o; o = up256(o + win * 8);
   L.wnum = o; o = up256(o + win * 8);
   L.wopt = o; o = up256(o + win * 8);
   L.wcnt = o; o = up256(o + win * 8);
   L.wstat = o; o = up256(o + win * 8);
-  L.tstat = o; o = up256(o + 8);
   L.end = o;
   return L;
 }
@@ -95,8 +113,9 @@ extern "C" rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records
   const rs_records& u = *records;
   if (n > 0 && (!u.worker || !u.completion || !u.ttft || !u.nbt || !u.n_frozen || !u.prefix))
     return RS_ERR_INVALID;
+  if (!noalloc_fits(n, cfg->W)) return RS_ERR_CAPACITY;
   const NoallocLayout L = layout(n, cfg->W);
-  if (L.end > (size_t)RS_NOALLOC_POA_BYTES) return RS_ERR_CAPACITY;
+  if (L.end > (size_t)RS_NOALLOC_POA_BYTES || L.win < (n > 0 ? n : 1) + 2) return RS_ERR_CAPACITY;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RS_ERR_CUDA;
   void* base = nullptr;
@@ -120,16 +139,11 @@ extern "C" rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records
   pr.n = n;
   pr.scratch_base = 0;
   pr.win_base = 0;
-  pr.win_cap = n + 2;
+  pr.win_cap = L.win;   // windows past this give *n_windows_dev = -1
   PoaProblem* dprob = reinterpret_cast<PoaProblem*>(s + L.prob);
   k_noalloc_setup<<<1, 1, 0, st>>>(pr, dprob);
   if (cudaGetLastError() != cudaSuccess) return RS_ERR_CUDA;
-  ModelConsts mc;
-  mc.lat_a = cfg->lat_a; mc.lat_b = cfg->lat_b; mc.lat_d = cfg->lat_d; mc.w_c = cfg->w_c;
-  mc.itl = cfg->itl; mc.dt = cfg->dt; mc.alpha = cfg->alpha; mc.theta1 = cfg->theta1;
-  mc.theta2 = cfg->theta2; mc.eps_frac = cfg->eps_frac; mc.poa_window = cfg->poa_window;
-  mc.cap = cfg->cap; mc.hyst_k = cfg->hyst_k; mc.W = cfg->W; mc.write_cost = 0;
-  for (int r = 0; r < 3; r++) { mc.regime_tau[r] = cfg->regime_tau[r]; mc.regime_omega[r] = cfg->regime_omega[r]; }
+  const ModelConsts mc = make_consts(*cfg);
   PoaBuffers b;
   b.rec = u;
   b.cost = reinterpret_cast<double*>(s + L.cost);

@@ -618,6 +618,46 @@ __global__ void __launch_bounds__(NT_POA) k_poa_total(int nprob, PoaBuffers b,
   }
 }
 
+// Last window of each problem: the largest floor(completion / window) over
+// its routed rows (-1 when none is routed).  The host sizes the
+// window-indexed scratch from it before k_poa_prep, so that every window the
+// records span has a slot.  A completion that is negative or not finite is
+// skipped here (k_poa_prep reports it as an overflow); indices are clamped
+// at 2^62.
+__global__ void __launch_bounds__(NT_POA) k_poa_span(const PoaProblem* __restrict__ probs,
+                                                     rs_records rec, double window,
+                                                     long long* __restrict__ maxw) {
+  __shared__ long long red[NT_POA / 32];
+  const PoaProblem pr = probs[blockIdx.x];
+  long long mx = -1;
+  for (int64_t q = threadIdx.x; q < pr.n; q += NT_POA) {
+    const int64_t r = pr.rec_base + q;
+    if (rec.worker[r] < 0) continue;
+    const double w = floor(__ddiv_rn(rec.completion[r], window));
+    if (!(w >= 0.0)) continue;
+    const long long k = w < 4.611686018427387904e18 ? (long long)w : (1ll << 62);
+    mx = k > mx ? k : mx;
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const long long v = __shfl_xor_sync(FULL_MASK, mx, o);
+    mx = v > mx ? v : mx;
+  }
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long m = red[0];
+    for (int w = 1; w < NT_POA / 32; w++) m = red[w] > m ? red[w] : m;
+    maxw[blockIdx.x] = m;
+  }
+}
+
+cudaError_t launch_poa_span(const PoaProblem* d_prob, int nprob, const rs_records& rec,
+                            double window, long long* maxw, cudaStream_t st) {
+  if (nprob <= 0) return cudaSuccess;
+  k_poa_span<<<nprob, NT_POA, 0, st>>>(d_prob, rec, window, maxw);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
                        const ModelConsts& mc, cudaStream_t st) {
   if (nprob <= 0) return cudaSuccess;

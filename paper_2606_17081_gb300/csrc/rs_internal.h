@@ -56,6 +56,10 @@ struct TableGeom {
 
 TableGeom table_geom(int64_t K);
 
+struct ModelConsts;
+// The kernels' model constants from a configuration (every field set).
+ModelConsts make_consts(const rs_config& c);
+
 // One simulated replica as the kernel sees it.
 struct SimDesc {
   const int64_t* offsets;
@@ -129,6 +133,9 @@ struct HashJob {
 constexpr int HASH_MAX_JOBS = 64;
 cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_req, uint64_t seed,
                               int64_t* nbmax_out, cudaStream_t st);
+// *nbmax = max(*nbmax, the largest floor(L/16) over the jobs' requests).
+cudaError_t launch_nbmax(const HashJob* jobs_dev, int njobs, int64_t total_req, int64_t* nbmax,
+                         cudaStream_t st);
 // flags[r] = 1 when two blocks of request r (numbered over the launch's jobs)
 // share a chained hash, 0 when none do, 2 when it has more than nbmax blocks
 // (not checked).  Fails with cudaErrorInvalidValue when one warp's set of
@@ -174,6 +181,9 @@ cudaError_t launch_sweep_knee(const int32_t* worker, const double* ttft, const i
                               int n_sweeps, int pct, double theta, double* stat, double* d1,
                               double* d2, double* knee_load, int32_t* knee_index,
                               cudaStream_t st);
+// maxw[p] = last window index of problem p's routed rows (-1 if none).
+cudaError_t launch_poa_span(const PoaProblem* d_prob, int nprob, const rs_records& rec,
+                            double window, long long* maxw, cudaStream_t st);
 cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
                        const ModelConsts& mc, cudaStream_t st);
 

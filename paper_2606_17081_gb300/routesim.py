@@ -42,7 +42,7 @@ class rs_config(C.Structure):
 
 class rs_trace(C.Structure):
     _fields_ = [("tokens", C.c_void_p), ("offsets", C.c_void_p), ("release", C.c_void_p),
-                ("out_len", C.c_void_p), ("n_req", C.c_int64)]
+                ("out_len", C.c_void_p), ("n_req", C.c_int64), ("hashes", C.c_void_p)]
 
 
 class rs_replica_params(C.Structure):
@@ -294,16 +294,20 @@ def poa_estimate_noalloc(cfg: rs_config, records: rs_records, n: int, numer_dev,
 
 @dataclass
 class TraceBuffers:
-    """A trace's arrays in one memory space, kept alive with its descriptor."""
+    """A trace's arrays in one memory space, kept alive with its descriptor.
+    tokens None: the trace is given by its block hashes (`hashes`)."""
     tokens: object
     offsets: object
     release: object
     out_len: object
     n_req: int
+    hashes: object = None
 
     def desc(self) -> rs_trace:
-        return rs_trace(_ptr(self.tokens).value, _ptr(self.offsets).value,
-                        _ptr(self.release).value, _ptr(self.out_len).value, self.n_req)
+        tok = _ptr(self.tokens)
+        return rs_trace(tok.value if tok is not None else None, _ptr(self.offsets).value,
+                        _ptr(self.release).value, _ptr(self.out_len).value, self.n_req,
+                        _ptr(self.hashes).value if self.tokens is None else None)
 
 
 def device_trace(trace, device="cuda") -> TraceBuffers:

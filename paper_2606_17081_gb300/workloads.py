@@ -14,6 +14,19 @@ reproduced; prompts are uniform token ids with shared-prefix groups.
 Token layout: one int32 array, requests stored back to back (CSR `offsets`,
 int64, n+1 entries), the array padded with zeros to a multiple of 4 entries so
 that 16-byte vector loads never leave it.
+
+Two ways of drawing the tokens:
+  "stream"   one numpy draw for the whole trace (every workload but the largest);
+  "counter"  for traces too large to draw or hold on the host (the W = 64
+             workload: about 2.7 G tokens per trace).  The random suffix token
+             at position x of the trace's token array is the (x+1)-th output
+             of SplitMix64 (Steele, Lea & Flood, OOPSLA 2014) from a per-trace
+             key, reduced to the vocabulary by Lemire's multiply-shift
+             ((z >> 32) * vocab) >> 32; prefix tokens come from the group's
+             prefix, as in "stream".  Any range of positions can then be
+             produced on its own: on the host with numpy (`TraceMeta.tokens`)
+             or on the device with torch integer ops (`TraceMeta.fill_device`),
+             bit for bit the same.
 """
 from __future__ import annotations
 
@@ -52,6 +65,9 @@ class TraceSpec:
     out_min: int = 1
     out_max: int = 4096
     rate: Optional[float] = None      # Poisson arrival rate (req/s); None = closed loop
+    tokens: str = "stream"            # "stream" | "counter" (see the module docstring)
+    n_meta: Optional[int] = None      # "counter": requests whose lengths etc. are drawn (>= n_req),
+                                      # so that a shorter n_req gives a prefix of the full trace
 
 
 @dataclass
@@ -91,6 +107,8 @@ def _lengths(rng, kind, median, sigma, lo, hi, n):
 
 def make_trace(spec: TraceSpec, seed: int) -> Trace:
     """Draw one trace.  Same (spec, seed) -> same bytes on any machine with numpy."""
+    if spec.tokens == "counter":
+        return trace_meta(spec, seed).trace(spec.n_req)
     rng = np.random.default_rng([int(seed), 0x5EED7ACE])
     n = int(spec.n_req)
     G = int(spec.n_groups)
@@ -118,6 +136,151 @@ def make_trace(spec: TraceSpec, seed: int) -> Trace:
         o = int(offsets[i])
         tokens[o:o + k] = prefixes[g][:k]
     return Trace(tokens, offsets, release.astype(np.float64), O.astype(np.int32), group)
+
+
+# SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): state_n = key + n * GAMMA, and
+# output_n is the state passed through its finalizer (two xor-shift-multiply
+# rounds and a last xor-shift).
+SM_GAMMA = 0x9E3779B97F4A7C15
+SM_M1 = 0xBF58476D1CE4E5B9
+SM_M2 = 0x94D049BB133111EB
+
+
+def sm_output_np(x: np.ndarray, key: int) -> np.ndarray:
+    """SplitMix64 outputs number x + 1 (x >= 0, int64 array) from `key`."""
+    z = (np.asarray(x).astype(np.uint64) + np.uint64(1)) * np.uint64(SM_GAMMA) + np.uint64(key)
+    z = (z ^ (z >> np.uint64(30))) * np.uint64(SM_M1)
+    z = (z ^ (z >> np.uint64(27))) * np.uint64(SM_M2)
+    return z ^ (z >> np.uint64(31))
+
+
+def _sm_tokens_np(x: np.ndarray, key: int, vocab: int) -> np.ndarray:
+    """Suffix tokens at trace positions x (int64): Lemire reduction of the
+    high 32 bits of SplitMix64 output x + 1."""
+    z = sm_output_np(x, key)
+    return (((z >> np.uint64(32)) * np.uint64(vocab)) >> np.uint64(32)).astype(np.int32)
+
+
+def _s64(c: int) -> int:
+    """A 64-bit constant as the signed value with the same bits."""
+    return c - (1 << 64) if c >= (1 << 63) else c
+
+
+def _sm_tokens_torch(x, key: int, vocab: int):
+    """The same on int64 torch tensors: products wrap modulo 2^64 and shifts
+    are made logical by masking the sign-extended bits."""
+    def lsr(z, k):
+        return (z >> k) & ((1 << (64 - k)) - 1)
+    z = (x + 1) * _s64(SM_GAMMA) + _s64(key)
+    z = (z ^ lsr(z, 30)) * _s64(SM_M1)
+    z = (z ^ lsr(z, 27)) * _s64(SM_M2)
+    z = z ^ lsr(z, 31)
+    import torch
+    return ((lsr(z, 32) * vocab) >> 32).to(torch.int32)
+
+
+@dataclass
+class TraceMeta:
+    """A "counter" trace without its tokens: per-request lengths, groups and
+    times for n_meta requests, the groups' prefix tokens (`pool`, CSR by
+    `pool_off`) and the suffix stream's key.  Tokens of any position range
+    come from `tokens` (host) or `fill_device` (device), identically."""
+    offsets: np.ndarray   # int64 [n+1]
+    release: np.ndarray   # float64 [n]
+    out_len: np.ndarray   # int32 [n]
+    group: np.ndarray     # int32 [n]
+    kpref: np.ndarray     # int64 [n]: leading tokens taken from the group's prefix
+    pool: np.ndarray      # int32: the groups' prefixes back to back
+    pool_off: np.ndarray  # int64 [G+1]
+    key: int
+    vocab: int
+
+    @property
+    def n_req(self) -> int:
+        return int(self.offsets.shape[0] - 1)
+
+    def tokens(self, x0: int, x1: int) -> np.ndarray:
+        """int32 tokens at trace positions x0 .. x1-1 (positions past the last
+        request hold suffix-stream values)."""
+        out = _sm_tokens_np(np.arange(x0, x1, dtype=np.int64), self.key, self.vocab)
+        # the leading kpref[i] tokens of every request in range come from its prefix
+        i0 = max(int(np.searchsorted(self.offsets, x0, side="right")) - 1, 0)
+        i1 = min(int(np.searchsorted(self.offsets, x1, side="left")), self.n_req)
+        for i in range(i0, i1):
+            a = int(self.offsets[i])
+            b = a + int(self.kpref[i])
+            lo, hi = max(a, x0), min(b, x1)
+            if lo < hi:
+                src = int(self.pool_off[int(self.group[i])]) + (lo - a)
+                out[lo - x0:hi - x0] = self.pool[src:src + (hi - lo)]
+        return out
+
+    def trace(self, n: int) -> Trace:
+        """The first n requests with their tokens (host memory)."""
+        n = min(int(n), self.n_req)
+        end = int(self.offsets[n])
+        toks = np.zeros(end + ((-end) % 4), np.int32)
+        step = 1 << 24
+        for x0 in range(0, end, step):
+            x1 = min(end, x0 + step)
+            toks[x0:x1] = self.tokens(x0, x1)
+        return Trace(toks, self.offsets[: n + 1].copy(), self.release[:n].copy(),
+                     self.out_len[:n].copy(), self.group[:n].copy())
+
+    def device(self, device="cuda") -> dict:
+        """The tables `fill_device` reads, as device tensors."""
+        import torch
+        return {k: torch.from_numpy(getattr(self, k)).to(device)
+                for k in ("offsets", "group", "kpref", "pool", "pool_off")}
+
+    def fill_device(self, dev: dict, x0: int, x1: int, out, step: int = 1 << 25) -> None:
+        """Writes the tokens of positions x0 .. x1-1 into the int32 device
+        tensor `out` (at least x1 - x0 entries) with torch integer ops, in
+        steps of `step` positions."""
+        import torch
+        offs, grp, kp = dev["offsets"], dev["group"], dev["kpref"]
+        pool, poff = dev["pool"], dev["pool_off"]
+        n = self.n_req
+        for a in range(x0, x1, step):
+            b = min(x1, a + step)
+            x = torch.arange(a, b, dtype=torch.int64, device=offs.device)
+            req = (torch.searchsorted(offs, x, right=True) - 1).clamp_(max=n - 1)
+            p = x - offs[req]
+            k = kp[req]
+            idx = poff[grp[req].long()] + torch.minimum(p, k - 1).clamp_(min=0)
+            pre = pool[idx.clamp_(max=pool.numel() - 1)]
+            suf = _sm_tokens_torch(x, self.key, self.vocab)
+            out[a - x0:b - x0] = torch.where(p < k, pre, suf)
+
+
+def trace_meta(spec: TraceSpec, seed: int) -> TraceMeta:
+    """Lengths, groups, times and prefix tokens of a "counter" trace, drawn for
+    spec.n_meta (default n_req) requests; the suffix tokens are never drawn
+    here.  Same (spec, seed) -> same values on any machine with numpy."""
+    rng = np.random.default_rng([int(seed), 0x5EED7ACE])
+    n = int(spec.n_meta if spec.n_meta is not None else spec.n_req)
+    G = int(spec.n_groups)
+    plen = rng.integers(spec.prefix_min, spec.prefix_max + 1, size=G).astype(np.int64)
+    pool = rng.integers(0, spec.vocab, size=int(plen.sum()), dtype=np.int32)
+    pool_off = np.zeros(G + 1, np.int64)
+    np.cumsum(plen, out=pool_off[1:])
+    if spec.zipf_s is None:
+        group = rng.integers(0, G, size=n).astype(np.int32)
+    else:
+        w = 1.0 / np.power(np.arange(1, G + 1, dtype=np.float64), spec.zipf_s)
+        group = rng.choice(G, size=n, p=w / w.sum()).astype(np.int32)
+    L = _lengths(rng, spec.len_kind, spec.len_median, spec.len_sigma, spec.len_min, spec.len_max, n)
+    O = _lengths(rng, spec.out_kind, spec.out_median, spec.out_sigma, spec.out_min, spec.out_max, n)
+    if spec.rate is None:
+        release = np.zeros(n, np.float64)
+    else:
+        release = np.cumsum(rng.exponential(1.0 / spec.rate, size=n))
+    key = int(rng.integers(0, 1 << 63, dtype=np.int64)) * 2 + int(rng.integers(0, 2))
+    offsets = np.zeros(n + 1, np.int64)
+    np.cumsum(L, out=offsets[1:])
+    kpref = np.minimum(plen[group], L).astype(np.int64)
+    return TraceMeta(offsets, release.astype(np.float64), O.astype(np.int32), group, kpref, pool,
+                     pool_off, key, int(spec.vocab))
 
 
 @dataclass
@@ -157,6 +320,18 @@ class Plan:
     def traces(self):
         return [make_trace(self.spec, s) for s in self.trace_seeds]
 
+    def metas(self):
+        """The traces without tokens ("counter" specs only), each cut to
+        spec.n_req requests."""
+        out = []
+        for s in self.trace_seeds:
+            m = trace_meta(self.spec, s)
+            n = self.spec.n_req
+            out.append(TraceMeta(m.offsets[: n + 1].copy(), m.release[:n].copy(),
+                                 m.out_len[:n].copy(), m.group[:n].copy(), m.kpref[:n].copy(),
+                                 m.pool, m.pool_off, m.key, m.vocab))
+        return out
+
 
 TINY_SPEC = TraceSpec(n_req=512, len_kind="uniform", len_min=64, len_max=512,
                       n_groups=16, prefix_min=256, prefix_max=256, zipf_s=None,
@@ -165,7 +340,7 @@ P2D_SPEC = TraceSpec(n_req=20000)
 P5D_SPEC = TraceSpec(n_req=50000)
 GRID_SPEC = TraceSpec(n_req=10000)
 LARGE_SPEC = TraceSpec(n_req=1_000_000, len_median=2048.0, len_max=32768, n_groups=1024,
-                       zipf_s=1.0)
+                       zipf_s=1.0, tokens="counter", n_meta=1_000_000)
 
 
 def plan(name: str, n_req: Optional[int] = None, replicas: Optional[list] = None) -> Plan:

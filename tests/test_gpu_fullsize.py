@@ -131,6 +131,21 @@ def test_p5d_full_size_prefix_of_sampled_replicas():
         o = oracle_run(cfg, traces[r.trace], rr)
         _prefix_equal(_rows(t, int(base[k]), N, p.W), o, p.W)
     assert sum(x.regime_switches for x in res) > 0
+    # one replica whole (C = 64, tau = 1: sampled decisions, controller on),
+    # its PoA included
+    k = 101
+    r = p.replicas[k]
+    assert r.tau == 1.0 and r.controller == 1
+    g, o = _whole_equal(p, ctx, traces, res, t, base, k,
+                        extra=("sampled", "near_ties", "exact_ties", "near_boundary", "ticks",
+                               "regime_switches", "final_regime", "max_regime"))
+    res_k = res[k].as_dict()
+    assert res_k["sampled"] > 0 and res_k["ticks"] > 0
+    assert list(res_k["ticks_in_regime"]) == list(o["summary"]["ticks_in_regime"])
+    cfg = oracle_cfg(ctx, theta1=p.theta1, theta2=p.theta2)
+    num, opt, cnt, tot = O.poa(cfg, o)
+    assert res_k["n_windows"] == num.size
+    assert abs(res_k["poa_total"] - tot) <= 1e-4 * tot
     ctx.close()
 
 
