@@ -1,10 +1,11 @@
 """The multi-rank logic of bench.py, run as two gloo ranks on the CPU.
 
-Replicas are independent, so under torchrun every rank simulates its own
-replica grid (weak scaling) and the ranks meet only to take the slowest rank's
-time.  Checked here: each rank draws its own traces and routing seeds, the
-grids have the same shape, the timing reduction is the maximum over ranks, and
-a rank other than 0 prints nothing.
+Replicas are independent, so under torchrun the ranks split the replicas of
+the one plan into contiguous ranges (strong scaling, no data-path collective)
+and meet only to take the slowest rank's time.  Checked here: the ranks'
+ranges cover the plan exactly once and each rank's replicas are the plan's
+(same traces, seeds and parameters), the timing reduction is the maximum over
+ranks, and a rank other than 0 prints nothing.
 """
 import contextlib
 import io
@@ -32,15 +33,16 @@ def _rank_main(rank: int, world: int, port: int, out_dir: str):
     import bench
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
-        p = bench._plan(rank, n_req=50)
+        p, lo, hi = bench._plan("grid", rank, world, n_req=50)
         # rank r's step time is r + 1 ms, its end-to-end time 10 - r s
         ms, e2e = bench._max_over_ranks([rank + 1.0, 10.0 - rank], "cpu")
         buf = io.StringIO()
         with contextlib.redirect_stdout(buf):
             if rank != 0:
-                bench.run_reference(type("A", (), {"steps": 1, "warmup": 0})())
-        rec = {"trace_seeds": p.trace_seeds, "seeds": [r.seed for r in p.replicas],
-               "shape": [(r.C, r.policy, r.omega, r.tau, r.n_req, r.trace) for r in p.replicas],
+                bench.run_reference(type("A", (), {"steps": 1, "warmup": 0, "workload": "tiny"})())
+        rec = {"range": [lo, hi],
+               "reps": [(p.trace_seeds[r.trace], r.seed, r.C, r.policy, r.omega, r.tau, r.n_req)
+                        for r in p.replicas],
                "max": [ms, e2e], "printed": buf.getvalue()}
         with open(os.path.join(out_dir, f"rank{rank}.json"), "w") as f:
             json.dump(rec, f)
@@ -66,10 +68,15 @@ def test_two_gloo_ranks_shard_replicas_and_take_max_time(tmp_path):
     assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
     r0 = json.loads((tmp_path / "rank0.json").read_text())
     r1 = json.loads((tmp_path / "rank1.json").read_text())
-    # same grid shape, disjoint traces and routing seeds
-    assert r0["shape"] == r1["shape"]
-    assert not set(r0["trace_seeds"]) & set(r1["trace_seeds"])
-    assert not set(r0["seeds"]) & set(r1["seeds"])
+    # the ranks' ranges partition the plan, and hold exactly its replicas
+    sys.path.insert(0, ROOT)
+    from paper_2606_17081_gb300 import workloads as wk
+    full = wk.plan("grid", n_req=50)
+    assert r0["range"][0] == 0 and r0["range"][1] == r1["range"][0]
+    assert r1["range"][1] == len(full.replicas) and r0["range"][1] > 0
+    want = [[full.trace_seeds[r.trace], r.seed, r.C, r.policy, r.omega, r.tau, r.n_req]
+            for r in full.replicas]
+    assert [list(x) for x in r0["reps"] + r1["reps"]] == want
     # the reported times are the slowest rank's
     assert r0["max"] == r1["max"] == [2.0, 10.0]
     # the reference arm prints only on rank 0
