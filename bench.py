@@ -380,8 +380,8 @@ def _aux_probe(rs, n_route: int = 4096, n_probe: int = 60000, reps: int = 5) -> 
     batch, then probes; the probe kernel's time is the call's device time
     (CUDA events) less a block-hash call on the same batch.  lookups = sum
     over (request, worker) of min(m_ij + 1, nb_i); algorithmic bytes = 32 B
-    per lookup (one bucket sector) + 8 B per block hash read + 4 B per m_ij
-    written."""
+    per lookup (one bucket sector) + 8 B per block hash (read once, then
+    reused by the request's W pairs) + 4 B per m_ij written."""
     import torch
     from paper_2606_17081_gb300 import workloads as wk
     p = wk.plan("large", n_req=n_route + n_probe)
@@ -412,7 +412,7 @@ def _aux_probe(rs, n_route: int = 4096, n_probe: int = 60000, reps: int = 5) -> 
     nb = (np.diff(offs.cpu().numpy()) // 16)[:, None]
     lookups = int(np.minimum(pre + 1, nb).sum())
     kern = min(tp) - min(th)
-    alg = 32.0 * lookups + 8.0 * float(nb.sum()) * W + 4.0 * m * W
+    alg = 32.0 * lookups + 8.0 * float(nb.sum()) + 4.0 * m * W
     peak, kind = _peaks()
     return {"workers": W, "cache_blocks": K, "table_bytes": _table_bytes(K) * W,
             "routed": n_route, "probed": m, "pairs": m * W, "lookups": lookups,

@@ -236,36 +236,152 @@ cudaError_t launch_clear_tables(uint64_t* keys, uint32_t* stamp, size_t nslots, 
   return cudaGetLastError();
 }
 
-// Batch probe (route_probe): one thread per (request, worker) pair walks the
-// request's blocks in order through the worker's table until the first one
-// absent: m_ij + 1 bucket reads (64 bytes each, two 32-byte sectors) and
-// m_ij + 1 hash reads, the first-miss prefix of S2.  The tables are only
-// read, so all pairs run at once; pairs are numbered request-major, so the
-// threads of a warp share requests' offsets and hash lines.
-__global__ void __launch_bounds__(256) k_probe_batch(RouterState s,
-                                                     const int64_t* __restrict__ offsets,
-                                                     const uint64_t* __restrict__ hashes,
-                                                     int64_t n_req, int W, TableGeom g,
-                                                     int32_t* __restrict__ prefix_out) {
+// Batch probe (route_probe): the first-miss prefix m_ij of S2 for every
+// (request, worker) pair against one snapshot of the tables (only read).
+//
+// A pair walks its request's blocks in order until the first one absent from
+// the worker's table; a walk of m_ij + 1 dependent lookups per thread would
+// leave a warp waiting for its longest walk with most lanes idle (most pairs
+// miss at block 0, a few follow a shared prefix for many blocks).  So a warp
+// takes 64 consecutive pairs (request-major, two per lane) and runs them
+// together in steps: at each step the a pairs still open share the warp's 64
+// lookup slots, each pair the next `share` blocks of its walk, share =
+// min(64 / a, 2^step) (one block per pair at the first step, doubling as the
+// open pairs thin out, so no pair looks up more than about twice the blocks
+// its answer needs); both slots of a lane are issued before either is used.
+// A pair's window ends its walk at its first absent block (or the prompt's
+// end), else the walk moves on by `share`.  Lookups: one 64-byte bucket (two
+// 32-byte sectors) and one 8-byte hash each.
+constexpr int PROBE_NT = 256;
+
+// Position of the n-th (0-based) set bit of x; x has more than n set bits.
+__device__ __forceinline__ int nth_set_bit64(uint64_t x, int n) {
+  int pos = 0;
+#pragma unroll
+  for (int w = 32; w >= 1; w >>= 1) {
+    const int c = __popcll(x & ((1ull << w) - 1ull));
+    if (n >= c) {
+      n -= c;
+      x >>= w;
+      pos += w;
+    }
+  }
+  return pos;
+}
+
+struct ProbePair {
+  int64_t hbase;   // index of the request's first block hash
+  int32_t start;   // next block of the walk
+  int32_t nb;      // full blocks of the request
+  int32_t j;       // worker
+  int32_t pad;
+};
+
+__global__ void __launch_bounds__(PROBE_NT) k_probe_batch(RouterState s,
+                                                          const int64_t* __restrict__ offsets,
+                                                          const uint64_t* __restrict__ hashes,
+                                                          int64_t n_req, int W, TableGeom g,
+                                                          int32_t* __restrict__ prefix_out) {
+  __shared__ ProbePair sp[PROBE_NT / 32][64];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  ProbePair* P = sp[warp];
   const int64_t total = n_req * W;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += stride) {
-    const int64_t i = e / W;
-    const int j = (int)(e - i * W);
-    const int64_t o0 = __ldg(offsets + i);
-    const int64_t nb = (__ldg(offsets + i + 1) - o0) >> 4;
-    const uint64_t* h = hashes + (o0 >> 4);
-    TableView t;
-    t.keys = s.keys + (size_t)j * g.slots;
-    t.stamp = s.stamp + (size_t)j * g.slots;
-    t.log = s.log + (size_t)j * g.R;
-    t.fexp = nullptr;
-    t.bmask = g.bmask;
-    t.rmask = g.rmask;
-    int64_t m = 0;
-    int err = 0;
-    while (m < nb && table_find(t, __ldg(h + m), &err) != SLOT_NONE) m++;
-    prefix_out[e] = (int32_t)(m < 0x7FFFFFFF ? m : 0x7FFFFFFF);
+  const int64_t ngroups = (total + 63) >> 6;
+  const int64_t gw = ((int64_t)blockIdx.x * PROBE_NT + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * PROBE_NT) >> 5;
+  for (int64_t grp = gw; grp < ngroups; grp += nw) {
+    const int64_t e0 = grp << 6;
+    // this lane's two pairs: slots lane and lane + 32
+    int32_t m[2] = {0, 0};
+    bool open[2] = {false, false};
+#pragma unroll
+    for (int h = 0; h < 2; h++) {
+      const int q = lane + 32 * h;
+      const int64_t e = e0 + q;
+      ProbePair pp{0, 0, 0, 0, 0};
+      if (e < total) {
+        const int64_t i = e / W;
+        const int64_t o0 = __ldg(offsets + i);
+        const int64_t nbl = (__ldg(offsets + i + 1) - o0) >> 4;
+        pp.hbase = o0 >> 4;
+        pp.nb = (int32_t)(nbl < 0x7FFFFFFF ? nbl : 0x7FFFFFFF);
+        pp.j = (int32_t)(e - i * W);
+        open[h] = pp.nb > 0;
+      }
+      P[q] = pp;
+    }
+    uint64_t act = (uint64_t)__ballot_sync(FULL_MASK, open[0]) |
+                   ((uint64_t)__ballot_sync(FULL_MASK, open[1]) << 32);
+    for (int step = 0; act != 0ull; step++) {
+      __syncwarp();
+      const int a = __popcll(act);
+      int share = 64 / a;
+      if (step < 6 && share > (1 << step)) share = 1 << step;
+      // lookups of slots lane and lane + 32: pair (its rank r among the open
+      // ones) and block start + off
+      bool miss[2] = {false, false};
+      bool live[2] = {false, false};
+      uint64_t hk[2] = {0ull, 0ull};
+      TableView tv[2];
+#pragma unroll
+      for (int h = 0; h < 2; h++) {
+        const int q = lane + 32 * h;
+        const int r = q / share;
+        if (r < a) {
+          const int pi = nth_set_bit64(act, r);
+          const ProbePair pp = P[pi];
+          const int64_t k = (int64_t)pp.start + (q - r * share);
+          live[h] = true;
+          if (k >= pp.nb) {
+            miss[h] = true;   // past the prompt: the walk ends at nb
+          } else {
+            hk[h] = __ldg(hashes + pp.hbase + k);
+            const size_t wj = (size_t)pp.j;
+            tv[h].keys = s.keys + wj * g.slots;
+            tv[h].stamp = s.stamp + wj * g.slots;
+            tv[h].log = s.log + wj * g.R;
+            tv[h].fexp = nullptr;
+            tv[h].bmask = g.bmask;
+            tv[h].rmask = g.rmask;
+          }
+        }
+      }
+      int err = 0;
+#pragma unroll
+      for (int h = 0; h < 2; h++)
+        if (live[h] && !miss[h]) miss[h] = table_find(tv[h], hk[h], &err) == SLOT_NONE;
+      const uint64_t mm = (uint64_t)__ballot_sync(FULL_MASK, miss[0]) |
+                          ((uint64_t)__ballot_sync(FULL_MASK, miss[1]) << 32);
+      // each pair's owner closes its walk at the window's first miss, or moves on
+      const uint64_t wmask = share >= 64 ? ~0ull : ((1ull << share) - 1ull);
+#pragma unroll
+      for (int h = 0; h < 2; h++) {
+        const int q = lane + 32 * h;
+        if (!open[h]) continue;
+        const int r = __popcll(act & ((1ull << q) - 1ull));
+        const uint64_t bits = (mm >> (r * share)) & wmask;
+        const int32_t st = P[q].start;
+        if (bits) {
+          m[h] = st + __ffsll((long long)bits) - 1;
+          open[h] = false;
+        } else if (st + share >= P[q].nb) {
+          m[h] = P[q].nb;
+          open[h] = false;
+        }
+      }
+      __syncwarp();   // every lane has read the starts of this step
+#pragma unroll
+      for (int h = 0; h < 2; h++)
+        if (open[h]) P[lane + 32 * h].start += share;
+      act = (uint64_t)__ballot_sync(FULL_MASK, open[0]) |
+            ((uint64_t)__ballot_sync(FULL_MASK, open[1]) << 32);
+    }
+#pragma unroll
+    for (int h = 0; h < 2; h++) {
+      const int64_t e = e0 + lane + 32 * h;
+      if (e < total) prefix_out[e] = m[h];
+    }
+    __syncwarp();
   }
 }
 
@@ -277,10 +393,10 @@ cudaError_t launch_probe_batch(const RouterState& s, const int64_t* offsets, con
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  const int64_t total = n_req * W;
-  int64_t nblk = (total + 255) / 256;
-  if (nblk > (int64_t)sms * 8) nblk = (int64_t)sms * 8;   // 8 x 256 threads resident per SM
-  k_probe_batch<<<(unsigned)nblk, 256, 0, st>>>(s, offsets, hashes, n_req, W, g, prefix_out);
+  const int64_t groups = (n_req * W + 63) / 64;   // 64 pairs per warp
+  int64_t nblk = (groups + PROBE_NT / 32 - 1) / (PROBE_NT / 32);
+  if (nblk > (int64_t)sms * 8) nblk = (int64_t)sms * 8;
+  k_probe_batch<<<(unsigned)nblk, PROBE_NT, 0, st>>>(s, offsets, hashes, n_req, W, g, prefix_out);
   return cudaGetLastError();
 }
 
