@@ -71,10 +71,6 @@ __global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restric
       if (w >= pr.win_cap || w < 0) P.overflow = 1;
       else key = (int)w;
       mx = w > mx ? w : mx;
-      const int nbt = b.rec.nbt[r];
-      double* cr = b.cost + (pr.scratch_base + q) * W;
-      for (int j = 0; j < W; j++)
-        cr[j] = frozen_cost(mc, b.rec.n_frozen[r * W + j], b.rec.prefix[r * W + j], nbt);
     }
     b.wkey[pr.scratch_base + q] = key;
   }
@@ -144,7 +140,14 @@ __global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restric
       for (int v = 0; v < warp; v++)
         for (int e = 0; e < P.wn[v]; e++)
           if (P.wk[v][e] == key) cross += P.wc[v][e];
-      b.order[pr.scratch_base + fill[key] + cross + intra] = (int32_t)q;
+      const int64_t d = pr.scratch_base + fill[key] + cross + intra;
+      b.order[d] = (int32_t)q;
+      // the frozen cost row, stored at the request's sorted position
+      const int64_t r = pr.rec_base + q;
+      const int nbt = b.rec.nbt[r];
+      double* cr = b.cost + d * W;
+      for (int j = 0; j < W; j++)
+        cr[j] = frozen_cost(mc, b.rec.n_frozen[r * W + j], b.rec.prefix[r * W + j], nbt);
     }
     __syncthreads();
     if (leader && key >= 0)
@@ -157,6 +160,8 @@ __global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restric
 
 struct PoaWarpShared {
   int counts[POA_WMAX];
+  double dist[POA_WMAX];                           // shortest-path distances of one augmentation
+  int pred[POA_WMAX];
   double wmin[POA_WMAX][POA_WMAX];
   int wrow[POA_WMAX][POA_WMAX];
   int mv_row[POA_WMAX + 1], mv_to[POA_WMAX + 1];   // requests moved by the last augmentation
@@ -171,28 +176,43 @@ struct PoaWarpShared {
 __device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffers& b,
                                                int64_t scratch_base, int64_t base, int64_t m,
                                                int W, int j, int lane) {
+  // per lane: the cheapest move to each k among its rows (registers: the
+  // loops run over the fixed POA_WMAX with k < W guards)
   double lm[POA_WMAX];
   int lr[POA_WMAX];
-  for (int k = 0; k < W; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
+#pragma unroll
+  for (int k = 0; k < POA_WMAX; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
   for (int64_t r = lane; r < m; r += 32) {
     if (b.asg[base + r] != j) continue;
-    const double* cr = b.cost + (scratch_base + b.order[base + r]) * W;
+    const double* cr = b.cost + (base + r) * W;
     const double cj = cr[j];
-    for (int k = 0; k < W; k++) {
-      const double v = __dsub_rn(cr[k], cj);
-      if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
+#pragma unroll
+    for (int k = 0; k < POA_WMAX; k++) {
+      if (k < W) {
+        const double v = __dsub_rn(cr[k], cj);
+        if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
+      }
     }
   }
-  for (int k = 0; k < W; k++) {
-    double v = lm[k];
-    int rr = lr[k];
-    for (int o = 16; o > 0; o >>= 1) {
-      const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
-      const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
-      if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
+#pragma unroll
+  for (int k = 0; k < POA_WMAX; k++) {
+    if (k < W) {
+      double v = lm[k];
+      int rr = lr[k];
+      for (int o = 16; o > 0; o >>= 1) {
+        const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
+        const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
+        if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
+      }
+      if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
     }
-    if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
   }
+}
+
+// Order-preserving map of a finite double onto uint64 (for integer compares).
+__device__ __forceinline__ uint64_t dorder(double x) {
+  const uint64_t u = (uint64_t)__double_as_longlong(x);
+  return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
 }
 
 struct PoaSolveShared {
@@ -236,7 +256,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
     double num = 0.0, nst = 0.0;
     for (int64_t r = lane; r < m; r += 32) {
       const int q = b.order[base + r];
-      const double* cr = b.cost + (pr.scratch_base + q) * W;
+      const double* cr = b.cost + (base + r) * W;
       nst += cr[b.rec.worker[pr.rec_base + q]];   // the realized assignment's frozen cost
       int best = 0;
       double bc = cr[0];
@@ -271,26 +291,43 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
-        const double* c0 = b.cost + (pr.scratch_base + b.order[base + r0]) * W;
-        if (lane == 0) {
-          double dist[POA_WMAX];
-          int pred[POA_WMAX];
-          for (int k = 0; k < W; k++) { dist[k] = c0[k]; pred[k] = -1; }
-          for (int it = 0; it < W; it++) {
-            bool ch = false;
-            for (int j = 0; j < W; j++)
-              for (int k = 0; k < W; k++) {
-                if (k == j || S.wrow[j][k] < 0) continue;
-                // exact cycles are >= 0; relaxing only on gains above 1e-12 keeps
-                // rounding-level negative cycles from looping the predecessors
-                const double nd = __dadd_rn(dist[j], S.wmin[j][k]);
-                if (nd < dist[k] - 1e-12) { dist[k] = nd; pred[k] = j; ch = true; }
-              }
-            if (!ch) break;
+        const double* c0 = b.cost + (base + r0) * W;
+        // Bellman-Ford from the request's costs, in Jacobi rounds: lane k < W
+        // owns target k and every round reads the previous round's distances
+        // (shortest paths have at most W - 1 edges).  Exact cycles are >= 0;
+        // relaxing only on gains above 1e-12 keeps rounding-level negative
+        // cycles from looping the predecessors.
+        double dk = __longlong_as_double(0x7FF0000000000000ll);
+        int pk = -1;
+        if (lane < W) dk = c0[lane];
+        for (int it = 0; it < W; it++) {
+          double nd = dk;
+          int np = pk, ch = 0;
+#pragma unroll
+          for (int j = 0; j < POA_WMAX; j++) {
+            const double dj = __shfl_sync(FULL_MASK, dk, j);
+            if (j < W && lane < W && j != lane && S.wrow[j][lane] >= 0) {
+              const double v = __dadd_rn(dj, S.wmin[j][lane]);
+              if (v < nd - 1e-12) { nd = v; np = j; ch = 1; }
+            }
           }
-          int tgt = -1;
-          for (int k = 0; k < W; k++)
-            if (S.counts[k] < capw && (tgt < 0 || dist[k] < dist[tgt])) tgt = k;
+          dk = nd;
+          pk = np;
+          if (!__any_sync(FULL_MASK, ch)) break;
+        }
+        // target: the nearest worker with room (ties: lowest index)
+        uint64_t key = ~0ull;
+        if (lane < W && S.counts[lane] < capw) key = dorder(dk);
+        int tl = lane;
+        for (int o = 16; o > 0; o >>= 1) {
+          const uint64_t k2 = __shfl_xor_sync(FULL_MASK, key, o);
+          const int t2 = __shfl_xor_sync(FULL_MASK, tl, o);
+          if (k2 < key || (k2 == key && t2 < tl)) { key = k2; tl = t2; }
+        }
+        if (lane < W) { S.dist[lane] = dk; S.pred[lane] = pk; }
+        __syncwarp();
+        if (lane == 0) {
+          const int tgt = key == ~0ull ? -1 : tl;
           int nmv = 0;
           for (int j = 0; j < W; j++) S.dirty[j] = 0;
           if (tgt < 0) {
@@ -299,8 +336,8 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
             // walk the path back from its end: each edge j -> k moves the
             // request behind S.wrow[j][k] from j to k
             int k = tgt, steps = 0;
-            while (pred[k] >= 0 && steps <= W) {
-              const int j = pred[k];
+            while (S.pred[k] >= 0 && steps <= W) {
+              const int j = S.pred[k];
               const int r = S.wrow[j][k];
               S.mv_row[nmv] = r;
               S.mv_to[nmv++] = k;
@@ -320,25 +357,27 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
               S.counts[tgt]++;
             }
           }
-          // requests that moved in lower their new worker's weights
-          for (int t = 0; t < nmv; t++) {
-            const int r = S.mv_row[t], to = S.mv_to[t];
-            const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
-            const double ct = cr[to];
-            for (int k2 = 0; k2 < W; k2++) {
-              if (k2 == to) continue;
-              const double v = __dsub_rn(cr[k2], ct);
-              const int wr = S.wrow[to][k2];
-              if (wr < 0 || v < S.wmin[to][k2] || (v == S.wmin[to][k2] && r < wr)) {
-                S.wmin[to][k2] = v;
-                S.wrow[to][k2] = r;
-              }
-            }
-          }
           S.nmv = nmv;
         }
         __syncwarp();
         if (S.err) break;
+        // requests that moved in lower their new worker's weights (lane k2
+        // keeps column k2; moves in path order)
+        const int nmv = S.nmv;
+        for (int t = 0; t < nmv; t++) {
+          const int r = S.mv_row[t], to = S.mv_to[t];
+          const int k2 = lane;
+          if (k2 < W && k2 != to) {
+            const double* cr = b.cost + (base + r) * W;
+            const double v = __dsub_rn(cr[k2], cr[to]);
+            const int wr = S.wrow[to][k2];
+            if (wr < 0 || v < S.wmin[to][k2] || (v == S.wmin[to][k2] && r < wr)) {
+              S.wmin[to][k2] = v;
+              S.wrow[to][k2] = r;
+            }
+          }
+        }
+        __syncwarp();
         for (int j = 0; j < W; j++)
           if (S.dirty[j]) poa_edges_from(S, b, pr.scratch_base, base, m, W, j, lane);
         __syncwarp();
@@ -346,9 +385,8 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
     }
     double opt = 0.0;
     for (int64_t r = lane; r < m; r += 32) {
-      const int q = b.order[base + r];
       const int a = b.asg[base + r];
-      opt += a >= 0 ? b.cost[(pr.scratch_base + q) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
+      opt += a >= 0 ? b.cost[(base + r) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
     }
     opt = warp_sum(opt);
     if (lane == 0) {
@@ -392,14 +430,25 @@ __device__ __forceinline__ void wide_rescan(const PoaWide& S, const PoaBuffers& 
   for (int k = lane; k < W; k += 32)
     for (int j = 0; j < W; j++)
       if (all || S.dirty[j]) { S.wmin[j * W + k] = inf; S.wrow[j * W + k] = -1; }
-  for (int64_t r = 0; r < m; r++) {
-    const int j = b.asg[base + r];
-    if (j < 0 || !(all || S.dirty[j])) continue;
-    const double* cr = b.cost + (scratch_base + b.order[base + r]) * W;
-    const double cj = cr[j];
-    for (int k = lane; k < W; k += 32) {
-      const double v = __dsub_rn(cr[k], cj);
-      if (k != j && v < S.wmin[j * W + k]) { S.wmin[j * W + k] = v; S.wrow[j * W + k] = (int)r; }
+  // rows in order, 32 at a time: the lanes read 32 assignments at once and
+  // the rows at a rescanned worker are taken one by one (lowest row first, so
+  // ties keep the lowest row)
+  for (int64_t r0 = 0; r0 < m; r0 += 32) {
+    const int64_t rl = r0 + lane;
+    int jl = -1;
+    if (rl < m) jl = b.asg[base + rl];
+    unsigned hit = __ballot_sync(FULL_MASK, jl >= 0 && (all || S.dirty[jl]));
+    while (hit) {
+      const int src = __ffs(hit) - 1;
+      hit &= hit - 1;
+      const int j = __shfl_sync(FULL_MASK, jl, src);
+      const int r = (int)(r0 + src);
+      const double* cr = b.cost + (base + r) * W;
+      const double cj = cr[j];
+      for (int k = lane; k < W; k += 32) {
+        const double v = __dsub_rn(cr[k], cj);
+        if (k != j && v < S.wmin[j * W + k]) { S.wmin[j * W + k] = v; S.wrow[j * W + k] = r; }
+      }
     }
   }
 }
@@ -448,7 +497,7 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
     double num = 0.0, nst = 0.0;
     for (int64_t r = lane; r < m; r += 32) {
       const int q = b.order[base + r];
-      const double* cr = b.cost + (pr.scratch_base + q) * W;
+      const double* cr = b.cost + (base + r) * W;
       nst += cr[b.rec.worker[pr.rec_base + q]];
       int best = 0;
       double bc = cr[0];
@@ -482,7 +531,7 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
       __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
-        const double* c0 = b.cost + (pr.scratch_base + b.order[base + r0]) * W;
+        const double* c0 = b.cost + (base + r0) * W;
         for (int k = lane; k < W; k += 32) { S.dist[k] = c0[k]; S.pred[k] = -1; }
         __syncwarp();
         // Jacobi rounds: every target reads the previous round's distances.
@@ -554,7 +603,7 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
         for (int t = 0; t < nmv; t++) {
           const int r = S.mv_row[t], to = S.mv_to[t];
           if (S.dirty[to]) continue;
-          const double* cr = b.cost + (pr.scratch_base + b.order[base + r]) * W;
+          const double* cr = b.cost + (base + r) * W;
           const double ct = cr[to];
           for (int k2 = lane; k2 < W; k2 += 32) {
             if (k2 == to) continue;
@@ -574,9 +623,8 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
     }
     double opt = 0.0;
     for (int64_t r = lane; r < m; r += 32) {
-      const int q = b.order[base + r];
       const int a = b.asg[base + r];
-      opt += a >= 0 ? b.cost[(pr.scratch_base + q) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
+      opt += a >= 0 ? b.cost[(base + r) * W + a] : __longlong_as_double(0x7FF8000000000000ll);
     }
     opt = warp_sum(opt);
     if (lane == 0) {
