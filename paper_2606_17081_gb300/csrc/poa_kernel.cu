@@ -171,48 +171,66 @@ struct PoaWarpShared {
   int err;
 };
 
+// Order-preserving map of a double onto uint64: x < y (IEEE, neither NaN,
+// not both zero) iff dorder(x) < dorder(y); comparisons on the serial paths
+// then run on the integer units instead of the FP64 pipe.
+__device__ __forceinline__ uint64_t dorder(double x) {
+  const uint64_t u = (uint64_t)__double_as_longlong(x);
+  return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
+}
+__device__ __forceinline__ double dunorder(uint64_t k) {
+  const uint64_t u = (k >> 63) ? (k & 0x7FFFFFFFFFFFFFFFull) : ~k;
+  return __longlong_as_double((long long)u);
+}
+constexpr uint64_t DKEY_NONE = ~0ull;   // above dorder of every double but NaN
+
 // Edge weights out of worker j: for every k, the cheapest move of a request now
 // at j to k, min over those requests of c_qk - c_qj (ties: lowest row).
 __device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffers& b,
-                                               int64_t scratch_base, int64_t base, int64_t m,
-                                               int W, int j, int lane) {
-  // per lane: the cheapest move to each k among its rows (registers: the
-  // loops run over the fixed POA_WMAX with k < W guards)
-  double lm[POA_WMAX];
+                                               int64_t base, int64_t m, int W, int j, int lane) {
+  // per lane: the cheapest move to each k among its rows, as order keys
+  // (registers: the loops run over the fixed POA_WMAX with k < W guards);
+  // four rows per lane in flight, each lane's rows in increasing order so
+  // that ties keep the lowest row
+  uint64_t lk[POA_WMAX];
   int lr[POA_WMAX];
 #pragma unroll
-  for (int k = 0; k < POA_WMAX; k++) { lm[k] = __longlong_as_double(0x7FF0000000000000ll); lr[k] = -1; }
-  for (int64_t r = lane; r < m; r += 32) {
-    if (b.asg[base + r] != j) continue;
-    const double* cr = b.cost + (base + r) * W;
-    const double cj = cr[j];
+  for (int k = 0; k < POA_WMAX; k++) { lk[k] = DKEY_NONE; lr[k] = -1; }
+  for (int64_t r0 = lane; r0 < m; r0 += 128) {
+    int at[4];
 #pragma unroll
-    for (int k = 0; k < POA_WMAX; k++) {
-      if (k < W) {
-        const double v = __dsub_rn(cr[k], cj);
-        if (k != j && v < lm[k]) { lm[k] = v; lr[k] = (int)r; }
+    for (int u = 0; u < 4; u++) at[u] = r0 + 32 * u < m ? b.asg[base + r0 + 32 * u] : -1;
+#pragma unroll
+    for (int u = 0; u < 4; u++) {
+      if (at[u] != j) continue;
+      const int64_t r = r0 + 32 * u;
+      const double* cr = b.cost + (base + r) * W;
+      const double cj = cr[j];
+#pragma unroll
+      for (int k = 0; k < POA_WMAX; k++) {
+        if (k < W && k != j) {
+          const uint64_t key = dorder(__dsub_rn(cr[k], cj));
+          if (key < lk[k]) { lk[k] = key; lr[k] = (int)r; }
+        }
       }
     }
   }
 #pragma unroll
   for (int k = 0; k < POA_WMAX; k++) {
     if (k < W) {
-      double v = lm[k];
+      uint64_t key = lk[k];
       int rr = lr[k];
       for (int o = 16; o > 0; o >>= 1) {
-        const double v2 = __shfl_xor_sync(FULL_MASK, v, o);
+        const uint64_t k2 = __shfl_xor_sync(FULL_MASK, key, o);
         const int r2 = __shfl_xor_sync(FULL_MASK, rr, o);
-        if (r2 >= 0 && (rr < 0 || v2 < v || (v2 == v && r2 < rr))) { v = v2; rr = r2; }
+        if (r2 >= 0 && (rr < 0 || k2 < key || (k2 == key && r2 < rr))) { key = k2; rr = r2; }
       }
-      if (lane == 0) { S.wmin[j][k] = v; S.wrow[j][k] = rr; }
+      if (lane == 0) {
+        S.wmin[j][k] = rr >= 0 ? dunorder(key) : __longlong_as_double(0x7FF0000000000000ll);
+        S.wrow[j][k] = rr;
+      }
     }
   }
-}
-
-// Order-preserving map of a finite double onto uint64 (for integer compares).
-__device__ __forceinline__ uint64_t dorder(double x) {
-  const uint64_t u = (uint64_t)__double_as_longlong(x);
-  return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
 }
 
 struct PoaSolveShared {
@@ -287,7 +305,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       }
       __syncwarp();
       const int64_t nrem = (int64_t)S.num;
-      for (int j = 0; j < W; j++) poa_edges_from(S, b, pr.scratch_base, base, m, W, j, lane);
+      for (int j = 0; j < W; j++) poa_edges_from(S, b, base, m, W, j, lane);
       __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
@@ -301,18 +319,23 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
         int pk = -1;
         if (lane < W) dk = c0[lane];
         for (int it = 0; it < W; it++) {
-          double nd = dk;
-          int np = pk, ch = 0;
+          // the best way into k this round (lowest j on ties), then one
+          // FP64 test against the gain threshold
+          uint64_t bk = DKEY_NONE;
+          int bj = -1;
 #pragma unroll
           for (int j = 0; j < POA_WMAX; j++) {
             const double dj = __shfl_sync(FULL_MASK, dk, j);
             if (j < W && lane < W && j != lane && S.wrow[j][lane] >= 0) {
-              const double v = __dadd_rn(dj, S.wmin[j][lane]);
-              if (v < nd - 1e-12) { nd = v; np = j; ch = 1; }
+              const uint64_t key = dorder(__dadd_rn(dj, S.wmin[j][lane]));
+              if (key < bk) { bk = key; bj = j; }
             }
           }
-          dk = nd;
-          pk = np;
+          int ch = 0;
+          if (bj >= 0) {
+            const double v = dunorder(bk);
+            if (v < dk - 1e-12) { dk = v; pk = bj; ch = 1; }
+          }
           if (!__any_sync(FULL_MASK, ch)) break;
         }
         // target: the nearest worker with room (ties: lowest index)
@@ -379,7 +402,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
         }
         __syncwarp();
         for (int j = 0; j < W; j++)
-          if (S.dirty[j]) poa_edges_from(S, b, pr.scratch_base, base, m, W, j, lane);
+          if (S.dirty[j]) poa_edges_from(S, b, base, m, W, j, lane);
         __syncwarp();
       }
     }
@@ -422,34 +445,66 @@ __host__ __device__ inline size_t poa_wide_smem(int W) {
 }
 
 // Recompute the weights out of every source j with dirty[j] (all of them when
-// all is set): min over the requests at j of c_qk - c_qj, ties to the lowest row.
-__device__ __forceinline__ void wide_rescan(const PoaWide& S, const PoaBuffers& b,
-                                            int64_t scratch_base, int64_t base, int64_t m,
-                                            int W, int lane, bool all) {
+// all is set): min over the requests at j of c_qk - c_qj, ties to the lowest
+// row.  Rows go 128 at a time: four assignment loads per lane, the rows at a
+// rescanned worker compacted in order into `sel`, then taken four at a time
+// with their cost slices loaded together (lane l keeps columns l, l + 32).
+__device__ __forceinline__ void wide_rescan(const PoaWide& S, const PoaBuffers& b, int64_t base,
+                                            int64_t m, int W, int lane, bool all, int* sel) {
   const double inf = __longlong_as_double(0x7FF0000000000000ll);
   for (int k = lane; k < W; k += 32)
     for (int j = 0; j < W; j++)
       if (all || S.dirty[j]) { S.wmin[j * W + k] = inf; S.wrow[j * W + k] = -1; }
-  // rows in order, 32 at a time: the lanes read 32 assignments at once and
-  // the rows at a rescanned worker are taken one by one (lowest row first, so
-  // ties keep the lowest row)
-  for (int64_t r0 = 0; r0 < m; r0 += 32) {
-    const int64_t rl = r0 + lane;
-    int jl = -1;
-    if (rl < m) jl = b.asg[base + rl];
-    unsigned hit = __ballot_sync(FULL_MASK, jl >= 0 && (all || S.dirty[jl]));
-    while (hit) {
-      const int src = __ffs(hit) - 1;
-      hit &= hit - 1;
-      const int j = __shfl_sync(FULL_MASK, jl, src);
-      const int r = (int)(r0 + src);
-      const double* cr = b.cost + (base + r) * W;
-      const double cj = cr[j];
-      for (int k = lane; k < W; k += 32) {
-        const double v = __dsub_rn(cr[k], cj);
-        if (k != j && v < S.wmin[j * W + k]) { S.wmin[j * W + k] = v; S.wrow[j * W + k] = r; }
+  for (int64_t r0 = 0; r0 < m; r0 += 128) {
+    int at[4];
+#pragma unroll
+    for (int u = 0; u < 4; u++) {
+      const int64_t r = r0 + 32 * u + lane;
+      at[u] = r < m ? b.asg[base + r] : -1;
+    }
+    int ns = 0;
+#pragma unroll
+    for (int u = 0; u < 4; u++) {
+      const bool hit = at[u] >= 0 && (all || S.dirty[at[u]]);
+      const unsigned msk = __ballot_sync(FULL_MASK, hit);
+      if (hit) sel[ns + __popc(msk & ((1u << lane) - 1u))] = (int)(32 * u + lane);
+      ns += __popc(msk);
+    }
+    __syncwarp();
+    for (int t0 = 0; t0 < ns; t0 += 4) {
+      double c0[4], c1[4], cj[4];
+      int rr[4], jj[4];
+#pragma unroll
+      for (int u = 0; u < 4; u++) {
+        rr[u] = -1;
+        if (t0 + u < ns) {
+          const int64_t r = r0 + sel[t0 + u];
+          rr[u] = (int)r;
+          jj[u] = b.asg[base + r];
+          const double* cr = b.cost + (base + r) * W;
+          c0[u] = lane < W ? cr[lane] : 0.0;
+          c1[u] = lane + 32 < W ? cr[lane + 32] : 0.0;
+          cj[u] = cr[jj[u]];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; u++) {
+        if (rr[u] < 0) continue;
+        const int j = jj[u];
+        if (lane < W && lane != j) {
+          const double v = __dsub_rn(c0[u], cj[u]);
+          if (v < S.wmin[j * W + lane]) { S.wmin[j * W + lane] = v; S.wrow[j * W + lane] = rr[u]; }
+        }
+        if (lane + 32 < W && lane + 32 != j) {
+          const double v = __dsub_rn(c1[u], cj[u]);
+          if (v < S.wmin[j * W + lane + 32]) {
+            S.wmin[j * W + lane + 32] = v;
+            S.wrow[j * W + lane + 32] = rr[u];
+          }
+        }
       }
     }
+    __syncwarp();
   }
 }
 
@@ -471,6 +526,8 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
   }
   __shared__ int s_err, s_nmv;
   __shared__ long long s_nrem;
+  __shared__ int s_sel[128];          // rows of a rescan chunk
+  __shared__ int s_pj[POA_WMAX_WIDE + 1], s_pr[POA_WMAX_WIDE + 1];   // the last path's edges
   const PoaProblem pr = probs[blockIdx.x];
   const int64_t nw = b.nwin[blockIdx.x];
   if (nw < 0) return;
@@ -527,46 +584,76 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
       }
       __syncwarp();
       const int64_t nrem = s_nrem;
-      wide_rescan(S, b, pr.scratch_base, base, m, W, lane, true);
+      wide_rescan(S, b, base, m, W, lane, true, s_sel);
       __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
         const double* c0 = b.cost + (base + r0) * W;
         for (int k = lane; k < W; k += 32) { S.dist[k] = c0[k]; S.pred[k] = -1; }
         __syncwarp();
-        // Jacobi rounds: every target reads the previous round's distances.
-        // Only gains above 1e-12 count (exact cycles are >= 0; rounding-level
-        // negative ones must not loop the predecessors).
-        for (int it = 0; it < W; it++) {
-          double nd0 = 0.0, nd1 = 0.0;
-          int np0 = -1, np1 = -1, ch = 0;
-          const int k0 = lane, k1 = lane + 32;
-          if (k0 < W) { nd0 = S.dist[k0]; np0 = S.pred[k0]; }
-          if (k1 < W) { nd1 = S.dist[k1]; np1 = S.pred[k1]; }
-          for (int j = 0; j < W; j++) {
-            const double dj = S.dist[j];
-            if (k0 < W && j != k0 && S.wrow[j * W + k0] >= 0) {
-              const double v = __dadd_rn(dj, S.wmin[j * W + k0]);
-              if (v < nd0 - 1e-12) { nd0 = v; np0 = j; ch = 1; }
+        // Jacobi rounds: every target reads the previous round's distances;
+        // the best way into a target (lowest j on ties) is found on order
+        // keys, then tested once against the gain threshold.  Only gains
+        // above 1e-12 count (exact cycles are >= 0; rounding-level negative
+        // ones must not loop the predecessors).  A round relaxes only the
+        // edges out of sources whose distance changed in the round before:
+        // an edge out of an unchanged source was tested against a distance
+        // that has only fallen since, so it cannot pass now.
+        uint64_t act = W >= 64 ? ~0ull : ((1ull << W) - 1ull);
+        for (int it = 0; it < W && act; it++) {
+          int ch[2] = {0, 0};
+          double nd[2];
+          int np[2];
+#pragma unroll
+          for (int h = 0; h < 2; h++) {
+            const int k = lane + 32 * h;
+            nd[h] = 0.0;
+            np[h] = -1;
+            if (k >= W) continue;
+            nd[h] = S.dist[k];
+            np[h] = S.pred[k];
+            uint64_t bk = DKEY_NONE;
+            int bj = -1;
+            for (uint64_t a = act; a; a &= a - 1) {
+              const int j = __ffsll((long long)a) - 1;
+              if (j == k || S.wrow[j * W + k] < 0) continue;
+              const uint64_t key = dorder(__dadd_rn(S.dist[j], S.wmin[j * W + k]));
+              if (key < bk || (key == bk && j < bj)) { bk = key; bj = j; }
             }
-            if (k1 < W && j != k1 && S.wrow[j * W + k1] >= 0) {
-              const double v = __dadd_rn(dj, S.wmin[j * W + k1]);
-              if (v < nd1 - 1e-12) { nd1 = v; np1 = j; ch = 1; }
+            if (bj >= 0) {
+              const double v = dunorder(bk);
+              if (v < nd[h] - 1e-12) { nd[h] = v; np[h] = bj; ch[h] = 1; }
             }
           }
           __syncwarp();
-          if (k0 < W) { S.dist[k0] = nd0; S.pred[k0] = np0; }
-          if (k1 < W) { S.dist[k1] = nd1; S.pred[k1] = np1; }
-          ch = __any_sync(FULL_MASK, ch);
+#pragma unroll
+          for (int h = 0; h < 2; h++) {
+            const int k = lane + 32 * h;
+            if (k < W) { S.dist[k] = nd[h]; S.pred[k] = np[h]; }
+          }
+          act = (uint64_t)__ballot_sync(FULL_MASK, ch[0]) |
+                ((uint64_t)__ballot_sync(FULL_MASK, ch[1]) << 32);
           __syncwarp();
-          if (!ch) break;
+        }
+        // target: the nearest worker with room (ties: lowest index)
+        uint64_t tkey = DKEY_NONE;
+        int tl = -1;
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+          const int k = lane + 32 * h;
+          if (k < W && S.counts[k] < capw) {
+            const uint64_t key = dorder(S.dist[k]);
+            if (tl < 0 || key < tkey) { tkey = key; tl = k; }
+          }
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+          const uint64_t k2 = __shfl_xor_sync(FULL_MASK, tkey, o);
+          const int t2 = __shfl_xor_sync(FULL_MASK, tl, o);
+          if (t2 >= 0 && (tl < 0 || k2 < tkey || (k2 == tkey && t2 < tl))) { tkey = k2; tl = t2; }
         }
         if (lane == 0) {
-          int tgt = -1;
-          for (int k = 0; k < W; k++)
-            if (S.counts[k] < capw && (tgt < 0 || S.dist[k] < S.dist[tgt])) tgt = k;
+          const int tgt = tl;
           int nmv = 0;
-          for (int j = 0; j < W; j++) S.dirty[j] = 0;
           if (tgt < 0) {
             s_err = 1;
           } else {
@@ -576,9 +663,10 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
             while (S.pred[k] >= 0 && steps <= W) {
               const int j = S.pred[k];
               const int r = S.wrow[j * W + k];
+              s_pj[nmv] = j;
+              s_pr[nmv] = r;
               S.mv_row[nmv] = r;
               S.mv_to[nmv++] = k;
-              for (int k2 = 0; k2 < W; k2++) S.dirty[j] |= S.wrow[j * W + k2] == r;
               k = j;
               steps++;
             }
@@ -595,6 +683,21 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
           }
           s_nmv = nmv;
         }
+        __syncwarp();
+        // a source that lost its request needs a rescan where that request
+        // was the minimum of one of its weights
+        for (int j = lane; j < W; j += 32) S.dirty[j] = 0;
+        __syncwarp();
+        if (!s_err) {
+          const int npath = s_nmv - 1;
+          for (int t = 0; t < npath; t++) {
+            const int j = s_pj[t], r = s_pr[t];
+            bool hit = false;
+            for (int k2 = lane; k2 < W; k2 += 32) hit |= S.wrow[j * W + k2] == r;
+            if (__any_sync(FULL_MASK, hit) && lane == 0) S.dirty[j] = 1;
+          }
+        }
+        __syncwarp();
         __syncwarp();
         if (s_err) break;
         // requests that moved in lower their new worker's weights; a dirty
@@ -617,7 +720,7 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
         }
         int anyd = 0;
         for (int j = lane; j < W; j += 32) anyd |= S.dirty[j];
-        if (__any_sync(FULL_MASK, anyd)) wide_rescan(S, b, pr.scratch_base, base, m, W, lane, false);
+        if (__any_sync(FULL_MASK, anyd)) wide_rescan(S, b, base, m, W, lane, false, s_sel);
         __syncwarp();
       }
     }
