@@ -190,6 +190,47 @@ __device__ __forceinline__ int select_worker(const float* c, int W, float tau, u
   return pick >= 0 ? pick : last;
 }
 
+// select_worker computed by a whole warp (W <= 64; every lane returns the
+// same worker): lane l computes the weights of workers l and l + 32, each
+// once, and every lane then accumulates them in worker order from shuffles,
+// so the sums, the draw and the statistics are those of select_worker bit
+// for bit.  b: the lowest-index argmin of c.  ds (nullable) is written by
+// lane 0.
+__device__ __forceinline__ int select_worker_warp(const float* c, int W, float tau, uint32_t u24,
+                                                  int b, float* ds, int lane) {
+  if (tau == 0.0f) return b;
+  const float cmin = c[b];
+  float e[2];
+#pragma unroll
+  for (int h = 0; h < 2; h++) {
+    const int j = lane + 32 * h;
+    e[h] = j < W ? exp_sm(-__fdiv_rn(__fsub_rn(c[j], cmin), tau)) : 0.0f;
+  }
+  float S = 0.0f;
+  for (int j = 0; j < W; j++) S = __fadd_rn(S, __shfl_sync(FULL_MASK, e[j >> 5], j & 31));
+  const float target = __fmul_rn(__fmul_rn((float)u24, 0x1p-24f), S);
+  const float qnan = __int_as_float(0x7FC00000);
+  float cum = 0.0f, lo = qnan, hi = qnan;
+  int pick = -1, last = b;
+  for (int j = 0; j < W; j++) {
+    const float ej = __shfl_sync(FULL_MASK, e[j >> 5], j & 31);
+    cum = __fadd_rn(cum, ej);
+    if (ej > 0.0f) last = j;
+    if (pick < 0 && target < cum) {
+      pick = j;
+      hi = cum;
+    }
+    if (!(target < cum)) lo = cum;
+  }
+  if (ds && lane == 0) {
+    ds[0] = target;
+    ds[1] = S;
+    ds[2] = lo;
+    ds[3] = hi;
+  }
+  return pick >= 0 ? pick : last;
+}
+
 // ---------------------------------------------------------------- CTA helpers
 
 // Barrier of a thread group made of the CTA's first NT threads: the whole

@@ -1185,17 +1185,19 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     }
     argmin_warp(bc, bj);   // the lowest-index argmin (the choice at tau = 0)
     int js = bj;
-    if (!eq2 || tau > 0.0f) {
+    if (!eq2) {
       __syncwarp();
       int x = 0;
-      if (lane == 0) {
-        const uint32_t u24 = eq2 ? draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM) : 0u;
-        // (the control warp also records where the draw fell)
-        x = !eq2 ? static_policy_worker(d.policy, wc, W, d.seed, (uint64_t)i, 0u, TAG_SIM)
-                 : select_worker(wc, W, tau, u24,
-                                 warp == NT_SIM / 32 - 1 ? b.dstat + row * 6 + 2 : nullptr);
-      }
+      if (lane == 0) x = static_policy_worker(d.policy, wc, W, d.seed, (uint64_t)i, 0u, TAG_SIM);
       js = __shfl_sync(FULL_MASK, x, 0);
+    } else if (tau > 0.0f) {
+      __syncwarp();
+      uint32_t u24 = 0;
+      if (lane == 0) u24 = draw_u24(d.seed, (uint64_t)i, 0u, TAG_SIM);
+      u24 = __shfl_sync(FULL_MASK, u24, 0);
+      // (the control warp also records where the draw fell)
+      js = select_worker_warp(wc, W, tau, u24, bj,
+                              warp == NT_SIM / 32 - 1 ? b.dstat + row * 6 + 2 : nullptr, lane);
     }
     if (warp < NT_SIM / 32 - 1) {
       // ---- the chosen worker's LRU cache (warps 0-6).  Its inputs are read
@@ -1277,10 +1279,13 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       }
       cp_async_wait_all();
       __syncwarp();   // every lane's copies of request i+1's hashes have landed
-      if (more && nq.full && nq.nb <= (int)L.g.K) {
+      if (MINB == 1 && more && nq.full && nq.nb <= (int)L.g.K) {
         // request i+1's home buckets on every worker, brought into L2 ahead
         // of its probe (the update running beside may still change the
-        // chosen worker's; L2 holds the current data either way)
+        // chosen worker's; L2 holds the current data either way).  Only
+        // with one replica per SM: with two, the other replica's warps fill
+        // the probe's waits, and the prefetch instructions cost more than
+        // they save (11% on the parameter grid)
         const uint64_t* hn = c.hbuf(p ^ 1);
         const int nbn = nq.nb;
         for (int e = lane; e < W * nbn; e += 32) {
