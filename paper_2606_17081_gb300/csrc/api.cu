@@ -44,7 +44,7 @@ struct rs_ctx {
   DevBuf rec_worker, rec_arrival, rec_start, rec_first, rec_completion, rec_ttft, rec_nbt, rec_nfz,
       rec_prefix;
   DevBuf p_cost, p_order, p_asg, p_wkey, p_wstart, p_wfill, p_wnum, p_wopt, p_wcnt, p_total,
-      p_nwin, p_prob, p_wstat, p_tstat;
+      p_nwin, p_prob, p_wstat, p_tstat, p_wprob, p_wnext;
   DevBuf k_rows, k_load, k_sweep, k_stat, k_d1, k_d2, k_kload, k_kidx;
   DevBuf h_tokens, h_offsets, h_release, h_outlen;
   int64_t* pinned = nullptr;   // small host staging for device -> host reads
@@ -307,7 +307,8 @@ void route_destroy(rs_ctx* ctx) {
                    &ctx->rec_ttft, &ctx->rec_nbt, &ctx->rec_nfz, &ctx->rec_prefix, &ctx->p_cost,
                    &ctx->p_order, &ctx->p_asg, &ctx->p_wkey, &ctx->p_wstart, &ctx->p_wfill,
                    &ctx->p_wnum, &ctx->p_wopt, &ctx->p_wcnt, &ctx->p_total, &ctx->p_nwin,
-                   &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->h_tokens, &ctx->h_offsets,
+                   &ctx->p_prob, &ctx->p_wstat, &ctx->p_tstat, &ctx->p_wprob, &ctx->p_wnext,
+                   &ctx->h_tokens, &ctx->h_offsets,
                    &ctx->h_release, &ctx->h_outlen, &ctx->k_rows, &ctx->k_load, &ctx->k_sweep,
                    &ctx->k_stat, &ctx->k_d1, &ctx->k_d2, &ctx->k_kload, &ctx->k_kidx,
                    &ctx->fexp, &ctx->tmpe, &ctx->djobs, &ctx->h_hashes};
@@ -601,7 +602,9 @@ static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, std::vector<PoaProb
       (r = ensure(ctx, ctx->p_wnum, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wopt, (size_t)win_slots * 8, "poa windows")) ||
       (r = ensure(ctx, ctx->p_wstat, (size_t)win_slots * 8, "poa windows")) ||
-      (r = ensure(ctx, ctx->p_wcnt, (size_t)win_slots * 8, "poa windows")))
+      (r = ensure(ctx, ctx->p_wcnt, (size_t)win_slots * 8, "poa windows")) ||
+      (r = ensure(ctx, ctx->p_wprob, (size_t)win_slots * 4, "poa windows")) ||
+      (r = ensure(ctx, ctx->p_wnext, 8, "poa work counter")))
     return r;
   CK(cudaMemcpyAsync(ctx->p_prob.p, probs.data(), np * sizeof(PoaProblem), cudaMemcpyHostToDevice,
                      ctx->st),
@@ -622,6 +625,9 @@ static rs_status run_poa(rs_ctx* ctx, const rs_records& rec, std::vector<PoaProb
   b.total_static = P<double>(ctx->p_tstat);
   b.nwin = P<int64_t>(ctx->p_nwin);
   b.res = res_dev;
+  b.wprob = P<int32_t>(ctx->p_wprob);
+  b.wnext = P<unsigned long long>(ctx->p_wnext);
+  b.nslots = win_slots;
   CK(launch_poa(P<PoaProblem>(ctx->p_prob), np, b, ctx->mc, ctx->st), "poa launch");
   return RS_OK;
 }

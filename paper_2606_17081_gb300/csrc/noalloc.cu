@@ -160,6 +160,9 @@ extern "C" rs_status poa_estimate_noalloc(const rs_config* cfg, const rs_records
   b.total = reinterpret_cast<double*>(s + L.total);
   b.nwin = reinterpret_cast<int64_t*>(s + L.nwin);
   b.res = nullptr;
+  b.wprob = nullptr;   // one problem: its windows stay on its own CTAs
+  b.wnext = nullptr;
+  b.nslots = 0;
   if (launch_poa(dprob, 1, b, mc, st) != cudaSuccess) return RS_ERR_CUDA;
   k_noalloc_out<<<64, 256, 0, st>>>(b.wnum, b.wopt, b.wcnt, b.total, b.nwin, max_windows,
                                     numer_dev, opt_dev, count_dev, poa_total_dev, n_windows_dev);

@@ -50,6 +50,8 @@ __global__ void __launch_bounds__(NT_POA) k_poa_prep(const PoaProblem* __restric
   const PoaProblem pr = probs[blockIdx.x];
   const int W = mc.W;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (b.wprob)   // the owner of every window slot of this problem
+    for (int64_t w = threadIdx.x; w < pr.win_cap; w += NT_POA) b.wprob[pr.win_base + w] = blockIdx.x;
   if (threadIdx.x == 0) {
     P.maxw = -1;
     P.overflow = W > POA_WMAX_WIDE;
@@ -242,18 +244,52 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
+// The next window a solver warp takes: with b.wnext the warps of the whole
+// grid take window slots from the counter in order (a replica's windows
+// spread over the GPU, so a few heavy replicas do not hold the end of the
+// launch); without it the warps of problem blockIdx.x's CTAs stride over its
+// windows (next, stride).  Returns false when no window is left.
+__device__ __forceinline__ bool poa_next(const PoaProblem* __restrict__ probs, const PoaBuffers& b,
+                                         int lane, int64_t& next, int64_t stride, int* pi,
+                                         int64_t* w) {
+  for (;;) {
+    if (b.wnext) {
+      unsigned long long item = 0;
+      if (lane == 0) item = atomicAdd(b.wnext, 1ull);
+      item = __shfl_sync(FULL_MASK, item, 0);
+      if ((int64_t)item >= b.nslots) return false;
+      const int p = b.wprob[item];
+      const int64_t ww = (int64_t)item - probs[p].win_base;
+      const int64_t nw = b.nwin[p];
+      if (nw < 0 || ww >= nw) continue;   // a spare slot, or a problem that overflowed
+      *pi = p;
+      *w = ww;
+      return true;
+    }
+    const int64_t nw = b.nwin[blockIdx.x];
+    const int64_t ww = next;
+    next += stride;
+    if (nw < 0 || ww >= nw) return false;
+    *pi = (int)blockIdx.x;
+    *w = ww;
+    return true;
+  }
+}
+
 __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restrict__ probs,
                                                       PoaBuffers b, ModelConsts mc) {
   __shared__ PoaSolveShared P;
-  const PoaProblem pr = probs[blockIdx.x];
-  const int64_t nw = b.nwin[blockIdx.x];
-  if (nw < 0) return;   // k_poa_total reports it
   const int W = mc.W;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   PoaWarpShared& S = P.w[warp];
-  const int64_t* wst = b.wstart + pr.win_base + blockIdx.x;
-  const int64_t nwarps = (int64_t)gridDim.y * (NT_POA / 32);
-  for (int64_t w = (int64_t)blockIdx.y * (NT_POA / 32) + warp; w < nw; w += nwarps) {
+  int64_t next = (int64_t)blockIdx.y * (NT_POA / 32) + warp;
+  const int64_t stride = (int64_t)gridDim.y * (NT_POA / 32);
+  int pi;
+  int64_t w;
+  // (a problem whose windows overflowed: k_poa_total reports it)
+  while (poa_next(probs, b, lane, next, stride, &pi, &w)) {
+    const PoaProblem pr = probs[pi];
+    const int64_t* wst = b.wstart + pr.win_base + pi;
     const int64_t s0 = wst[w];
     const int64_t m = wst[w + 1] - s0;
     const int64_t base = pr.scratch_base + s0;   // window rows in order[], asg[]
@@ -528,12 +564,14 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
   __shared__ long long s_nrem;
   __shared__ int s_sel[128];          // rows of a rescan chunk
   __shared__ int s_pj[POA_WMAX_WIDE + 1], s_pr[POA_WMAX_WIDE + 1];   // the last path's edges
-  const PoaProblem pr = probs[blockIdx.x];
-  const int64_t nw = b.nwin[blockIdx.x];
-  if (nw < 0) return;
   const int lane = threadIdx.x;
-  const int64_t* wst = b.wstart + pr.win_base + blockIdx.x;
-  for (int64_t w = blockIdx.y; w < nw; w += gridDim.y) {
+  int64_t next = blockIdx.y;
+  const int64_t stride = gridDim.y;
+  int pi;
+  int64_t w;
+  while (poa_next(probs, b, lane, next, stride, &pi, &w)) {
+    const PoaProblem pr = probs[pi];
+    const int64_t* wst = b.wstart + pr.win_base + pi;
     const int64_t s0 = wst[w];
     const int64_t m = wst[w + 1] - s0;
     const int64_t base = pr.scratch_base + s0;
@@ -821,16 +859,38 @@ cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int split = (4 * sms + nprob - 1) / nprob;
   split = split < 1 ? 1 : (split > 16 ? 16 : split);
-  if (mc.W <= POA_WMAX) {
+  const size_t wsmem = poa_wide_smem(mc.W);
+  if (mc.W > POA_WMAX &&
+      (e = cudaFuncSetAttribute(k_poa_solve_wide, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)wsmem)) != cudaSuccess)
+    return e;
+  if (b.wnext) {
+    // one wave of CTAs whose warps take the windows from the counter
+    if ((e = cudaMemsetAsync(b.wnext, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+    int per_sm = 0;
+    if (mc.W <= POA_WMAX) {
+      if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_poa_solve, NT_POA, 0)) !=
+          cudaSuccess)
+        return e;
+      int64_t g = (b.nslots + NT_POA / 32 - 1) / (NT_POA / 32);
+      const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+      g = g < cap ? g : cap;
+      k_poa_solve<<<(unsigned)(g > 0 ? g : 1), NT_POA, 0, st>>>(d_prob, b, mc);
+    } else {
+      if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_poa_solve_wide, 32,
+                                                             wsmem)) != cudaSuccess)
+        return e;
+      int64_t g = b.nslots;
+      const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+      g = g < cap ? g : cap;
+      k_poa_solve_wide<<<(unsigned)(g > 0 ? g : 1), 32, wsmem, st>>>(d_prob, b, mc);
+    }
+  } else if (mc.W <= POA_WMAX) {
     k_poa_solve<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
   } else {
     // one warp per CTA: 8x the CTAs for the same windows in flight
-    const size_t smem = poa_wide_smem(mc.W);
-    if ((e = cudaFuncSetAttribute(k_poa_solve_wide, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)smem)) != cudaSuccess)
-      return e;
     const int wsplit = split * (NT_POA / 32) > 128 ? 128 : split * (NT_POA / 32);
-    k_poa_solve_wide<<<dim3(nprob, wsplit), 32, smem, st>>>(d_prob, b, mc);
+    k_poa_solve_wide<<<dim3(nprob, wsplit), 32, wsmem, st>>>(d_prob, b, mc);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   k_poa_total<<<(nprob + NT_POA / 32 - 1) / (NT_POA / 32), NT_POA, 0, st>>>(nprob, b, d_prob);

@@ -173,6 +173,13 @@ struct PoaBuffers {
   double* total_static;     // [problems]: realized assignment's frozen cost / OPT
   int64_t* nwin;            // [problems]: windows spanned (or -1 on overflow)
   rs_replica_result* res;   // optional [problems] (poa_total, n_windows filled)
+  // optional: the window slots (nslots of them) go to the solver warps of the
+  // whole grid through the counter wnext, zeroed by launch_poa; wprob[slot]
+  // = the problem owning the slot.  NULL: each problem's windows stay on its
+  // own CTAs.
+  int32_t* wprob;
+  unsigned long long* wnext;
+  int64_t nslots;
 };
 
 // Saturation knee of load sweeps: per-replica percentile, divided differences, knee.
