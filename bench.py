@@ -85,11 +85,30 @@ def rank_range(n: int, ws: int, rank: int):
     return n * rank // ws, n * (rank + 1) // ws
 
 
-def _plan(name: str, rank: int = 0, ws: int = 1, n_req=None):
+def _subset(full, spec):
+    """Replica indices of a profiling subset: "N" = the plan's first N
+    replicas, "per-trace" = the first replica of every trace."""
+    if spec == "per-trace":
+        seen, idx = set(), []
+        for k, r in enumerate(full.replicas):
+            if r.trace not in seen:
+                seen.add(r.trace)
+                idx.append(k)
+        return idx
+    return list(range(min(int(spec), len(full.replicas))))
+
+
+def _plan(name: str, rank: int = 0, ws: int = 1, n_req=None, subset=None):
     """The workload's replicas that rank `rank` of ws runs (its contiguous
-    range of the one plan, traces remapped to the ones it uses)."""
+    range of the one plan, traces remapped to the ones it uses); `subset`
+    (a profiling option) first narrows the plan to those replicas."""
     from paper_2606_17081_gb300 import workloads as wk
     full = wk.plan(name, n_req=n_req)
+    if subset is not None:
+        full = wk.plan(name, n_req=n_req, replicas=_subset(full, subset))
+        if ws > 1:
+            raise ValueError("--replicas is a single-GPU profiling option")
+        return full, 0, len(full.replicas)
     lo, hi = rank_range(len(full.replicas), ws, rank)
     if (lo, hi) == (0, len(full.replicas)):
         return full, lo, hi
@@ -168,10 +187,16 @@ def _table_bytes(K: int) -> int:
 
 
 # DRAM bytes (read + write) of one full-size k_sim launch of the headline
-# workload, from a one-pass ncu capture (dram__bytes_read.sum +
-# dram__bytes_write.sum), with the SHA-256 of the simulation kernel's sources
-# it was taken with; None until such a capture exists for these sources.
-SIM_TRAFFIC = {"bytes": None, "sources_sha256": None, "summary": "profiles/k_sim_grid.md"}
+# workload (dram__bytes_read.sum + dram__bytes_write.sum), with the SHA-256 of
+# the simulation kernel's sources it was taken with; None until such a
+# capture exists for these sources.  The full grid holds about 103 GB of
+# cache tables, so the capture ran on 304 of its 8192 simulations (one
+# resident wave, two per SM, 10 000 requests each: 238.10 GB) and is scaled by
+# 8192 / 304; every simulation's tables and requests are of the same kind.
+SIM_TRAFFIC = {"bytes": 238101519872 * 8192 / 304,
+               "sources_sha256": "df83565d6780133147266487b3928c6001b83d1a99934e09215ac275302f8ea6",
+               "summary": "profiles/k_sim_grid.md",
+               "scaled_from": "304 simulations x 10 000 requests, times 8192 / 304"}
 
 
 def _sim_traffic(full_size: bool):
@@ -371,7 +396,8 @@ def _aux_variants(rs, reps: int = 2) -> dict:
     return out
 
 
-def _aux_probe(rs, n_route: int = 4096, n_probe: int = 60000, reps: int = 5) -> dict:
+def _aux_probe(rs, n_route: int = 4096, n_probe: int = 60000, reps: int = 5,
+               cache_blocks=None) -> dict:
     """Outside the timed steps: the batch probe (route_probe: S2's cached
     prefix for many requests against one cache snapshot) where its tables do
     not fit in L2: a router instance of 64 workers with 2^20-block caches (the
@@ -386,7 +412,7 @@ def _aux_probe(rs, n_route: int = 4096, n_probe: int = 60000, reps: int = 5) -> 
     from paper_2606_17081_gb300 import workloads as wk
     p = wk.plan("large", n_req=n_route + n_probe)
     tr = p.traces()[0]
-    W, K = p.W, p.K
+    W, K = p.W, (cache_blocks or p.K)
     ctx = rs.Context(W=W, K=K, n_instances=1)
     d = rs.device_trace(tr)
     wo = torch.zeros(n_route, dtype=torch.int32, device="cuda")
@@ -432,8 +458,12 @@ def run_gpu(args):
     if ws > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     name = args.workload
-    p, lo, hi = _plan(name, rank, ws, args.n_req)
-    full = args.n_req is None
+    if args.probe_only:
+        if rank == 0:
+            print(json.dumps({"probe_batch_hbm": _aux_probe(rs, cache_blocks=args.probe_cache_blocks)}))
+        return
+    p, lo, hi = _plan(name, rank, ws, args.n_req, args.replicas)
+    full = args.n_req is None and args.replicas is None
     traces = p.traces()
     ctx = rs.Context(W=p.W, K=p.K, theta1=p.theta1, theta2=p.theta2)
     dev = [rs.device_trace(t) for t in traces]
@@ -513,6 +543,7 @@ def run_gpu(args):
     roof = _roofline(res, p.W, sim_avg, peak, peak_kind)
     roof["traffic"] = _sim_traffic(full and ws == 1)
     roof["traffic_source"] = SIM_TRAFFIC["summary"]
+    roof["traffic_scaled_from"] = SIM_TRAFFIC["scaled_from"]
     roof["note"] = (f"latency-bound event loop: {len(params)} simulations, "
                     f"{'two' if len(params) > 152 else 'one'} resident per SM")
     hash_avg = statistics.mean(hash_ms)
@@ -711,6 +742,14 @@ def main():
                          "batch probe)")
     ap.add_argument("--n-req", type=int, default=None,
                     help="truncate every replica's trace (profiling of a small case)")
+    ap.add_argument("--replicas", default=None,
+                    help="profiling of a small case: the plan's first N replicas, or "
+                         "'per-trace' (the first replica of every trace)")
+    ap.add_argument("--probe-only", action="store_true",
+                    help="run only the batch-probe measurement (aux.probe_batch_hbm)")
+    ap.add_argument("--probe-cache-blocks", type=int, default=None,
+                    help="cache blocks per worker of the batch-probe instance "
+                         "(default: the W = 64 workload's 2^20)")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
