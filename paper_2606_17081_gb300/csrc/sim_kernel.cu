@@ -237,10 +237,16 @@ __device__ __forceinline__ bool ev_less(const SimCtx& c, uint64_t ka, int fa, ui
   return ka < kb || (ka == kb && c.f_req[fa] < c.f_req[fb]);
 }
 
+// The completions heap: 4-ary (children of i at 4i+1 .. 4i+4), half the
+// levels of a binary heap on the control thread's dependent chain; ev_less is
+// a strict total order (time, then request), so the pops are the same events
+// in the same order whatever the heap's shape.
+constexpr int HEAP_D = 4;
+
 __device__ __forceinline__ void heap_push(SimCtx& c, uint64_t k, int f) {
   int i = c.S->nheap++;
   while (i > 0) {
-    const int p = (i - 1) >> 1;
+    const int p = (i - 1) / HEAP_D;
     if (!ev_less(c, k, f, c.h_k[p], c.h_f[p])) break;
     c.h_k[i] = c.h_k[p];
     c.h_f[i] = c.h_f[p];
@@ -258,13 +264,29 @@ __device__ __forceinline__ void heap_pop(SimCtx& c, uint64_t* k, int* f) {
   const int lf = c.h_f[n];
   int i = 0;
   for (;;) {
-    const int l = 2 * i + 1, r = l + 1;
-    if (l >= n) break;
-    int s = l;
-    if (r < n && ev_less(c, c.h_k[r], c.h_f[r], c.h_k[l], c.h_f[l])) s = r;
-    if (!ev_less(c, c.h_k[s], c.h_f[s], lk, lf)) break;
-    c.h_k[i] = c.h_k[s];
-    c.h_f[i] = c.h_f[s];
+    const int c0 = HEAP_D * i + 1;
+    if (c0 >= n) break;
+    const int c1 = min(c0 + HEAP_D, n);
+    // the children's keys first (independent loads), then their minimum
+    uint64_t kk[HEAP_D];
+#pragma unroll
+    for (int q = 0; q < HEAP_D; q++) kk[q] = c0 + q < c1 ? c.h_k[c0 + q] : KEY_INF;
+    int s = c0;
+    uint64_t ks = kk[0];
+    int fs = c.h_f[c0];
+#pragma unroll
+    for (int q = 1; q < HEAP_D; q++) {
+      if (c0 + q >= c1) break;
+      const int fq = c.h_f[c0 + q];
+      if (ev_less(c, kk[q], fq, ks, fs)) {
+        s = c0 + q;
+        ks = kk[q];
+        fs = fq;
+      }
+    }
+    if (!ev_less(c, ks, fs, lk, lf)) break;
+    c.h_k[i] = ks;
+    c.h_f[i] = fs;
     i = s;
   }
   c.h_k[i] = lk;
@@ -531,45 +553,104 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
 // ------------------------------------------------------------ routing step
 
 // m_j: leading blocks of the prompt found in worker j's cache, for every j
-// (all threads).  Rounds of CH blocks per still-undecided worker; a worker is
-// decided once a miss is found below the round's end.
-template <int NT>
+// (threads of the group), when W nb is too large to look every pair up at
+// once.  Rounds over the workers still undecided: a round looks up the next
+// `len` blocks of each open worker, with len = ILP NT / (open workers) so
+// that a round is ILP lookups per thread (4 with one replica per SM, 1 within
+// the two-per-SM register budget), all issued before any is resolved;
+// a worker is decided once a miss falls in its window.  Most workers miss at
+// their first block, so the few left open after the first round get long
+// windows.
+template <int NT, int ILP>
 __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
-  const int CH = max(32, ((4 * NT) / W) & ~31);
   int c0 = 0;
   int err = 0;
   unsigned cnt = 0;
   for (;;) {
     const int nopen = S.nopen;
-    const int len = min(CH, nb - c0);
+    int len = (ILP * NT) / nopen;
+    if (len < 1) len = 1;
+    if (len > nb - c0) len = nb - c0;
     const int total = len > 0 ? nopen * len : 0;
-    const int rounds = (total + NT - 1) / NT;
-    for (int q = 0; q < rounds; q++) {        // uniform trip count: warp reductions below
-      const int it = q * NT + threadIdx.x;
-      int jj = -1, miss = 0x7FFFFFFF;
-      if (it < total) {
-        jj = c.wopen[it / len];
-        const int k = c0 + it % len;
-        if (k < c.wm[jj]) {
-          cnt++;
-          if (table_find(c.table(jj), hbuf[k], &err) == SLOT_NONE) miss = k;
+    // open worker of lookup `it` = floor(it / len): (it + 0.5) / len lies at
+    // least 0.5 / len from an integer and it < ILP NT, so the float product
+    // truncates to it exactly
+    const float inv_len = len > 0 ? 1.0f / (float)len : 0.0f;
+    for (int base = 0; base < total; base += ILP * NT) {   // uniform
+      if constexpr (ILP == 1) {
+        // one lookup per thread, resolved where it is issued
+        const int it = base + threadIdx.x;
+        int jj = -1, miss = 0x7FFFFFFF;
+        if (it < total) {
+          const int o = (int)(((float)it + 0.5f) * inv_len);
+          const int j = c.wopen[o];
+          const int k = c0 + (it - o * len);
+          if (k < c.wm[j]) {   // (no miss known below k yet)
+            jj = j;
+            cnt++;
+            if (table_find(c.table(j), hbuf[k], &err) == SLOT_NONE) miss = k;
+          }
+        }
+        const unsigned grp = __match_any_sync(FULL_MASK, jj);
+        const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
+        if (jj >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
+          atomicMin(&c.wm[jj], m);
+        continue;
+      }
+      int jj[ILP], kk[ILP];
+      uint64_t v[ILP][BUCKET];
+      uint32_t bk[ILP];
+#pragma unroll
+      for (int r = 0; r < ILP; r++) {
+        const int it = base + r * NT + threadIdx.x;
+        jj[r] = -1;
+        if (it < total) {
+          const int o = (int)(((float)it + 0.5f) * inv_len);
+          const int j = c.wopen[o];
+          const int k = c0 + (it - o * len);
+          if (k < c.wm[j]) {   // (no miss known below k yet)
+            jj[r] = j;
+            kk[r] = k;
+            const TableView t = c.table(j);
+            bk[r] = home_bucket(hbuf[k], t.bmask);
+            ld_bucket(t.keys, bk[r], v[r]);
+          }
         }
       }
-      const unsigned grp = __match_any_sync(FULL_MASK, jj);
-      const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
-      if (jj >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
-        atomicMin(&c.wm[jj], m);
+#pragma unroll
+      for (int r = 0; r < ILP; r++) {
+        int miss = 0x7FFFFFFF;
+        if (jj[r] >= 0) {
+          cnt++;
+          const uint64_t h = hbuf[kk[r]];
+          uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
+          if (bucket_scan(v[r], bk[r], h, &sl, &fr) < 0) {
+            const TableView t = c.table(jj[r]);
+            sl = table_find_free_from(t, h, (bk[r] + 1) & t.bmask, &err, &fr);
+          }
+          if (sl == SLOT_NONE) miss = kk[r];
+        }
+        const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
+        const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
+        if (jj[r] >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
+          atomicMin(&c.wm[jj[r]], m);
+      }
     }
     grp_bar<NT>();
-    c0 += CH;
-    if (threadIdx.x == 0) {
+    c0 += len;
+    if (threadIdx.x < 32) {
+      // the workers still open, in order, by ballots of warp 0
       int no = 0;
-      if (c0 < nb)
-        for (int j = 0; j < W; j++)
-          if (c.wm[j] >= c0) c.wopen[no++] = j;
-      S.nopen = no;
+      for (int j0 = 0; j0 < W; j0 += 32) {
+        const int j = j0 + (int)threadIdx.x;
+        const bool op = c0 < nb && j < W && c.wm[j] >= c0;
+        const unsigned bal = __ballot_sync(FULL_MASK, op);
+        if (op) c.wopen[no + __popc(bal & ((1u << threadIdx.x) - 1u))] = j;
+        no += __popc(bal);
+      }
+      if (threadIdx.x == 0) S.nopen = no;
     }
     grp_bar<NT>();
     if (S.nopen == 0) break;
@@ -1153,7 +1234,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
         if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
       } else {
-        probe_prefixes<NT_UPD>(c, hb, nb);
+        probe_prefixes<NT_UPD, MINB == 1 ? 4 : 1>(c, hb, nb);
       }
     } else if (lane == 0) {
       // ---- control thread, at the same time: completions and controller
