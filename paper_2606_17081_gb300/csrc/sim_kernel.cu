@@ -33,12 +33,7 @@ constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (w
 constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
 constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
 constexpr int PROBE_CAP = SIM_PROBE_CAP;   // W * nb up to which the probe captures every slot
-// lookups a thread keeps in flight in the full probe: 4 with one replica per
-// SM (2.9% faster on p2d than 2), 2 with two (the 128-register budget)
-template <int MINB>
-struct ProbeIlp {
-  static constexpr int value = MINB == 1 ? 4 : 2;
-};
+constexpr int PROBE_ILP = 2;             // lookups a thread keeps in flight
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -667,7 +662,7 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
 // TIER: m_j counts the leading blocks in G1 (a found slot's stamp at or
 // past the worker's b1); every pair's tier goes to ptier; the absent count
 // is of blocks in no tier.
-template <int NT, int PROBE_ILP, bool TIER = false>
+template <int NT, bool TIER = false>
 __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
@@ -1230,7 +1225,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     if (warp < NT_SIM / 32 - 1) {
       // ---- cached prefix on every worker (warps 0-6)
       if (full) {
-        probe_full<NT_UPD, ProbeIlp<MINB>::value, TIER>(c, hb, nb);
+        probe_full<NT_UPD, TIER>(c, hb, nb);
       } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
         if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
       } else {
