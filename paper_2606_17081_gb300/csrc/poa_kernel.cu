@@ -188,16 +188,18 @@ constexpr uint64_t DKEY_NONE = ~0ull;   // above dorder of every double but NaN
 
 // Edge weights out of worker j: for every k, the cheapest move of a request now
 // at j to k, min over those requests of c_qk - c_qj (ties: lowest row).
+template <int WT>
 __device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffers& b,
                                                int64_t base, int64_t m, int W, int j, int lane) {
   // per lane: the cheapest move to each k among its rows, as order keys
-  // (registers: the loops run over the fixed POA_WMAX with k < W guards);
+  // (registers: the loops run over the compile-time bound WT >= W with k < W
+  // guards);
   // four rows per lane in flight, each lane's rows in increasing order so
   // that ties keep the lowest row
-  uint64_t lk[POA_WMAX];
-  int lr[POA_WMAX];
+  uint64_t lk[WT];
+  int lr[WT];
 #pragma unroll
-  for (int k = 0; k < POA_WMAX; k++) { lk[k] = DKEY_NONE; lr[k] = -1; }
+  for (int k = 0; k < WT; k++) { lk[k] = DKEY_NONE; lr[k] = -1; }
   for (int64_t r0 = lane; r0 < m; r0 += 128) {
     int at[4];
 #pragma unroll
@@ -209,7 +211,7 @@ __device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffer
       const double* cr = b.cost + (base + r) * W;
       const double cj = cr[j];
 #pragma unroll
-      for (int k = 0; k < POA_WMAX; k++) {
+      for (int k = 0; k < WT; k++) {
         if (k < W && k != j) {
           const uint64_t key = dorder(__dsub_rn(cr[k], cj));
           if (key < lk[k]) { lk[k] = key; lr[k] = (int)r; }
@@ -218,7 +220,7 @@ __device__ __forceinline__ void poa_edges_from(PoaWarpShared& S, const PoaBuffer
     }
   }
 #pragma unroll
-  for (int k = 0; k < POA_WMAX; k++) {
+  for (int k = 0; k < WT; k++) {
     if (k < W) {
       uint64_t key = lk[k];
       int rr = lr[k];
@@ -276,6 +278,11 @@ __device__ __forceinline__ bool poa_next(const PoaProblem* __restrict__ probs, c
   }
 }
 
+// WT: a compile-time bound on W (the exact W for the common 3 and 6, else
+// POA_WMAX), so that the unrolled per-worker loops hold no dead iterations:
+// the solver's warps run different phases at once and its code must stay
+// small for the instruction cache.
+template <int WT>
 __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restrict__ probs,
                                                       PoaBuffers b, ModelConsts mc) {
   __shared__ PoaSolveShared P;
@@ -341,7 +348,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
       }
       __syncwarp();
       const int64_t nrem = (int64_t)S.num;
-      for (int j = 0; j < W; j++) poa_edges_from(S, b, base, m, W, j, lane);
+      for (int j = 0; j < W; j++) poa_edges_from<WT>(S, b, base, m, W, j, lane);
       __syncwarp();
       for (int64_t e = 0; e < nrem; e++) {
         const int64_t r0 = b.wkey[base + e];
@@ -360,7 +367,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
           uint64_t bk = DKEY_NONE;
           int bj = -1;
 #pragma unroll
-          for (int j = 0; j < POA_WMAX; j++) {
+          for (int j = 0; j < WT; j++) {
             const double dj = __shfl_sync(FULL_MASK, dk, j);
             if (j < W && lane < W && j != lane && S.wrow[j][lane] >= 0) {
               const uint64_t key = dorder(__dadd_rn(dj, S.wmin[j][lane]));
@@ -438,7 +445,7 @@ __global__ void __launch_bounds__(NT_POA) k_poa_solve(const PoaProblem* __restri
         }
         __syncwarp();
         for (int j = 0; j < W; j++)
-          if (S.dirty[j]) poa_edges_from(S, b, base, m, W, j, lane);
+          if (S.dirty[j]) poa_edges_from<WT>(S, b, base, m, W, j, lane);
         __syncwarp();
       }
     }
@@ -869,13 +876,15 @@ cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
     if ((e = cudaMemsetAsync(b.wnext, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
     int per_sm = 0;
     if (mc.W <= POA_WMAX) {
-      if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_poa_solve, NT_POA, 0)) !=
+      void (*kern)(const PoaProblem*, PoaBuffers, ModelConsts) =
+          mc.W == 3 ? k_poa_solve<3> : (mc.W == 6 ? k_poa_solve<6> : k_poa_solve<POA_WMAX>);
+      if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT_POA, 0)) !=
           cudaSuccess)
         return e;
       int64_t g = (b.nslots + NT_POA / 32 - 1) / (NT_POA / 32);
       const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
       g = g < cap ? g : cap;
-      k_poa_solve<<<(unsigned)(g > 0 ? g : 1), NT_POA, 0, st>>>(d_prob, b, mc);
+      kern<<<(unsigned)(g > 0 ? g : 1), NT_POA, 0, st>>>(d_prob, b, mc);
     } else {
       if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_poa_solve_wide, 32,
                                                              wsmem)) != cudaSuccess)
@@ -886,7 +895,9 @@ cudaError_t launch_poa(const PoaProblem* d_prob, int nprob, const PoaBuffers& b,
       k_poa_solve_wide<<<(unsigned)(g > 0 ? g : 1), 32, wsmem, st>>>(d_prob, b, mc);
     }
   } else if (mc.W <= POA_WMAX) {
-    k_poa_solve<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
+    void (*kern)(const PoaProblem*, PoaBuffers, ModelConsts) =
+        mc.W == 3 ? k_poa_solve<3> : (mc.W == 6 ? k_poa_solve<6> : k_poa_solve<POA_WMAX>);
+    kern<<<dim3(nprob, split), NT_POA, 0, st>>>(d_prob, b, mc);
   } else {
     // one warp per CTA: 8x the CTAs for the same windows in flight
     const int wsplit = split * (NT_POA / 32) > 128 ? 128 : split * (NT_POA / 32);
