@@ -81,3 +81,17 @@ def test_two_gloo_ranks_shard_replicas_and_take_max_time(tmp_path):
     assert r0["max"] == r1["max"] == [2.0, 10.0]
     # the reference arm prints only on rank 0
     assert r1["printed"] == ""
+
+
+def test_profiling_subsets():
+    # --replicas N keeps the plan's first N replicas; per-trace keeps the
+    # first replica of every trace (one hash launch over every trace)
+    import bench
+    from paper_2606_17081_gb300 import workloads as wk
+    full = wk.plan("grid", n_req=50)
+    assert bench._subset(full, "5") == [0, 1, 2, 3, 4]
+    idx = bench._subset(full, "per-trace")
+    assert len(idx) == len(full.trace_seeds)
+    assert sorted({full.replicas[k].trace for k in idx}) == list(range(len(full.trace_seeds)))
+    p, lo, hi = bench._plan("grid", n_req=50, subset="per-trace")
+    assert (lo, hi) == (0, len(idx)) and len(p.trace_seeds) == len(idx)
