@@ -194,11 +194,15 @@ def test_edge_cases():
 
 # ------------------------------------------------------------------ PoA (K4)
 
-def test_poa_matches_oracle_per_window():
+# W = 3 and W = 6 run the solver compiled for exactly that many workers, the
+# others the one compiled for up to 16; the selfish replicas' windows bind
+# their capacity (thousands of augmentations)
+@pytest.mark.parametrize("W,C", [(3, 256), (6, 512), (5, 320), (12, 768)])
+def test_poa_matches_oracle_per_window(W, C):
     tr = _rand_trace(3000, 41, len_hi=900)
-    reps = [wk.Replica(0, 256, wk.POLICY_DYNAMO, 0, 1.0, 0.0, 0, tr.n_req),
-            wk.Replica(0, 24, wk.POLICY_LOADBAL, 0, 0.0, 0.0, 0, tr.n_req)]
-    ctx = rs.Context(W=3, K=500)
+    reps = [wk.Replica(0, C, wk.POLICY_DYNAMO, 0, 1.0, 0.0, 0, tr.n_req),
+            wk.Replica(0, 8 * W, wk.POLICY_LOADBAL, 0, 0.0, 0.0, 0, tr.n_req)]
+    ctx = rs.Context(W=W, K=500)
     st, g = gpu_run(ctx, [tr], reps)
     assert st == 0
     cfg = oracle_cfg(ctx)
@@ -208,7 +212,7 @@ def test_poa_matches_oracle_per_window():
         assert abs(g[k]["result"]["poa_total"] - tot) <= 1e-4 * tot
         assert g[k]["result"]["n_windows"] == num.size
         # per-window values through poa_estimate on the same records
-        rec, t = rs.device_records(tr.n_req, 3)
+        rec, t = rs.device_records(tr.n_req, W)
         for f in ("worker", "completion", "ttft", "nbt"):
             t[f].copy_(torch.from_numpy(np.ascontiguousarray(o[f])))
         for f in ("n_frozen", "prefix"):
