@@ -551,7 +551,7 @@ __device__ __forceinline__ void wide_rescan(const PoaWide& S, const PoaBuffers& 
   }
 }
 
-__global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restrict__ probs,
+__global__ void __launch_bounds__(32, 1) k_poa_solve_wide(const PoaProblem* __restrict__ probs,
                                                        PoaBuffers b, ModelConsts mc) {
   extern __shared__ __align__(16) unsigned char wsm[];
   const int W = mc.W;
@@ -649,6 +649,39 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
           int ch[2] = {0, 0};
           double nd[2];
           int np[2];
+          uint64_t bk[2] = {DKEY_NONE, DKEY_NONE};
+          int bj[2] = {-1, -1};
+          // sources four at a time, both targets together: the loads and
+          // additions of a group are independent (one warp per CTA has no
+          // other warps to hide their latency); sources in increasing order,
+          // so ties keep the lowest j
+          for (uint64_t a = act; a;) {
+            int js[4];
+#pragma unroll
+            for (int u = 0; u < 4; u++) {
+              js[u] = a ? __ffsll((long long)a) - 1 : -1;
+              a &= a ? a - 1 : 0ull;
+            }
+            double dj[4];
+#pragma unroll
+            for (int u = 0; u < 4; u++) dj[u] = js[u] >= 0 ? S.dist[js[u]] : 0.0;
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+              const int k = lane + 32 * h;
+              if (k >= W) continue;
+              uint64_t key[4];
+#pragma unroll
+              for (int u = 0; u < 4; u++) {
+                const int j = js[u];
+                key[u] = DKEY_NONE;
+                if (j >= 0 && j != k && S.wrow[j * W + k] >= 0)
+                  key[u] = dorder(__dadd_rn(dj[u], S.wmin[j * W + k]));
+              }
+#pragma unroll
+              for (int u = 0; u < 4; u++)
+                if (key[u] < bk[h]) { bk[h] = key[u]; bj[h] = js[u]; }
+            }
+          }
 #pragma unroll
           for (int h = 0; h < 2; h++) {
             const int k = lane + 32 * h;
@@ -657,17 +690,9 @@ __global__ void __launch_bounds__(32) k_poa_solve_wide(const PoaProblem* __restr
             if (k >= W) continue;
             nd[h] = S.dist[k];
             np[h] = S.pred[k];
-            uint64_t bk = DKEY_NONE;
-            int bj = -1;
-            for (uint64_t a = act; a; a &= a - 1) {
-              const int j = __ffsll((long long)a) - 1;
-              if (j == k || S.wrow[j * W + k] < 0) continue;
-              const uint64_t key = dorder(__dadd_rn(S.dist[j], S.wmin[j * W + k]));
-              if (key < bk || (key == bk && j < bj)) { bk = key; bj = j; }
-            }
-            if (bj >= 0) {
-              const double v = dunorder(bk);
-              if (v < nd[h] - 1e-12) { nd[h] = v; np[h] = bj; ch[h] = 1; }
+            if (bj[h] >= 0) {
+              const double v = dunorder(bk[h]);
+              if (v < nd[h] - 1e-12) { nd[h] = v; np[h] = bj[h]; ch[h] = 1; }
             }
           }
           __syncwarp();
