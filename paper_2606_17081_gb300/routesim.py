@@ -280,8 +280,9 @@ def sweep_knee(ctx, records: rs_records, row_start, load, sweep_start, pct: int 
 def poa_estimate_noalloc(cfg: rs_config, records: rs_records, n: int, numer_dev, opt_dev,
                          count_dev, max_windows: int, poa_total_dev, n_windows_dev,
                          stream: int = 0) -> None:
-    """Eq. (12) estimate in the library's static scratch (no allocation);
-    outputs stay in device memory."""
+    """Same result as poa_estimate, computed in the library's fixed static
+    device array (nothing allocated, for callers that cannot allocate device
+    memory); outputs stay in device memory."""
     st = lib().poa_estimate_noalloc(C.byref(cfg), C.byref(records), n, _ptr(numer_dev),
                                     _ptr(opt_dev), _ptr(count_dev), max_windows,
                                     _ptr(poa_total_dev), _ptr(n_windows_dev),
