@@ -47,13 +47,13 @@ __device__ __forceinline__ uint64_t content_of(const BlockBytes& b, int shift) {
                           (uint32_t)b.v2.x, (uint32_t)b.v2.y, (uint32_t)b.v2.z, (uint32_t)b.v2.w,
                           (uint32_t)b.v3.x, (uint32_t)b.v3.y, (uint32_t)b.v3.z, (uint32_t)b.v3.w,
                           (uint32_t)b.v4.x, (uint32_t)b.v4.y, (uint32_t)b.v4.z, (uint32_t)b.v4.w};
-  uint32_t w[16];
-  switch (shift) {
-    case 0: take16<0>(a, w); break;
-    case 1: take16<1>(a, w); break;
-    case 2: take16<2>(a, w); break;
-    default: take16<3>(a, w); break;
-  }
+  // w[j] = a[j + shift] by two selects on the shift's bits (no branch)
+  uint32_t c[19], w[16];
+  const bool s1 = shift & 1, s2 = shift & 2;
+#pragma unroll
+  for (int j = 0; j < 19; j++) c[j] = s1 ? a[j + 1] : a[j];
+#pragma unroll
+  for (int j = 0; j < 16; j++) w[j] = s2 ? c[j + 2] : c[j];
   return block_content16(w);
 }
 
