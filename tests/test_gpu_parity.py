@@ -350,3 +350,28 @@ def test_static_policies_and_static_poa(W):
     if W == 3:   # queueing at C = 256: the observed estimate exceeds the static one
         sat = [g[k]["result"] for k, r in enumerate(reps) if r.C == 256]
         assert all(x["poa_total"] > x["poa_static"] for x in sat)
+
+
+# W nb above the 2048 pairs the full probe captures: the prompts' cached
+# prefixes come from the rounds of first-miss walks (four lookups in flight
+# per thread with one replica per SM, one with two), checked in both launch
+# modes against the oracle
+@pytest.mark.parametrize("nrep", [8, 160])
+def test_long_prompts_first_miss_rounds(nrep):
+    spec = wk.TraceSpec(n_req=120, len_kind="uniform", len_min=4200, len_max=8000, n_groups=5,
+                        prefix_min=1000, prefix_max=4000, zipf_s=0.8, out_kind="uniform",
+                        out_min=1, out_max=200)
+    tr = wk.make_trace(spec, 13)
+    W = 8
+    assert int((np.diff(tr.offsets) // 16).min()) * W > 2048
+    ctx = rs.Context(W=W, K=1024)
+    reps = [wk.Replica(0, 4 + (k % 5) * 8, wk.POLICY_DYNAMO if k % 2 == 0 else wk.POLICY_LOADBAL,
+                       0, 1.0 if k % 2 == 0 else 0.0, 0.5 if k % 4 == 0 else 0.0, k, tr.n_req)
+            for k in range(nrep)]
+    st, g = gpu_run(ctx, [tr], reps)
+    assert st == 0
+    cfg = oracle_cfg(ctx)
+    for k in sorted({0, 1, nrep // 2 + 1, nrep - 1}):
+        o = oracle_run(cfg, tr, reps[k])
+        assert_replica_equal(g[k], o, W)
+    assert max(x["result"]["evicted_blocks"] for x in g) > 0
