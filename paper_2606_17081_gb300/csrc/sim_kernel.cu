@@ -551,8 +551,9 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
 // (threads of the group), when W nb is too large to look every pair up at
 // once.  Rounds over the workers still undecided: a round looks up the next
 // `len` blocks of each open worker, with len = ILP NT / (open workers) so
-// that a round is ILP lookups per thread (4 with one replica per SM, 1 within
-// the two-per-SM register budget), all issued before any is resolved;
+// that a round is ILP lookups per thread (4 with one replica per SM under LRU,
+// 1 within the two-per-SM register budget or under frequency eviction, whose
+// heap leaves no registers for more), all issued before any is resolved;
 // a worker is decided once a miss falls in its window.  Most workers miss at
 // their first block, so the few left open after the first round get long
 // windows.
@@ -1229,7 +1230,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
       } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
         if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
       } else {
-        probe_prefixes<NT_UPD, MINB == 1 ? 4 : 1>(c, hb, nb);
+        probe_prefixes<NT_UPD, MINB == 1 && MODE == SIM_LRU ? 4 : 1>(c, hb, nb);
       }
     } else if (lane == 0) {
       // ---- control thread, at the same time: completions and controller

@@ -354,10 +354,10 @@ def test_static_policies_and_static_poa(W):
 
 # W nb above the 2048 pairs the full probe captures: the prompts' cached
 # prefixes come from the rounds of first-miss walks (four lookups in flight
-# per thread with one replica per SM, one with two), checked in both launch
-# modes against the oracle
-@pytest.mark.parametrize("nrep", [8, 160])
-def test_long_prompts_first_miss_rounds(nrep):
+# per thread with one replica per SM under LRU, one with two per SM or under
+# frequency eviction), checked in both launch modes against the oracle
+@pytest.mark.parametrize("nrep,freq", [(8, False), (160, False), (8, True)])
+def test_long_prompts_first_miss_rounds(nrep, freq):
     spec = wk.TraceSpec(n_req=120, len_kind="uniform", len_min=4200, len_max=8000, n_groups=5,
                         prefix_min=1000, prefix_max=4000, zipf_s=0.8, out_kind="uniform",
                         out_min=1, out_max=200)
@@ -368,6 +368,9 @@ def test_long_prompts_first_miss_rounds(nrep):
     reps = [wk.Replica(0, 4 + (k % 5) * 8, wk.POLICY_DYNAMO if k % 2 == 0 else wk.POLICY_LOADBAL,
                        0, 1.0 if k % 2 == 0 else 0.0, 0.5 if k % 4 == 0 else 0.0, k, tr.n_req)
             for k in range(nrep)]
+    if freq:
+        for r in reps:
+            r.eviction, r.freq_max, r.decay_s = rs.RS_EVICT_FREQ, 6, 2.0
     st, g = gpu_run(ctx, [tr], reps)
     assert st == 0
     cfg = oracle_cfg(ctx)
