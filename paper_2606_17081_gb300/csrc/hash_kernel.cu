@@ -138,8 +138,11 @@ cudaError_t launch_block_hash(const HashJob* jobs_dev, int njobs, int64_t total_
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  int64_t nblk = (total_req + HASH_NT / 32 - 1) / (HASH_NT / 32);   // one warp per request
-  if (nblk > (int64_t)sms * 16) nblk = (int64_t)sms * 16;
+  // one warp per request, up to 64 CTAs per SM (six are resident at a time):
+  // prompt lengths vary, and short grid-stride runs per warp leave a shorter
+  // tail than long ones (the cap was chosen by measurement)
+  int64_t nblk = (total_req + HASH_NT / 32 - 1) / (HASH_NT / 32);
+  if (nblk > (int64_t)sms * 64) nblk = (int64_t)sms * 64;
   k_block_hash<<<(unsigned)nblk, HASH_NT, 0, st>>>(jobs_dev, njobs, total_req, seed, nbmax_out);
   return cudaGetLastError();
 }
