@@ -344,21 +344,30 @@ __device__ __forceinline__ void ld_bucket(const uint64_t* keys, uint32_t b, uint
 constexpr uint32_t FREE_TOMB = 0x80000000u;
 
 // Resolves one loaded bucket: returns 1 (found, *slot set), 0 (absent: the
-// bucket holds an EMPTY key) or -1 (continue with the next bucket).
+// bucket holds an EMPTY key) or -1 (continue with the next bucket).  *fr, if
+// still SLOT_NONE, becomes the bucket's first EMPTY or TOMB slot before the
+// match (before the end when h is absent).  Branch-free: the eight keys give
+// three bit masks, so the lanes of a warp never diverge on where h sits.
 __device__ __forceinline__ int bucket_scan(const uint64_t (&v)[BUCKET], uint32_t b, uint64_t h,
                                            uint32_t* slot, uint32_t* fr) {
-  bool empty = false;
+  unsigned hit = 0, fre = 0, tomb = 0;
 #pragma unroll
   for (int q = 0; q < BUCKET; q++) {
-    if (v[q] == h) {
-      *slot = (uint32_t)BUCKET * b + q;
-      return 1;
-    }
-    if (v[q] < 2 && *fr == SLOT_NONE)
-      *fr = ((uint32_t)BUCKET * b + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
-    empty |= v[q] == KEY_EMPTY;
+    hit |= (unsigned)(v[q] == h) << q;
+    fre |= (unsigned)(v[q] < 2) << q;   // EMPTY or TOMB
+    tomb |= (unsigned)(v[q] == KEY_TOMB) << q;
   }
-  return empty ? 0 : -1;
+  const unsigned before = hit ? (hit & (0u - hit)) - 1u : (1u << BUCKET) - 1u;   // before the match
+  const unsigned f = fre & before;
+  if (f && *fr == SLOT_NONE) {
+    const int q = __ffs(f) - 1;
+    *fr = ((uint32_t)BUCKET * b + q) | ((tomb >> q) & 1u ? FREE_TOMB : 0u);
+  }
+  if (hit) {
+    *slot = (uint32_t)BUCKET * b + (__ffs(hit) - 1);
+    return 1;
+  }
+  return (fre & ~tomb) ? 0 : -1;
 }
 
 __device__ __forceinline__ uint32_t table_find_free_from(const TableView& t, uint64_t h,

@@ -547,6 +547,20 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
 
 // ------------------------------------------------------------ routing step
 
+// A warp's lookups of one worker sit at consecutive lanes, on consecutive
+// blocks (lanes past the work or past a known miss hold j = -1): the run of
+// equal j around this lane as a lane mask, from the run heads by one shuffle
+// and one ballot.
+__device__ __forceinline__ unsigned run_mask(int j, int lane) {
+  const int jp = __shfl_up_sync(FULL_MASK, j, 1);
+  const unsigned heads = __ballot_sync(FULL_MASK, lane == 0 || jp != j);
+  const unsigned upto = (2u << lane) - 1u;   // lanes 0..lane
+  const int lo = 31 - __clz(heads & upto);
+  const unsigned above = heads & ~upto;
+  const unsigned below_next = above ? (above & (0u - above)) - 1u : FULL_MASK;
+  return below_next & ~((1u << lo) - 1u);
+}
+
 // m_j: leading blocks of the prompt found in worker j's cache, for every j
 // (threads of the group), when W nb is too large to look every pair up at
 // once.  Rounds over the workers still undecided: a round looks up the next
@@ -578,21 +592,24 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
       if constexpr (ILP == 1) {
         // one lookup per thread, resolved where it is issued
         const int it = base + threadIdx.x;
-        int jj = -1, miss = 0x7FFFFFFF;
+        int jj = -1, k = 0;
+        bool miss = false;
         if (it < total) {
           const int o = (int)(((float)it + 0.5f) * inv_len);
           const int j = c.wopen[o];
-          const int k = c0 + (it - o * len);
+          k = c0 + (it - o * len);
           if (k < c.wm[j]) {   // (no miss known below k yet)
             jj = j;
             cnt++;
-            if (table_find(c.table(j), hbuf[k], &err) == SLOT_NONE) miss = k;
+            miss = table_find(c.table(j), hbuf[k], &err) == SLOT_NONE;
           }
         }
-        const unsigned grp = __match_any_sync(FULL_MASK, jj);
-        const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
-        if (jj >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
-          atomicMin(&c.wm[jj], m);
+        // the run's first miss: blocks rise by one per lane along a run
+        const int lane = (int)(threadIdx.x & 31);
+        const unsigned grp = run_mask(jj, lane);
+        const unsigned mb = __ballot_sync(FULL_MASK, miss) & grp;
+        if (jj >= 0 && mb && (__ffs(grp) - 1) == lane)
+          atomicMin(&c.wm[jj], k + (__ffs(mb) - 1) - lane);
         continue;
       }
       int jj[ILP], kk[ILP];
@@ -628,10 +645,12 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
           }
           if (sl == SLOT_NONE) miss = kk[r];
         }
-        const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
-        const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
-        if (jj[r] >= 0 && m != 0x7FFFFFFF && (__ffs(grp) - 1) == (int)(threadIdx.x & 31))
-          atomicMin(&c.wm[jj[r]], m);
+        // the run's first miss: blocks rise by one per lane along a run
+        const int lane = (int)(threadIdx.x & 31);
+        const unsigned grp = run_mask(jj[r], lane);
+        const unsigned mb = __ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp;
+        if (jj[r] >= 0 && mb && (__ffs(grp) - 1) == lane)
+          atomicMin(&c.wm[jj[r]], kk[r] + (__ffs(mb) - 1) - lane);
       }
     }
     grp_bar<NT>();
@@ -729,14 +748,16 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
           miss = kk[r];
         }
       }
-      const unsigned grp = __match_any_sync(FULL_MASK, jj[r]);
-      const int m = (int)__reduce_min_sync(grp, (unsigned)miss);
+      // per run of lanes on one worker (blocks rise by one per lane): the
+      // first miss and the absent count
+      const int lane = (int)(threadIdx.x & 31);
+      const unsigned grp = run_mask(jj[r], lane);
+      const unsigned mb = __ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp;
       const unsigned nab =
-          __popc(__ballot_sync(FULL_MASK, TIER ? absent : miss != 0x7FFFFFFF) & grp);
+          TIER ? __popc(__ballot_sync(FULL_MASK, absent) & grp) : __popc(mb);
       // (tiers: a block below G1 ends the prefix though it is present)
-      if (jj[r] >= 0 && (__ffs(grp) - 1) == (int)(threadIdx.x & 31) &&
-          (nab || (TIER && m != 0x7FFFFFFF))) {
-        atomicMin(&c.wm[jj[r]], m);
+      if (jj[r] >= 0 && (__ffs(grp) - 1) == lane && (nab || (TIER && mb))) {
+        if (mb) atomicMin(&c.wm[jj[r]], kk[r] + (__ffs(mb) - 1) - lane);
         if (nab) atomicAdd(&c.wabs[jj[r]], (int)nab);   // absent blocks, for the victim count
       }
     }
