@@ -108,7 +108,7 @@ __host__ __device__ inline SimLayout make_sim_layout(int W, int nbmax, int cmax,
   TAKE(wqt, 4 * (size_t)W, 4)
   TAKE(wm, 4 * (size_t)W, 4)
   TAKE(wcost, 4 * (size_t)W * (NT_SIM / 32), 4)   // one cost row per warp
-  TAKE(wopen, 4 * (size_t)W, 4)
+  TAKE(wopen, (size_t)(NT_SIM / 32) * WMAX, 4)
   TAKE(wabs, 4 * (size_t)W, 4)
   TAKE(kind, nb, 1)
   TAKE(evk, nb, 1)
@@ -161,7 +161,7 @@ struct SimScalars {
   unsigned long long probes;
   uint64_t sel_prefix;
   int32_t in_flight, nheap, nfree, evres, status, jstar, regime, up_cnt, down_cnt;
-  int32_t have_L, have_ewma, max_regime, pend_cur, nopen, sel_kk;
+  int32_t have_L, have_ewma, max_regime, pend_cur, sel_kk;
   uint32_t dclock;             // decay step of the request being updated (frequency eviction)
   int64_t kv[5];               // Game 2: own G1 / G2 / G3, remote, recompute blocks
   double kv_cost;              // summed Eq. kv-cost
@@ -190,7 +190,8 @@ struct SimCtx {
   FreqMeta* wfreq;
   TierMeta* wtier;    // Game 2 band boundaries per worker (tiered)
   uint8_t* ptier;     // [W][nb] tier of each (worker, block) pair, 0 = absent (tiered)
-  int32_t *winserv, *wqh, *wqt, *wm, *wopen, *wabs;
+  int32_t *winserv, *wqh, *wqt, *wm, *wabs;
+  uint8_t* wopen;     // [NT_SIM / 32][WMAX] each probing warp's open workers
   uint32_t *pslot, *pfree;
   int64_t* wA;
   float* wcost;
@@ -547,18 +548,43 @@ __device__ __forceinline__ void tick_cta(SimCtx& c) {
 
 // ------------------------------------------------------------ routing step
 
-// A warp's lookups of one worker sit at consecutive lanes, on consecutive
-// blocks (lanes past the work or past a known miss hold j = -1): the run of
-// equal j around this lane as a lane mask, from the run heads by one shuffle
-// and one ballot.
-__device__ __forceinline__ unsigned run_mask(int j, int lane) {
-  const int jp = __shfl_up_sync(FULL_MASK, j, 1);
-  const unsigned heads = __ballot_sync(FULL_MASK, lane == 0 || jp != j);
-  const unsigned upto = (2u << lane) - 1u;   // lanes 0..lane
-  const int lo = 31 - __clz(heads & upto);
-  const unsigned above = heads & ~upto;
-  const unsigned below_next = above ? (above & (0u - above)) - 1u : FULL_MASK;
-  return below_next & ~((1u << lo) - 1u);
+// A warp's lookups sit at consecutive lanes; those of one worker cover
+// consecutive blocks, the lane holding the window's position kw on the
+// worker's span of `span` blocks.  The lanes of that span in this warp, as a
+// mask: from lane - kw to lane - kw + span - 1, clipped to the warp.
+__device__ __forceinline__ unsigned span_mask(int lane, int kw, int span) {
+  const int lo = lane - kw > 0 ? lane - kw : 0;
+  const int hi = lane - kw + span;   // one past the span's last lane
+  const unsigned below_hi = hi >= 32 ? FULL_MASK : (hi > 0 ? (1u << hi) - 1u : 0u);
+  return below_hi & ~((1u << lo) - 1u);
+}
+
+// Resolves ILP loaded home buckets: sl[r] the slot holding hh[r] or
+// SLOT_NONE, fr[r] the first free slot of its probe path.  A bucket full of
+// other keys (rare at the tables' load) continues along the probe sequence
+// after all of them are scanned, so the common case runs straight through.
+template <int ILP>
+__device__ __forceinline__ void resolve_buckets(const SimCtx& c, const uint64_t (&v)[ILP][BUCKET],
+                                                const uint32_t (&bk)[ILP],
+                                                const uint64_t (&hh)[ILP], const int (&jj)[ILP],
+                                                uint32_t (&sl)[ILP], uint32_t (&fr)[ILP],
+                                                int* err) {
+  bool cont[ILP], any = false;
+#pragma unroll
+  for (int r = 0; r < ILP; r++) {
+    sl[r] = SLOT_NONE;
+    fr[r] = SLOT_NONE;
+    cont[r] = bucket_scan(v[r], bk[r], hh[r], &sl[r], &fr[r]) < 0 && jj[r] >= 0;
+    any |= cont[r];
+  }
+  if (any) {
+#pragma unroll
+    for (int r = 0; r < ILP; r++)
+      if (cont[r]) {
+        const TableView t = c.table(jj[r]);
+        sl[r] = table_find_free_from(t, hh[r], (bk[r] + 1) & t.bmask, err, &fr[r]);
+      }
+  }
 }
 
 // m_j: leading blocks of the prompt found in worker j's cache, for every j
@@ -570,108 +596,79 @@ __device__ __forceinline__ unsigned run_mask(int j, int lane) {
 // heap leaves no registers for more), all issued before any is resolved;
 // a worker is decided once a miss falls in its window.  Most workers miss at
 // their first block, so the few left open after the first round get long
-// windows.
+// windows.  Each warp lists the open workers for itself after the round's
+// barrier: a miss of the next round lowers m_j only to a block at or past
+// that round's start, so a worker's open state does not depend on when a
+// warp reads it, and no second barrier is needed.
 template <int NT, int ILP>
 __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
+  const int lane = (int)(threadIdx.x & 31);
+  uint8_t* wl = c.wopen + (threadIdx.x >> 5) * WMAX;   // this warp's open workers
+  for (int j = lane; j < W; j += 32) wl[j] = (uint8_t)j;
+  __syncwarp();
+  int nopen = W;
   int c0 = 0;
   int err = 0;
   unsigned cnt = 0;
   for (;;) {
-    const int nopen = S.nopen;
     int len = (ILP * NT) / nopen;
     if (len < 1) len = 1;
-    if (len > nb - c0) len = nb - c0;
-    const int total = len > 0 ? nopen * len : 0;
+    if (len > nb - c0) len = nb - c0;   // (>= 1: the workers listed are open, so c0 < nb)
+    const int total = nopen * len;      // <= ILP NT
     // open worker of lookup `it` = floor(it / len): (it + 0.5) / len lies at
     // least 0.5 / len from an integer and it < ILP NT, so the float product
     // truncates to it exactly
-    const float inv_len = len > 0 ? 1.0f / (float)len : 0.0f;
-    for (int base = 0; base < total; base += ILP * NT) {   // uniform
-      if constexpr (ILP == 1) {
-        // one lookup per thread, resolved where it is issued
-        const int it = base + threadIdx.x;
-        int jj = -1, k = 0;
-        bool miss = false;
-        if (it < total) {
-          const int o = (int)(((float)it + 0.5f) * inv_len);
-          const int j = c.wopen[o];
-          k = c0 + (it - o * len);
-          if (k < c.wm[j]) {   // (no miss known below k yet)
-            jj = j;
-            cnt++;
-            miss = table_find(c.table(j), hbuf[k], &err) == SLOT_NONE;
-          }
-        }
-        // the run's first miss: blocks rise by one per lane along a run
-        const int lane = (int)(threadIdx.x & 31);
-        const unsigned grp = run_mask(jj, lane);
-        const unsigned mb = __ballot_sync(FULL_MASK, miss) & grp;
-        if (jj >= 0 && mb && (__ffs(grp) - 1) == lane)
-          atomicMin(&c.wm[jj], k + (__ffs(mb) - 1) - lane);
-        continue;
-      }
-      int jj[ILP], kk[ILP];
-      uint64_t v[ILP][BUCKET];
-      uint32_t bk[ILP];
+    const float inv_len = 1.0f / (float)len;
+    int jj[ILP], kk[ILP], kw[ILP];
+    uint64_t hh[ILP], v[ILP][BUCKET];
+    uint32_t bk[ILP];
+    // every lookup's home bucket requested before any is resolved; a thread
+    // past the round's lookups repeats the round's last one (in bounds, unused)
 #pragma unroll
-      for (int r = 0; r < ILP; r++) {
-        const int it = base + r * NT + threadIdx.x;
-        jj[r] = -1;
-        if (it < total) {
-          const int o = (int)(((float)it + 0.5f) * inv_len);
-          const int j = c.wopen[o];
-          const int k = c0 + (it - o * len);
-          if (k < c.wm[j]) {   // (no miss known below k yet)
-            jj[r] = j;
-            kk[r] = k;
-            const TableView t = c.table(j);
-            bk[r] = home_bucket(hbuf[k], t.bmask);
-            ld_bucket(t.keys, bk[r], v[r]);
-          }
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < ILP; r++) {
-        int miss = 0x7FFFFFFF;
-        if (jj[r] >= 0) {
-          cnt++;
-          const uint64_t h = hbuf[kk[r]];
-          uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
-          if (bucket_scan(v[r], bk[r], h, &sl, &fr) < 0) {
-            const TableView t = c.table(jj[r]);
-            sl = table_find_free_from(t, h, (bk[r] + 1) & t.bmask, &err, &fr);
-          }
-          if (sl == SLOT_NONE) miss = kk[r];
-        }
-        // the run's first miss: blocks rise by one per lane along a run
-        const int lane = (int)(threadIdx.x & 31);
-        const unsigned grp = run_mask(jj[r], lane);
-        const unsigned mb = __ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp;
-        if (jj[r] >= 0 && mb && (__ffs(grp) - 1) == lane)
-          atomicMin(&c.wm[jj[r]], kk[r] + (__ffs(mb) - 1) - lane);
-      }
+    for (int r = 0; r < ILP; r++) {
+      const int it0 = r * NT + (int)threadIdx.x;
+      const int it = it0 < total ? it0 : total - 1;
+      const int o = (int)(((float)it + 0.5f) * inv_len);
+      const int j = wl[o];
+      kw[r] = it - o * len;
+      kk[r] = c0 + kw[r];
+      jj[r] = it0 < total && kk[r] < c.wm[j] ? j : -1;   // (no miss known below k yet)
+      hh[r] = hbuf[kk[r]];
+      const TableView t = c.table(j);
+      bk[r] = home_bucket(hh[r], t.bmask);
+      ld_bucket(t.keys, bk[r], v[r]);
     }
-    grp_bar<NT>();
+    uint32_t sl[ILP], fr[ILP];
+    resolve_buckets<ILP>(c, v, bk, hh, jj, sl, fr, &err);
+#pragma unroll
+    for (int r = 0; r < ILP; r++) {
+      if (r > 0 && r * NT >= total) break;   // (uniform)
+      cnt += jj[r] >= 0;
+      // the first miss of the worker's window in this warp: its lanes rise
+      // by one block each, so it is the window's lowest missing lane, and
+      // the window's lowest lane here (kw = 0, or lane 0) records it
+      const unsigned mb =
+          __ballot_sync(FULL_MASK, jj[r] >= 0 && sl[r] == SLOT_NONE) & span_mask(lane, kw[r], len);
+      if (jj[r] >= 0 && mb && (kw[r] == 0 || lane == 0))
+        atomicMin(&c.wm[jj[r]], kk[r] + (__ffs(mb) - 1) - lane);
+    }
+    grp_bar<NT>();   // every miss of the round is in wm
     c0 += len;
-    if (threadIdx.x < 32) {
-      // the workers still open, in order, by ballots of warp 0
-      int no = 0;
-      for (int j0 = 0; j0 < W; j0 += 32) {
-        const int j = j0 + (int)threadIdx.x;
-        const bool op = c0 < nb && j < W && c.wm[j] >= c0;
-        const unsigned bal = __ballot_sync(FULL_MASK, op);
-        if (op) c.wopen[no + __popc(bal & ((1u << threadIdx.x) - 1u))] = j;
-        no += __popc(bal);
-      }
-      if (threadIdx.x == 0) S.nopen = no;
+    nopen = 0;
+    for (int j0 = 0; j0 < W; j0 += 32) {
+      const int j = j0 + lane;
+      const bool op = c0 < nb && j < W && c.wm[j] >= c0;
+      const unsigned bal = __ballot_sync(FULL_MASK, op);
+      if (op) wl[nopen + __popc(bal & ((1u << lane) - 1u))] = (uint8_t)j;
+      nopen += __popc(bal);
     }
-    grp_bar<NT>();
-    if (S.nopen == 0) break;
+    __syncwarp();
+    if (nopen == 0) break;
   }
   cnt = __reduce_add_sync(FULL_MASK, cnt);
-  if ((threadIdx.x & 31) == 0 && cnt) atomicAdd(&S.probes, (unsigned long long)cnt);
+  if (lane == 0 && cnt) atomicAdd(&S.probes, (unsigned long long)cnt);
   if (err) S.status = RS_ERR_TIMEOUT;
 }
 
@@ -687,76 +684,75 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
   const int total = W * nb;
+  const int lane = (int)(threadIdx.x & 31);
+  // worker of pair `it` = floor(it / nb): (it + 0.5) / nb lies at least
+  // 0.5 / nb from an integer, and with W nb <= PROBE_CAP the float product's
+  // error stays far below that, so it truncates to the quotient exactly
+  const float inv_nb = nb > 0 ? 1.0f / (float)nb : 0.0f;
   int err = 0;
   for (int base = 0; base < total; base += NT * PROBE_ILP) {   // uniform
     int jj[PROBE_ILP], kk[PROBE_ILP];
-    uint64_t v[PROBE_ILP][BUCKET];
+    uint64_t hh[PROBE_ILP], v[PROBE_ILP][BUCKET];
     uint64_t stw[PROBE_ILP][TIER ? 4 : 1];   // tiers: the home bucket's 8 stamps, beside its keys
     uint32_t bk[PROBE_ILP];
+    // every pair's home bucket requested before any is resolved; a thread
+    // past the pairs repeats the last one (in bounds, unused)
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
-      const int it = base + r * NT + threadIdx.x;
-      jj[r] = -1;
-      if (it < total) {
-        const int j = it / nb;
-        jj[r] = j;
-        kk[r] = it - j * nb;
-        const TableView t = c.table(j);
-        bk[r] = home_bucket(hbuf[kk[r]], t.bmask);
-        ld_bucket(t.keys, bk[r], v[r]);
-        if (TIER)   // one 32-byte sector: stamps are 4-byte, buckets of 8 start 32-byte aligned
-          ld_keys4(reinterpret_cast<const uint64_t*>(t.stamp + (size_t)BUCKET * bk[r]), stw[r][0],
-                   stw[r][TIER ? 1 : 0], stw[r][TIER ? 2 : 0], stw[r][TIER ? 3 : 0]);
-      }
+      const int it0 = base + r * NT + (int)threadIdx.x;
+      const int it = it0 < total ? it0 : total - 1;
+      const int j = (int)(((float)it + 0.5f) * inv_nb);
+      jj[r] = it0 < total ? j : -1;
+      kk[r] = it - j * nb;
+      hh[r] = hbuf[kk[r]];
+      const TableView t = c.table(j);
+      bk[r] = home_bucket(hh[r], t.bmask);
+      ld_bucket(t.keys, bk[r], v[r]);
+      if (TIER)   // one 32-byte sector: stamps are 4-byte, buckets of 8 start 32-byte aligned
+        ld_keys4(reinterpret_cast<const uint64_t*>(t.stamp + (size_t)BUCKET * bk[r]), stw[r][0],
+                 stw[r][TIER ? 1 : 0], stw[r][TIER ? 2 : 0], stw[r][TIER ? 3 : 0]);
     }
+    uint32_t sl[PROBE_ILP], fr[PROBE_ILP];
+    resolve_buckets<PROBE_ILP>(c, v, bk, hh, jj, sl, fr, &err);
 #pragma unroll
     for (int r = 0; r < PROBE_ILP; r++) {
-      const int it = base + r * NT + threadIdx.x;
-      int miss = 0x7FFFFFFF;
-      bool absent = false;
+      const int it = base + r * NT + (int)threadIdx.x;
+      bool miss = false, absent = false;
       if (jj[r] >= 0) {
-        const uint64_t h = hbuf[kk[r]];
-        uint32_t sl = SLOT_NONE, fr = SLOT_NONE;
-        if (bucket_scan(v[r], bk[r], h, &sl, &fr) < 0) {
-          // bucket full of other keys: continue along the probe sequence
-          const TableView t = c.table(jj[r]);
-          sl = table_find_free_from(t, h, (bk[r] + 1) & t.bmask, &err, &fr);
-        }
-        c.pslot[it] = sl;
-        c.pfree[it] = fr;
+        c.pslot[it] = sl[r];
+        c.pfree[it] = fr[r];
         if (TIER) {
           int tier = 0;
-          if (sl != SLOT_NONE) {
+          if (sl[r] != SLOT_NONE) {
             uint32_t st;
-            if (sl / BUCKET == bk[r]) {   // in the home bucket: its stamp came with the keys
-              const uint32_t q = sl % BUCKET;
+            if (sl[r] / BUCKET == bk[r]) {   // in the home bucket: its stamp came with the keys
+              const uint32_t q = sl[r] % BUCKET;
               const uint64_t w2 = q < 2 ? stw[r][0]
                                         : (q < 4 ? stw[r][TIER ? 1 : 0]
                                                  : (q < 6 ? stw[r][TIER ? 2 : 0]
                                                           : stw[r][TIER ? 3 : 0]));
               st = (uint32_t)(q & 1u ? w2 >> 32 : w2);
             } else {
-              st = __ldcg(c.table(jj[r]).stamp + sl);
+              st = __ldcg(c.table(jj[r]).stamp + sl[r]);
             }
             const TierMeta tm = c.wtier[jj[r]];
             tier = st >= tm.b1 ? 1 : (st >= tm.b2 ? 2 : 3);
           }
           c.ptier[it] = (uint8_t)tier;
-          absent = sl == SLOT_NONE;
-          if (tier != 1) miss = kk[r];
-        } else if (sl == SLOT_NONE) {
-          miss = kk[r];
+          absent = sl[r] == SLOT_NONE;
+          miss = tier != 1;
+        } else {
+          miss = sl[r] == SLOT_NONE;
         }
       }
-      // per run of lanes on one worker (blocks rise by one per lane): the
-      // first miss and the absent count
-      const int lane = (int)(threadIdx.x & 31);
-      const unsigned grp = run_mask(jj[r], lane);
-      const unsigned mb = __ballot_sync(FULL_MASK, miss != 0x7FFFFFFF) & grp;
-      const unsigned nab =
-          TIER ? __popc(__ballot_sync(FULL_MASK, absent) & grp) : __popc(mb);
+      // per worker's lanes in this warp (blocks rise by one per lane): the
+      // first miss and the absent count, recorded by the worker's lowest
+      // lane here (block 0, or lane 0)
+      const unsigned span = span_mask(lane, kk[r], nb);
+      const unsigned mb = __ballot_sync(FULL_MASK, miss) & span;
+      const unsigned nab = TIER ? __popc(__ballot_sync(FULL_MASK, absent) & span) : __popc(mb);
       // (tiers: a block below G1 ends the prefix though it is present)
-      if (jj[r] >= 0 && (__ffs(grp) - 1) == lane && (nab || (TIER && mb))) {
+      if (jj[r] >= 0 && (kk[r] == 0 || lane == 0) && (nab || (TIER && mb))) {
         if (mb) atomicMin(&c.wm[jj[r]], kk[r] + (__ffs(mb) - 1) - lane);
         if (nab) atomicAdd(&c.wabs[jj[r]], (int)nab);   // absent blocks, for the victim count
       }
@@ -1089,10 +1085,8 @@ __device__ __forceinline__ void probe_setup(SimCtx& c, const ReqState& q, int la
   const int W = c.L->mc.W;
   for (int j = lane; j < W; j += 32) {
     c.wm[j] = q.nb;
-    c.wopen[j] = j;
     c.wabs[j] = 0;
   }
-  if (lane == 0) c.S->nopen = W;
 }
 
 // Block hashes of a request into a staging buffer (lanes of one warp).
@@ -1154,7 +1148,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
   c.wqh = reinterpret_cast<int32_t*>(smem + lay.wqh);
   c.wqt = reinterpret_cast<int32_t*>(smem + lay.wqt);
   c.wm = reinterpret_cast<int32_t*>(smem + lay.wm);
-  c.wopen = reinterpret_cast<int32_t*>(smem + lay.wopen);
+  c.wopen = reinterpret_cast<uint8_t*>(smem + lay.wopen);
   c.wabs = reinterpret_cast<int32_t*>(smem + lay.wabs);
   c.wA = reinterpret_cast<int64_t*>(smem + lay.wA);
   c.wcost = reinterpret_cast<float*>(smem + lay.wcost);
