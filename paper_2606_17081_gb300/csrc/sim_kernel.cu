@@ -33,7 +33,6 @@ constexpr int NT_UPD = NT_SIM - 32;      // threads of the cache-update group (w
 constexpr int CTL = NT_SIM - 32;         // the control thread (lane 0 of warp 7)
 constexpr int FTAB_MAX = 1024;           // f(n) tabulated for n < FTAB_MAX
 constexpr int PROBE_CAP = SIM_PROBE_CAP;   // W * nb up to which the probe captures every slot
-constexpr int PROBE_ILP = 2;             // lookups a thread keeps in flight
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -673,13 +672,13 @@ __device__ __forceinline__ void probe_prefixes(SimCtx& c, const uint64_t* hbuf, 
 }
 
 // The same m_j with every (worker, block) pair looked up at once (W nb <=
-// PROBE_CAP): each thread issues the first-bucket loads of PROBE_ILP pairs
+// PROBE_CAP): each thread issues the first-bucket loads of ILP pairs
 // before resolving them, and the slot found (or the first free slot of the
 // probe path) is kept for the chosen worker's update.
 // TIER: m_j counts the leading blocks in G1 (a found slot's stamp at or
 // past the worker's b1); every pair's tier goes to ptier; the absent count
 // is of blocks in no tier.
-template <int NT, bool TIER = false>
+template <int NT, int ILP, bool TIER = false>
 __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int nb) {
   SimScalars& S = *c.S;
   const int W = c.L->mc.W;
@@ -690,15 +689,15 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
   // error stays far below that, so it truncates to the quotient exactly
   const float inv_nb = nb > 0 ? 1.0f / (float)nb : 0.0f;
   int err = 0;
-  for (int base = 0; base < total; base += NT * PROBE_ILP) {   // uniform
-    int jj[PROBE_ILP], kk[PROBE_ILP];
-    uint64_t hh[PROBE_ILP], v[PROBE_ILP][BUCKET];
-    uint64_t stw[PROBE_ILP][TIER ? 4 : 1];   // tiers: the home bucket's 8 stamps, beside its keys
-    uint32_t bk[PROBE_ILP];
+  for (int base = 0; base < total; base += NT * ILP) {   // uniform
+    int jj[ILP], kk[ILP];
+    uint64_t hh[ILP], v[ILP][BUCKET];
+    uint64_t stw[ILP][TIER ? 4 : 1];   // tiers: the home bucket's 8 stamps, beside its keys
+    uint32_t bk[ILP];
     // every pair's home bucket requested before any is resolved; a thread
     // past the pairs repeats the last one (in bounds, unused)
 #pragma unroll
-    for (int r = 0; r < PROBE_ILP; r++) {
+    for (int r = 0; r < ILP; r++) {
       const int it0 = base + r * NT + (int)threadIdx.x;
       const int it = it0 < total ? it0 : total - 1;
       const int j = (int)(((float)it + 0.5f) * inv_nb);
@@ -712,10 +711,10 @@ __device__ __forceinline__ void probe_full(SimCtx& c, const uint64_t* hbuf, int 
         ld_keys4(reinterpret_cast<const uint64_t*>(t.stamp + (size_t)BUCKET * bk[r]), stw[r][0],
                  stw[r][TIER ? 1 : 0], stw[r][TIER ? 2 : 0], stw[r][TIER ? 3 : 0]);
     }
-    uint32_t sl[PROBE_ILP], fr[PROBE_ILP];
-    resolve_buckets<PROBE_ILP>(c, v, bk, hh, jj, sl, fr, &err);
+    uint32_t sl[ILP], fr[ILP];
+    resolve_buckets<ILP>(c, v, bk, hh, jj, sl, fr, &err);
 #pragma unroll
-    for (int r = 0; r < PROBE_ILP; r++) {
+    for (int r = 0; r < ILP; r++) {
       const int it = base + r * NT + (int)threadIdx.x;
       bool miss = false, absent = false;
       if (jj[r] >= 0) {
@@ -1106,6 +1105,7 @@ template <int MINB, bool SG, int MODE>
 __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict__ descs, SimBuffers b,
                                                 SimLaunch L) {
   constexpr bool FREQ = MODE == SIM_FREQ, TIER = MODE == SIM_TIER;
+  constexpr int PROBE_FULL_ILP = 2;   // lookups a thread of the full probe keeps in flight
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ SimScalars S;
   const int sid = blockIdx.x;
@@ -1241,7 +1241,7 @@ __global__ void __launch_bounds__(NT_SIM, MINB) k_sim(const SimDesc* __restrict_
     if (warp < NT_SIM / 32 - 1) {
       // ---- cached prefix on every worker (warps 0-6)
       if (full) {
-        probe_full<NT_UPD, TIER>(c, hb, nb);
+        probe_full<NT_UPD, PROBE_FULL_ILP, TIER>(c, hb, nb);
       } else if (TIER) {   // the tiers need every pair's slot (the host checks W nb)
         if (threadIdx.x == 0) S.status = RS_ERR_CAPACITY;
       } else {
