@@ -191,10 +191,10 @@ def _table_bytes(K: int) -> int:
 # the simulation kernel's sources it was taken with; None until such a
 # capture exists for these sources.  The full grid holds about 103 GB of
 # cache tables, so the capture ran on 304 of its 8192 simulations (one
-# resident wave, two per SM, 10 000 requests each: 236.93 GB) and is scaled by
+# resident wave, two per SM, 10 000 requests each: 234.69 GB) and is scaled by
 # 8192 / 304; every simulation's tables and requests are of the same kind.
-SIM_TRAFFIC = {"bytes": 236932571904 * 8192 / 304,
-               "sources_sha256": "11078cb6a316e279fdc61f5fa6fe6a749dca50ee076998290241ed3f4442738d",
+SIM_TRAFFIC = {"bytes": 234692720384 * 8192 / 304,
+               "sources_sha256": "188fdf42bea8a811467ab449087524e9d353034642b819cda337c020b3f84b3f",
                "summary": "profiles/k_sim_grid.md",
                "scaled_from": "304 simulations x 10 000 requests, times 8192 / 304"}
 

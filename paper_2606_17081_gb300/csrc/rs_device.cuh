@@ -346,10 +346,29 @@ constexpr uint32_t FREE_TOMB = 0x80000000u;
 // Resolves one loaded bucket: returns 1 (found, *slot set), 0 (absent: the
 // bucket holds an EMPTY key) or -1 (continue with the next bucket).  *fr, if
 // still SLOT_NONE, becomes the bucket's first EMPTY or TOMB slot before the
-// match (before the end when h is absent).  Branch-free: the eight keys give
-// three bit masks, so the lanes of a warp never diverge on where h sits.
+// match (before the end when h is absent).
 __device__ __forceinline__ int bucket_scan(const uint64_t (&v)[BUCKET], uint32_t b, uint64_t h,
                                            uint32_t* slot, uint32_t* fr) {
+  bool empty = false;
+#pragma unroll
+  for (int q = 0; q < BUCKET; q++) {
+    if (v[q] == h) {
+      *slot = (uint32_t)BUCKET * b + q;
+      return 1;
+    }
+    if (v[q] < 2 && *fr == SLOT_NONE)
+      *fr = ((uint32_t)BUCKET * b + q) | (v[q] == KEY_TOMB ? FREE_TOMB : 0u);
+    empty |= v[q] == KEY_EMPTY;
+  }
+  return empty ? 0 : -1;
+}
+
+// bucket_scan without branches: the eight keys give three bit masks, so the
+// lanes of a warp never diverge on where h sits (the simulation's probes,
+// which keep several buckets in flight per thread; a one-lookup-at-a-time
+// walk is better served by the early exit above).
+__device__ __forceinline__ int bucket_scan_masks(const uint64_t (&v)[BUCKET], uint32_t b,
+                                                 uint64_t h, uint32_t* slot, uint32_t* fr) {
   unsigned hit = 0, fre = 0, tomb = 0;
 #pragma unroll
   for (int q = 0; q < BUCKET; q++) {

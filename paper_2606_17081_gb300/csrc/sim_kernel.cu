@@ -573,7 +573,7 @@ __device__ __forceinline__ void resolve_buckets(const SimCtx& c, const uint64_t 
   for (int r = 0; r < ILP; r++) {
     sl[r] = SLOT_NONE;
     fr[r] = SLOT_NONE;
-    cont[r] = bucket_scan(v[r], bk[r], hh[r], &sl[r], &fr[r]) < 0 && jj[r] >= 0;
+    cont[r] = bucket_scan_masks(v[r], bk[r], hh[r], &sl[r], &fr[r]) < 0 && jj[r] >= 0;
     any |= cont[r];
   }
   if (any) {
