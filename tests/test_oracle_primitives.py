@@ -3,13 +3,14 @@
 - SplitMix64 finalizer: the published SplitMix64 generator seeded with 0
   returns 0xE220A8397B1DCDAF as its first output (state 0x9E3779B97F4A7C15).
 - Philox4x32-10: the known-answer vectors distributed with Random123
-  (Salmon et al., SC 2011).
+  (Salmon et al., SC 2011), read from tests/golden/philox4x32_10_kat.txt.
 - exp: accuracy against numpy's float64 exp (<= 1 ulp of float32).
 - Worker selection, Eq. (2): argmin with lowest-index ties; the softmax draw
   against Eq. (2) probabilities computed here with numpy; tau limits (§4.3).
 - Nearest-rank P99 against numpy's inverted-CDF percentile.
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -28,12 +29,19 @@ def test_mix64_is_a_bijection_on_samples():
     assert len(ys) == len(set(xs))
 
 
-@pytest.mark.parametrize("ctr,key,expect", [
-    ((0, 0, 0, 0), (0, 0), (0x6627E8D5, 0xE169C58D, 0xBC57AC4C, 0x9B00DBD8)),
-    ((0xFFFFFFFF,) * 4, (0xFFFFFFFF,) * 2, (0x408F276D, 0x41C83B0E, 0xA20BC7C6, 0x6D5451FD)),
-    ((0x243F6A88, 0x85A308D3, 0x13198A2E, 0x03707344), (0xA4093822, 0x299F31D0),
-     (0xD16CFE09, 0x94FDCCEB, 0x5001E420, 0x24126EA1)),
-])
+def _philox_kat():
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden",
+                        "philox4x32_10_kat.txt")
+    out = []
+    with open(path) as fh:
+        for ln in fh:
+            if ln.strip() and not ln.startswith("#"):
+                v = [int(x, 16) for x in ln.split()]
+                out.append((tuple(v[0:4]), tuple(v[4:6]), tuple(v[6:10])))
+    return out
+
+
+@pytest.mark.parametrize("ctr,key,expect", _philox_kat())
 def test_philox_known_answers(ctr, key, expect):
     assert O.philox4x32_10(ctr, key) == expect
 
