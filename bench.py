@@ -726,7 +726,7 @@ def run_reference(args):
                 "d2h_bytes_per_step": 0}}))
 
 
-def main():
+def arg_parser() -> argparse.ArgumentParser:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
@@ -750,7 +750,11 @@ def main():
     ap.add_argument("--probe-cache-blocks", type=int, default=None,
                     help="cache blocks per worker of the batch-probe instance "
                          "(default: the W = 64 workload's 2^20)")
-    args = ap.parse_args()
+    return ap
+
+
+def main():
+    args = arg_parser().parse_args()
     if args.impl == "reference":
         run_reference(args)
     else:

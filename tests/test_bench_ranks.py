@@ -95,3 +95,24 @@ def test_profiling_subsets():
     assert sorted({full.replicas[k].trace for k in idx}) == list(range(len(full.trace_seeds)))
     p, lo, hi = bench._plan("grid", n_req=50, subset="per-trace")
     assert (lo, hi) == (0, len(idx)) and len(p.trace_seeds) == len(idx)
+
+
+def test_profile_commands_are_bench_options():
+    # every bench command a profile summary gives parses with the bench's
+    # own options, and its replica subset selects replicas of the plan
+    import glob
+    import re
+    import shlex
+    import bench
+    from paper_2606_17081_gb300 import workloads as wk
+    cmds = []
+    for md in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
+        text = open(md).read().replace("\\\n", " ")
+        cmds += [m.group(1) for m in re.finditer(r"python bench\.py([^\n]*)", text)]
+    assert cmds
+    for cmd in cmds:
+        args = bench.arg_parser().parse_args(shlex.split(cmd))
+        if args.replicas is not None:
+            full = wk.plan(args.workload, n_req=50)
+            idx = bench._subset(full, args.replicas)
+            assert idx and max(idx) < len(full.replicas)
